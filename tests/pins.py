@@ -1,0 +1,272 @@
+"""Pins for the CPU oracle: checks against facts that do not come from the oracle.
+
+Each ``check_*`` takes an :class:`oracle.OracleLib` and raises AssertionError on
+a mismatch.  They are run on the real oracle (``test_oracle_pins.py``) and on
+deliberately broken copies of it (``test_oracle_mutants.py``) to show that a
+plausible slip in the oracle fails at least one of them.
+
+Sources of truth:
+* hand-worked examples (``golden/hand_examples.json``), worked out from the
+  model's rules (§2.1, Factor A/B of §2.3, Table 1 caption);
+* closed forms: serial chains, identical fan-outs, the all-cpu critical path;
+* a textbook special case: with no contention, no gpu_queue and no VRAM
+  pressure every makespan is the longest path of the DAG under per-mode
+  durations (critical-path DP);
+* invariants: the argmin is feasible and no worse than all-cpu; a fan-out from
+  t=0 is infeasible exactly when its gpu_now footprints exceed M; contention
+  never shortens a feasible mapping without gpu_queue;
+* the paper's printed numbers: Table 1 speedups (gpu_now = GPU time, queued =
+  GPU + Load), Table 3 totals and feasibility (§4.4, §4.5), Figure 7's
+  per-probe memory and status;
+* a structurally different Python restatement (``oracle.pysim``) on every
+  mapping of small random DAGs, and the exact rational model
+  (``oracle.exact``) within its rounding bound.
+"""
+from __future__ import annotations
+
+import json
+import math
+import os
+
+import numpy as np
+
+from paper_2607_22242_gb300 import scenarios as S
+from paper_2607_22242_gb300.scenarios import CPU, GPU_NOW, GPU_QUEUE, Scenario
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+INF = 0xFFFFFFFF
+MODE_OF = {"cpu": CPU, "gpu_now": GPU_NOW, "gpu_queue": GPU_QUEUE}
+
+
+def _load(name):
+    with open(os.path.join(GOLDEN, name)) as fh:
+        return json.load(fh)
+
+
+def _chain(n, c, g, x, l, m, budget, f):
+    return Scenario(n, [0] + [1 << (i - 1) for i in range(1, n)], c, g, x, l, m, budget, f)
+
+
+def _longest_path(scn, dur):
+    """Critical-path length: finish[v] = dur[v] + max(finish[u] for u in pred(v))."""
+    finish = []
+    for v in range(scn.n):
+        start = max([finish[u] for u in range(v) if (scn.pred_mask[v] >> u) & 1], default=0)
+        finish.append(start + dur[v])
+    return max(finish)
+
+
+# ---------------------------------------------------------------------------
+
+def check_hand_examples(lib):
+    for ex in _load("hand_examples.json")["examples"]:
+        scn = Scenario.from_dict(ex["scenario"])
+        for idx, want in ex["expected"].items():
+            got = lib.evaluate(scn, int(idx))
+            assert got == want, f"{ex['name']}: idx {idx}: {got} != {want}"
+        if "argmin" in ex:
+            assert list(lib.search(scn)) == ex["argmin"], ex["name"]
+
+
+def check_chain_closed_forms(lib, trials=40, seed=11):
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 9))
+        c = [int(v) for v in rng.integers(1, 100000, n)]
+        g = [int(v) for v in rng.integers(1, 100000, n)]
+        x = [int(v) for v in rng.integers(0, 30000, n)]
+        l = [int(v) for v in rng.integers(0, 50000, n)]
+        m = [int(v) for v in rng.integers(1, 5000, n)]
+        f = S.random_small(rng, 2).slowdown_q10  # any table: a chain never runs two GPU tools
+        scn = _chain(n, c, g, x, l, m, max(m), f)
+        all_now = sum(3 ** i for i in range(n))
+        assert lib.evaluate(scn, 0) == sum(c)
+        assert lib.evaluate(scn, all_now) == sum(g) + sum(x)
+        assert lib.evaluate(scn, 2 * all_now) == sum(l) + sum(g) + sum(x)
+        # any mixed mapping of a chain: the sum of per-mode durations
+        for idx in rng.integers(0, 3 ** n, 8):
+            modes = S.mapping_modes(int(idx), n)
+            dur = [(c[i], g[i] + x[i], l[i] + g[i] + x[i])[a] for i, a in enumerate(modes)]
+            assert lib.evaluate(scn, int(idx)) == sum(dur)
+        # a tool larger than the budget: gpu_now or gpu_queue on it is infeasible
+        big = Scenario(n, scn.pred_mask, c, g, x, l, [max(m) + 1] + m[1:], max(m), f)
+        assert lib.evaluate(big, 1) == INF and lib.evaluate(big, 2) == INF
+
+
+def check_identical_fanout(lib, seed=12):
+    rng = np.random.default_rng(seed)
+    for n in range(1, 13):
+        w = int(rng.integers(1, 200000))
+        f = S.slowdown_linear(int(rng.integers(0, 80)))
+        scn = Scenario(n, [0] * n, [10 ** 7] * n, [w] * n, [0] * n, [0] * n, [1] * n, n, f)
+        all_now = sum(3 ** i for i in range(n))
+        want = -(-w * f[n] // 1024)  # ceil(w * f[n] / 1024)
+        assert lib.evaluate(scn, all_now) == want, (n, w, f[n])
+
+
+def check_longest_path(lib, trials=30, seed=13):
+    """No contention, no queue, no VRAM pressure: every makespan is a critical path."""
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 8))
+        scn = S.random_small(rng, n, tight=False, contention=False, max_time=1000)
+        ms, fe = lib.eval_range(scn, 0, 3 ** n)
+        for idx in range(3 ** n):
+            modes = S.mapping_modes(idx, n)
+            if GPU_QUEUE in modes:
+                continue
+            dur = [scn.cpu_us[i] if a == CPU else scn.gpu_us[i] + scn.xfer_us[i] for i, a in enumerate(modes)]
+            assert fe[idx] == 1 and int(ms[idx]) == _longest_path(scn, dur), (scn, idx)
+
+
+def check_all_cpu_is_critical_path(lib, trials=40, seed=14):
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 12))
+        scn = S.random_small(rng, n, tight=True, max_time=500)
+        assert lib.evaluate(scn, 0) == _longest_path(scn, scn.cpu_us)
+
+
+def check_argmin_invariants(lib, trials=40, seed=15):
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 7))
+        scn = S.random_small(rng, n)
+        ms, fe = lib.eval_range(scn, 0, 3 ** n)
+        idx, best = lib.search(scn)
+        assert fe[0] == 1 and fe[idx] == 1
+        assert best == int(ms[idx]) <= int(ms[0])
+        feas = np.flatnonzero(fe)
+        assert best == int(ms[feas].min())
+        assert idx == int(feas[np.argmax(ms[feas] == best)])  # lowest index among ties
+        assert np.all(ms[fe == 0] == INF)
+
+
+def check_fanout_feasibility(lib, trials=40, seed=16):
+    """Fan-out from t=0 with every footprint <= M: infeasible iff sum(gpu_now m) > M."""
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 7))
+        base = S.random_small(rng, n, edge_p=0.0)
+        budget = int(rng.integers(max(base.vram_mib), 3 * max(base.vram_mib) + 1))
+        scn = Scenario(n, [0] * n, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us,
+                       base.vram_mib, budget, base.slowdown_q10)
+        ms, fe = lib.eval_range(scn, 0, 3 ** n)
+        for idx in range(3 ** n):
+            modes = S.mapping_modes(idx, n)
+            now_mem = sum(scn.vram_mib[i] for i, a in enumerate(modes) if a == GPU_NOW)
+            assert bool(fe[idx]) == (now_mem <= budget), (scn, idx)
+
+
+def check_contention_monotone(lib, trials=40, seed=17):
+    """Without gpu_queue, a mapping feasible with and without contention is never faster with it."""
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 7))
+        scn = S.random_small(rng, n, max_time=int(rng.choice([20, 500])))
+        flat = Scenario(**{**scn.to_dict(), "slowdown_q10": S.slowdown_flat()})
+        ms_f, fe_f = lib.eval_range(scn, 0, 3 ** n)
+        ms_1, fe_1 = lib.eval_range(flat, 0, 3 ** n)
+        for idx in range(3 ** n):
+            if GPU_QUEUE in S.mapping_modes(idx, n) or not (fe_f[idx] and fe_1[idx]):
+                continue
+            assert ms_f[idx] >= ms_1[idx], (scn, idx)
+
+
+def check_against_pysim(lib, trials=120, seed=18):
+    from oracle import pysim
+    rng = np.random.default_rng(seed)
+    for t in range(trials):
+        n = int(rng.integers(1, 6 if t % 4 else 7))
+        scn = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.3, 0.7])),
+                             tight=bool(t % 3), contention=bool(t % 5),
+                             max_time=int(rng.choice([6, 30, 2000])))
+        ms, fe = lib.eval_range(scn, 0, 3 ** n)
+        for idx in range(3 ** n):
+            want, ok = pysim.evaluate(scn, idx)
+            assert (int(ms[idx]), bool(fe[idx])) == (want if ok else INF, ok), (scn, idx)
+
+
+def check_rational_bound(lib, trials=60, seed=19):
+    """Mappings without gpu_queue whose feasibility agrees: |integer - exact| <= 2N*ceil(f[N]/1024)."""
+    from oracle import exact
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 6))
+        scn = S.random_small(rng, n, max_time=int(rng.choice([10, 1000])))
+        ms, fe = lib.eval_range(scn, 0, 3 ** n)
+        bound = 2 * n * math.ceil(scn.slowdown_q10[n] / 1024)
+        for idx in range(3 ** n):
+            modes = S.mapping_modes(idx, n)
+            if GPU_QUEUE in modes:
+                continue
+            t, ok, _ = exact.simulate(scn, modes)
+            if ok != bool(fe[idx]) or not ok:
+                continue
+            assert abs(int(ms[idx]) - t) <= bound, (scn, idx, int(ms[idx]), float(t))
+
+
+# ---------------------------------------------------------------------------
+# The paper's printed numbers.
+# ---------------------------------------------------------------------------
+
+def _one_tool(cpu_ms, gpu_ms, load_ms, vram):
+    us = lambda v: int(round(v * 1000))
+    return Scenario(1, [0], [us(cpu_ms)], [us(gpu_ms)], [0], [us(load_ms)], [vram], vram, S.slowdown_flat())
+
+
+def _printed_close(value, printed):
+    if printed.startswith("<"):
+        return value < float(printed[1:])
+    decimals = len(printed.split(".")[1]) if "." in printed else 0
+    return abs(value - float(printed)) <= 10.0 ** (-decimals) + 1e-12
+
+
+def check_table1_speedups(lib):
+    """Table 1: CPU/GPU speedup from the cpu and gpu_now runs, CPU/(GPU+Load) from the queued run."""
+    for t in _load("paper_table1.json")["tools"]:
+        if t["vram_mb"] is None:
+            continue
+        scn = _one_tool(t["cpu_ms"], t["gpu_ms"], t["load_ms"], t["vram_mb"])
+        cpu, now, queued = (lib.evaluate(scn, i) for i in range(3))
+        assert _printed_close(cpu / now, t["speedup"]), (t["tool"], cpu / now)
+        assert _printed_close(cpu / queued, t["queue_speedup"]), (t["tool"], cpu / queued)
+
+
+def _fanout(tools, budget):
+    n = len(tools)
+    us = lambda v: int(round(v * 1000))
+    return Scenario(n, [0] * n, [us(t["cpu_ms"]) for t in tools], [us(t["gpu_ms"]) for t in tools],
+                    [0] * n, [us(t["load_ms"]) for t in tools], [t["vram_mb"] for t in tools],
+                    budget, S.slowdown_linear())
+
+
+def check_table3_feasibility(lib):
+    tools = {t["tool"]: t for t in _load("paper_table1.json")["tools"]}
+    t3 = _load("paper_table3.json")
+    by_id = {s["id"]: s for s in t3["scenarios"]}
+    for case in t3["feasibility"]["cases"]:
+        sc = by_id[case["scenario"]]
+        scn = _fanout([tools[name] for name in sc["tools"]], sc["budget"])
+        idx = S.mapping_index([MODE_OF[m] for m in case["modes"]])
+        assert (lib.evaluate(scn, idx) != INF) == case["feasible"], case
+
+
+def check_fig7_probes(lib):
+    """Figure 7: status of every probe; printed memory = gpu_now footprints within 2 MB."""
+    f7 = _load("paper_fig7.json")
+    tools = [dict(cpu_ms=t["cpu"], gpu_ms=t["gpu"], load_ms=t["load"], vram_mb=t["mem"]) for t in f7["tools"]]
+    for p in f7["probes"]:
+        idx = S.mapping_index([MODE_OF[m] for m in p["modes"]])
+        assert (lib.evaluate(_fanout(tools, f7["budget_mb"]), idx) != INF) == p["feasible"], p
+        # the memory the probe holds at once lies in [mem-2, mem+2]
+        assert lib.evaluate(_fanout(tools, p["mem"] + 2), idx) != INF, p
+        assert lib.evaluate(_fanout(tools, p["mem"] - 3), idx) == INF, p
+
+
+ALL_CHECKS = [
+    check_hand_examples, check_chain_closed_forms, check_identical_fanout, check_longest_path,
+    check_all_cpu_is_critical_path, check_argmin_invariants, check_fanout_feasibility,
+    check_contention_monotone, check_against_pysim, check_rational_bound,
+    check_table1_speedups, check_table3_feasibility, check_fig7_probes,
+]
