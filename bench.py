@@ -1,0 +1,296 @@
+#!/usr/bin/env python3
+"""Benchmark: brute-force optimal device-mapping search on GB300.
+
+One step = one full search of the N=19 workload (scenarios.config3(): a spine
+plus two fan-outs, tools from all four scheduling zones of §2.2, 32 GiB VRAM
+budget, contention f[k] = 1 + 0.35(k-1)): all 3^19 = 1,162,261,467 mappings
+enumerated, simulated and reduced to the argmin in one bf_search_best call.
+
+Prints ONE JSON line (rank 0).  Metric: mappings evaluated per second (whole
+job).  Also reported: the per-step wall time to the optimum, the kernel's
+integer-issue roofline, the oracle timed on the host cores on a bounded sample
+(cpu_baseline), and the end-to-end rate through the host-buffer API (create
+scenario from host tables, search, result back on the host, release).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl bf|reference]
+
+With --impl reference the CPU oracle is timed instead (rank 0 only), on
+bounded samples of the same workload.  Under torchrun each rank searches the
+same scenario independently (replicas, no collective on the data path); the
+step time is the max over ranks.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "mappings evaluated/sec on 1 GB300; wall time to optimum at N=19; % of issue peak"
+UNIT = "mappings/s"
+WORKLOAD = ("config3: N=19 tools (spine of 7 + two fan-outs of 6; 11 GPU-preferred, 4 ambiguous, "
+            "1 CPU-preferred, 3 neutral), 32 GiB VRAM budget, f[k]=1+0.35(k-1), seed 3; full 3^19 search")
+# Algorithmic integer operations per simulated mapping: N events, each with an
+# N-wide next-completion scan and an N-wide readiness scan (2 N^2).
+N_TOOLS = 19
+OPS_PER_MAPPING = 2 * N_TOOLS * N_TOOLS
+INT_LANES_PER_SM = 128  # 4 SMSPs x 32 lanes issue one integer op each per clock
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", str(rank)))
+    return rank, world, local
+
+
+def emit(obj):
+    print(json.dumps(obj), flush=True)
+
+
+# --------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi samples every 200 ms while the timed region runs."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_id: str):
+        self.device_id = device_id
+        self.proc = None
+        self.lines = []
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "200",
+                 "-i", self.device_id], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.thread = threading.Thread(target=self._read, daemon=True)
+            self.thread.start()
+            time.sleep(0.3)
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.thread.join(timeout=2)
+
+    def summary(self):
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in self.lines:
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for name, val in zip(names, parts[5:9]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def device_id_for_smi(torch, dev: int) -> str:
+    try:
+        return "GPU-" + str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        return str(dev)
+
+
+# --------------------------------------------------------------------------- CPU oracle timing
+
+def oracle_sample_time(scn, budget_mappings: int, threads: int):
+    """Time the oracle on `budget_mappings` indices in 16 evenly spaced contiguous chunks."""
+    import oracle
+    total = 3 ** scn.n
+    chunks = 16
+    per = budget_mappings // chunks
+    t0 = time.perf_counter()
+    for c in range(chunks):
+        oracle.search_range(scn, (total // chunks) * c, per, threads)
+    dt = time.perf_counter() - t0
+    return per * chunks, dt
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return 0
+    import oracle
+    from paper_2607_22242_gb300 import scenarios as S
+    oracle.build()
+    scn = S.config3()
+    threads = oracle.default_threads()
+    per_step = args.ref_sample
+    for _ in range(args.warmup):
+        oracle_sample_time(scn, per_step, threads)
+    times = []
+    for _ in range(args.steps):
+        n, dt = oracle_sample_time(scn, per_step, threads)
+        times.append(dt)
+    ms = 1e3 * statistics.mean(times)
+    value = per_step / (ms / 1e3)
+    sample = (f"{per_step} mappings per step: 16 contiguous chunks spread evenly over [0, 3^19), "
+              f"oracle search over {threads} host threads")
+    emit({"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+          "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+          "scaling": "weak", "vs_baseline": None, "dtype": "u64", "data": "synthetic",
+          "config": {"workload": WORKLOAD, "mappings_per_step": per_step},
+          "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "kind": "oracle", "sample": sample},
+          "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}})
+    return 0
+
+
+# --------------------------------------------------------------------------- GPU arm
+
+def run_gpu(args):
+    import torch
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    else:
+        torch.cuda.set_device(0)
+    dev = torch.cuda.current_device()
+
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_22242_gb300 import bf
+    from paper_2607_22242_gb300 import scenarios as S
+
+    scn = S.config3()
+    total = 3 ** scn.n
+    stream = torch.cuda.current_stream()
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device="cuda")  # > 129 MB L2
+
+    def barrier():
+        if world > 1:
+            torch.distributed.barrier()
+        torch.cuda.synchronize()
+
+    h = bf.create_scenario(scn)
+    for _ in range(args.warmup):
+        res = bf.search_best(h, stream)
+
+    # ---- timed region: K full searches, L2 flushed between them -------------
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(device_id_for_smi(torch, dev))
+    with sampler:
+        barrier()
+        wall0 = time.perf_counter()
+        for i in range(args.steps):
+            flush.zero_()
+            starts[i].record(stream)
+            res = bf.search_best(h, stream)
+            ends[i].record(stream)
+        barrier()
+        wall = time.perf_counter() - wall0
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    mean_ms = statistics.mean(step_ms)
+    worst_ms = mean_ms
+    if world > 1:
+        t = torch.tensor([mean_ms], device="cuda")
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        worst_ms = float(t.item())
+    value = world * total / (worst_ms / 1e3)
+    clocks = sampler.summary()
+
+    # ---- end to end through the host-buffer API ------------------------------
+    e2e_times = []
+    barrier()
+    for _ in range(max(3, args.steps // 4)):
+        t0 = time.perf_counter()
+        with bf.create_scenario(scn) as h2:       # host tables in, validated, scratch allocated
+            r2 = bf.search_best(h2, stream)       # tables travel with the launch; 8-byte key back
+        e2e_times.append(time.perf_counter() - t0)
+        assert (r2.index, r2.makespan_us) == (res.index, res.makespan_us)
+    e2e_value = world * total / statistics.mean(e2e_times)
+    h.close()
+
+    if rank != 0:
+        torch.distributed.destroy_process_group()
+        return 0
+
+    sm_count = torch.cuda.get_device_properties(dev).multi_processor_count
+    clk_mhz = clocks["sm_mhz"] or 2070.0
+    peak_ops = sm_count * INT_LANES_PER_SM * clk_mhz * 1e6
+    achieved_ops = OPS_PER_MAPPING * total / (mean_ms / 1e3)
+    roofline = {"bound": "alu", "achieved": achieved_ops / 1e12, "peak": peak_ops / 1e12, "unit": "Tops/s",
+                "frac": achieved_ops / peak_ops, "traffic": None,
+                "peak_basis": f"{sm_count} SMs x {INT_LANES_PER_SM} int lanes x "
+                              f"{clk_mhz:.0f} MHz ({'sampled median under load' if clocks['sm_mhz'] else 'max clock, no samples'})",
+                "ops_per_mapping": OPS_PER_MAPPING}
+
+    out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+           "warmup": args.warmup, "ms_per_step": mean_ms, "higher_is_better": True, "scaling": "weak",
+           "vs_baseline": None, "dtype": "u32", "data": "synthetic",
+           "config": {"workload": WORKLOAD, "mappings_per_step": total, "parallelism": f"replicas x{world}",
+                      "l2": "flushed between steps (256 MiB write, outside the timed events)"},
+           "wall_time_to_optimum_ms": {"median": statistics.median(step_ms), "min": min(step_ms),
+                                       "max": max(step_ms)},
+           "result": {"index": res.index, "makespan_us": res.makespan_us, "modes": res.modes},
+           "roofline": roofline,
+           "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 572, "d2h_bytes_per_step": 8,
+                   "path": "bf_create_scenario(host desc) + bf_search_best + bf_destroy_scenario"},
+           "gpu_launches": args.steps,
+           "clocks": clocks, "timed_wall_s": wall, "sm_count": sm_count}
+    if world == 1 and not args.no_cpu_baseline:
+        import oracle
+        oracle.build()
+        threads = oracle.default_threads()
+        n, dt = oracle_sample_time(scn, args.cpu_sample, threads)
+        out["cpu_baseline"] = {"value": n / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+                               "sample": f"{n} mappings of the same workload in 16 contiguous chunks spread "
+                                         f"evenly over [0, 3^19), oracle search, {dt:.1f} s"}
+    emit(out)
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=("bf", "reference"), default="bf")
+    ap.add_argument("--cpu-sample", type=int, default=1 << 25, help="mappings for the oracle CPU baseline")
+    ap.add_argument("--ref-sample", type=int, default=1 << 23, help="mappings per --impl reference step")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,169 @@
+/*
+ * bf.h -- C ABI of the brute-force optimal device-mapping search (libbf.so).
+ *
+ * The problem (§2.1 of "Agentic CPU-GPU Scheduling for Heterogeneous AI
+ * Workloads"): a workflow is a DAG G=(V,E) of N tool invocations; each tool v
+ * is mapped to a mode a_v in {cpu, gpu_now, gpu_queue}; a mapping is feasible
+ * only if the VRAM of the GPU tools running at any instant stays within the
+ * budget M; its end-to-end latency T_e2e is the largest completion time over
+ * the sinks.  The brute-force oracle the paper grades its scheduler against
+ * (§2.3, §4.1) is the feasible mapping of lowest T_e2e among all 3^N.
+ *
+ * The paper measures T_e2e on hardware.  This library evaluates it under a
+ * fixed integer latency model (version 1), exact to the microsecond:
+ *
+ *   - Times are integer microseconds.  GPU progress is a virtual clock V in
+ *     1/1024 isolated-microsecond units; a GPU tool of isolated time w that
+ *     starts at V ends when V reaches V + 1024*w.
+ *   - GPU contention (Factor A, §2.3): while k GPU tools run, each runs at
+ *     1024/f[k] of its isolated speed (processor sharing).  CPU tools are
+ *     unaffected; CPU cores are unlimited.
+ *   - cpu: duration c.  gpu_now: isolated work g + x (Table 1's GPU time
+ *     includes PCIe transfer), starts when its predecessors are done, holds
+ *     its VRAM m while running; a start that brings live VRAM above M makes
+ *     the mapping infeasible (out of memory, Factor B).  gpu_queue: waits in
+ *     one serialised FIFO queue (ready time, then index) without holding VRAM;
+ *     the head starts when no queued tool is running and live VRAM + m <= M;
+ *     isolated work l + g + x (Table 1's gpu_queue column = GPU + Load).  A
+ *     queued tool with m > M can never start: infeasible.  No bypass.
+ *   - Event loop: next CPU completion vs next GPU completion
+ *     T + ceil((Vmin - V) * f[k] / 2^20); if a CPU tool ends first, V advances
+ *     by floor((t_cpu - T) * 2^20 / f[k]).  At each event every tool ending at
+ *     that instant retires (freeing VRAM), then newly ready tools start in
+ *     index order, then the queue head is tried.  Makespan = time of the last
+ *     retirement; infeasible mappings have makespan 0xFFFFFFFF.
+ *
+ * Mapping index: idx = sum_i a_i * 3^i, a_i in {0=cpu, 1=gpu_now,
+ * 2=gpu_queue}; tool 0 is the least-significant digit.  Searches return the
+ * feasible mapping of lowest makespan, ties to the lowest index.  The all-cpu
+ * mapping (index 0) is always feasible, so a full search always succeeds.
+ *
+ * Conventions for every entry point:
+ *   - Return 0 (BF_OK) or a BF_E* status; bf_last_error() then describes the
+ *     failure (thread-local string owned by the library, valid until the next
+ *     call on that thread).  Outputs are written only on BF_OK.
+ *   - Host pointers are caller-owned and only read during the call (inputs are
+ *     copied).  Device pointers are caller-owned CUDA device memory on the
+ *     current device.  `cuda_stream` is a cudaStream_t (NULL = legacy default
+ *     stream); work is ordered on it.
+ *   - Blocking calls wait with a time limit (bf_set_wait_timeout_ms) and
+ *     return BF_ETIMEOUT if it passes; the GPU work is then still in flight,
+ *     and the scenario must not be destroyed until the stream has finished.
+ */
+#ifndef BF_H_
+#define BF_H_
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BF_MAX_TOOLS 20
+
+enum bf_status {
+  BF_OK = 0,
+  BF_EINVAL = 1,    /* invalid argument or scenario */
+  BF_ERANGE = 2,    /* index range outside [0, 3^n) */
+  BF_ENOMEM = 3,    /* device or pinned-host allocation failed */
+  BF_ECUDA = 4,     /* a CUDA runtime call failed (message names it) */
+  BF_ETIMEOUT = 5   /* a blocking wait exceeded its time limit */
+};
+
+enum bf_mode { BF_MODE_CPU = 0, BF_MODE_GPU_NOW = 1, BF_MODE_GPU_QUEUE = 2 };
+
+/*
+ * One workflow (§2.1) with the per-tool profile of Table 1 / §3.1 plus a
+ * transfer time.  Tools are numbered 0..n-1 in a topological order.
+ * Validity (checked by every entry point that takes a desc):
+ *   1 <= n <= 20; pred_mask[v] has bits only below v (u < v) and below n;
+ *   cpu_us >= 1, gpu_us >= 1; load_us + gpu_us + xfer_us < 2^22;
+ *   vram_mib <= 2^27, vram_budget_mib <= 2^31;
+ *   slowdown_q10[1] == 1024, slowdown_q10[k] non-decreasing and <= 65536 for
+ *   k = 1..n (entries 0 and > n are ignored);
+ *   the makespan bound sum_i max(c_i, floor((l_i+g_i+x_i)*f[n]/1024) + n + 1)
+ *   is <= 0xFFFFFFFD, so every makespan fits in 32 bits.
+ * Entries at index >= n are ignored.
+ */
+typedef struct bf_scenario_desc {
+  uint32_t n;                               /* number of tools, 1..20 */
+  uint32_t pred_mask[BF_MAX_TOOLS];         /* bit u of pred_mask[v] <=> edge u->v */
+  uint32_t cpu_us[BF_MAX_TOOLS];            /* c_i: CPU latency, us */
+  uint32_t gpu_us[BF_MAX_TOOLS];            /* g_i: isolated GPU latency, us */
+  uint32_t xfer_us[BF_MAX_TOOLS];           /* x_i: host<->device transfer, us (GPU modes only) */
+  uint32_t load_us[BF_MAX_TOOLS];           /* l_i: gpu_queue load-in, us */
+  uint32_t vram_mib[BF_MAX_TOOLS];          /* m_i: VRAM footprint, MiB */
+  uint32_t vram_budget_mib;                 /* M */
+  uint32_t slowdown_q10[BF_MAX_TOOLS + 1];  /* f[k], k=1..n, 1024 = isolated speed */
+} bf_scenario_desc;
+
+/* Result of a search: the argmin mapping and its makespan. */
+typedef struct bf_result {
+  uint64_t index;                  /* canonical mapping index */
+  uint32_t makespan_us;            /* 0xFFFFFFFF if feasible == 0 */
+  uint32_t feasible;               /* 1 if a feasible mapping was found in the searched range */
+  uint8_t mode[BF_MAX_TOOLS];      /* decoded digits of `index` (bf_mode), 0 beyond n */
+} bf_result;
+
+/* Opaque handle: validated scenario, its device-format tables and a small
+ * device/pinned scratch area.  Owned by the library. */
+typedef struct bf_scenario bf_scenario;
+
+/* Validate a desc without touching the GPU.  BF_OK or BF_EINVAL. */
+int bf_validate_desc(const bf_scenario_desc* desc);
+
+/* Validate `desc`, copy it, allocate the handle's scratch (8-byte device key,
+ * 8-byte pinned host key) on the current device and return it in *out.
+ * The caller releases it with bf_destroy_scenario.  BF_EINVAL, BF_ENOMEM,
+ * BF_ECUDA. */
+int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out);
+
+/* Release a handle (NULL is accepted).  Synchronises with nothing: the caller
+ * must make sure no work using it is still in flight. */
+int bf_destroy_scenario(bf_scenario* scn);
+
+/* Evaluate mappings [first, first+count) (§2.1's T_e2e under the model):
+ * d_makespan[j] = makespan of mapping first+j (0xFFFFFFFF if infeasible),
+ * d_feasible[j] = 1/0.  Both are caller-owned device arrays of >= count
+ * elements.  Asynchronous on `cuda_stream`.  count == 0 is a no-op.
+ * BF_ERANGE if first+count > 3^n; BF_EINVAL on NULL pointers. */
+int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count,
+                     uint32_t* d_makespan, uint8_t* d_feasible, void* cuda_stream);
+
+/* Brute-force oracle of §2.3/§4.1 under the model: the feasible mapping of
+ * lowest makespan over all 3^n, ties to the lowest index.  Blocks until the
+ * result is on the host (bounded wait).  Writes *out on BF_OK. */
+int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_stream);
+
+/* As bf_search_best over mappings [first, first+count) only; out->feasible is
+ * 0 (and index = first) when no mapping in the range is feasible.  Range
+ * searches compose: the best of the parts' results (lowest makespan, then
+ * lowest index) is the result of their union -- used to split one search
+ * across devices or to resume it piecewise.  BF_ERANGE if outside [0, 3^n);
+ * count == 0 gives feasible = 0. */
+int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
+                    bf_result* out, void* cuda_stream);
+
+/* Full search of `count` independent scenarios in one launch (the batched
+ * path): out[i] is the result for descs[i].  All descs are validated first;
+ * the first invalid one fails the call with BF_EINVAL naming its position.
+ * Allocates and frees its device scratch (packed tables + one key per
+ * scenario) per call.  Blocks until the results are on the host. */
+int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
+                    void* cuda_stream);
+
+/* Time limit of blocking waits, in milliseconds (default 600000; 0 = none).
+ * Process-wide. */
+void bf_set_wait_timeout_ms(uint32_t ms);
+
+/* Description of the last failure on this thread ("" if none). */
+const char* bf_last_error(void);
+
+/* Library version string, e.g. "bf 1.0 (model v1)". */
+const char* bf_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BF_H_ */

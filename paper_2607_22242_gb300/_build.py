@@ -1,0 +1,84 @@
+"""Build ``libbf.so`` in-tree with nvcc for sm_103a (GB300).
+
+Each tool-count bucket of ``csrc/bf_kernels.cu`` is its own translation unit
+(``-DBF_NT=<NT>``); the units compile in parallel and link with ``bf_capi.cu``
+into ``paper_2607_22242_gb300/_build/libbf.so`` (CUDA runtime linked
+statically, so the library carries no path to a toolkit).
+"""
+from __future__ import annotations
+
+import concurrent.futures as cf
+import hashlib
+import os
+import shutil
+import subprocess
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+CSRC = os.path.join(HERE, "csrc")
+INCLUDE = os.path.join(os.path.dirname(HERE), "include")
+BUILD_DIR = os.path.join(HERE, "_build")
+LIB_PATH = os.path.join(BUILD_DIR, "libbf.so")
+BUCKETS = (4, 6, 8, 10, 12, 14, 16, 18, 19, 20)
+ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
+NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", f"-I{INCLUDE}"]
+
+
+def nvcc() -> str:
+    path = shutil.which("nvcc") or "/usr/local/cuda/bin/nvcc"
+    if not os.path.exists(path):
+        raise RuntimeError("nvcc not found: the CUDA toolkit is required to build libbf.so")
+    return path
+
+
+def _sources():
+    return [os.path.join(CSRC, f) for f in sorted(os.listdir(CSRC))] + [os.path.join(INCLUDE, "bf.h")]
+
+
+def _fingerprint(extra) -> str:
+    h = hashlib.sha256()
+    for path in _sources():
+        with open(path, "rb") as fh:
+            h.update(path.encode() + fh.read())
+    h.update(" ".join(ARCH + NVCC_FLAGS + list(extra)).encode())
+    return h.hexdigest()
+
+
+def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
+    """Compile and link libbf.so unless an up-to-date copy exists; return its path."""
+    os.makedirs(BUILD_DIR, exist_ok=True)
+    stamp = os.path.join(BUILD_DIR, "libbf.stamp")
+    fp = _fingerprint(extra_flags)
+    if not force and os.path.exists(LIB_PATH) and os.path.exists(stamp):
+        with open(stamp) as fh:
+            if fh.read().strip() == fp:
+                return LIB_PATH
+    cc = nvcc()
+    jobs = []
+    for nt in BUCKETS:
+        obj = os.path.join(BUILD_DIR, f"bf_kernels_nt{nt}.o")
+        jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, f"-DBF_NT={nt}", "-c",
+                     os.path.join(CSRC, "bf_kernels.cu"), "-o", obj])
+    capi_obj = os.path.join(BUILD_DIR, "bf_capi.o")
+    jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, "bf_capi.cu"), "-o", capi_obj])
+
+    def run(cmd):
+        res = subprocess.run(cmd, capture_output=True, text=True)
+        if res.returncode != 0:
+            raise RuntimeError(f"nvcc failed: {' '.join(cmd)}\n{res.stdout}\n{res.stderr}")
+        if verbose:
+            print(res.stdout + res.stderr)
+        return cmd[-1]
+
+    workers = min(len(jobs), max(1, os.cpu_count() or 1))
+    with cf.ThreadPoolExecutor(workers) as pool:
+        objs = list(pool.map(run, jobs))
+    tmp = LIB_PATH + f".tmp{os.getpid()}"
+    run([cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs])
+    os.replace(tmp, LIB_PATH)
+    with open(stamp, "w") as fh:
+        fh.write(fp)
+    return LIB_PATH
+
+
+if __name__ == "__main__":
+    print(build(force=True, verbose=False))

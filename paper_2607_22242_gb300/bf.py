@@ -1,0 +1,246 @@
+"""Python binding of ``libbf.so`` (C ABI in ``include/bf.h``).
+
+Argument marshalling only: every step of the search runs in the library's
+CUDA kernels.  PyTorch supplies device buffers (``eval_mappings`` outputs) and
+streams (``torch.cuda.current_stream()`` by default).  The functions mirror
+the C entry points without their ``bf_`` prefix: ``validate_desc``,
+``create_scenario``, ``destroy_scenario``, ``eval_mappings``, ``search_best``,
+``search_range``, ``search_batch``, ``set_wait_timeout_ms``, ``last_error``,
+``version``.
+
+There is no CPU fallback: if ``libbf.so`` has not been built, or no CUDA
+device is present, these calls raise.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+import os
+from typing import List, Optional, Sequence, Tuple, Union
+
+from .scenarios import MAX_TOOLS, Scenario
+
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "_build", "libbf.so")
+
+BF_OK, BF_EINVAL, BF_ERANGE, BF_ENOMEM, BF_ECUDA, BF_ETIMEOUT = range(6)
+STATUS_NAMES = {0: "BF_OK", 1: "BF_EINVAL", 2: "BF_ERANGE", 3: "BF_ENOMEM", 4: "BF_ECUDA", 5: "BF_ETIMEOUT"}
+INFEASIBLE = 0xFFFFFFFF
+EXPORTED = ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
+            "bf_search_best", "bf_search_range", "bf_search_batch", "bf_set_wait_timeout_ms",
+            "bf_last_error", "bf_version")
+
+
+class BfError(RuntimeError):
+    def __init__(self, code: int, message: str):
+        super().__init__(f"{STATUS_NAMES.get(code, code)}: {message}")
+        self.code = code
+        self.message = message
+
+
+U32x20 = ctypes.c_uint32 * MAX_TOOLS
+
+
+class Desc(ctypes.Structure):
+    """``bf_scenario_desc``."""
+    _fields_ = [("n", ctypes.c_uint32), ("pred_mask", U32x20), ("cpu_us", U32x20), ("gpu_us", U32x20),
+                ("xfer_us", U32x20), ("load_us", U32x20), ("vram_mib", U32x20),
+                ("vram_budget_mib", ctypes.c_uint32), ("slowdown_q10", ctypes.c_uint32 * (MAX_TOOLS + 1))]
+
+
+class CResult(ctypes.Structure):
+    """``bf_result``."""
+    _fields_ = [("index", ctypes.c_uint64), ("makespan_us", ctypes.c_uint32), ("feasible", ctypes.c_uint32),
+                ("mode", ctypes.c_uint8 * MAX_TOOLS)]
+
+
+@dataclasses.dataclass
+class Result:
+    index: int
+    makespan_us: int
+    feasible: bool
+    modes: List[int]
+
+
+_lib = None
+
+
+def load(path: str = LIB_PATH):
+    """Load libbf.so (raises if it has not been built)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with `python -c 'import __graft_entry__ as g; g.build()'`")
+    lib = ctypes.CDLL(path)
+    vp, u64, u32 = ctypes.c_void_p, ctypes.c_uint64, ctypes.c_uint32
+    lib.bf_validate_desc.argtypes = [ctypes.POINTER(Desc)]
+    lib.bf_create_scenario.argtypes = [ctypes.POINTER(Desc), ctypes.POINTER(vp)]
+    lib.bf_destroy_scenario.argtypes = [vp]
+    lib.bf_eval_mappings.argtypes = [vp, u64, u64, vp, vp, vp]
+    lib.bf_search_best.argtypes = [vp, ctypes.POINTER(CResult), vp]
+    lib.bf_search_range.argtypes = [vp, u64, u64, ctypes.POINTER(CResult), vp]
+    lib.bf_search_batch.argtypes = [ctypes.POINTER(Desc), u32, ctypes.POINTER(CResult), vp]
+    for name in ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
+                 "bf_search_best", "bf_search_range", "bf_search_batch"):
+        getattr(lib, name).restype = ctypes.c_int
+    lib.bf_set_wait_timeout_ms.argtypes = [u32]
+    lib.bf_set_wait_timeout_ms.restype = None
+    lib.bf_last_error.restype = ctypes.c_char_p
+    lib.bf_version.restype = ctypes.c_char_p
+    _lib = lib
+    return lib
+
+
+def _check(code: int):
+    if code != BF_OK:
+        raise BfError(code, last_error())
+
+
+def last_error() -> str:
+    return load().bf_last_error().decode()
+
+
+def version() -> str:
+    return load().bf_version().decode()
+
+
+def set_wait_timeout_ms(ms: int) -> None:
+    load().bf_set_wait_timeout_ms(ms)
+
+
+def to_desc(scn: Scenario) -> Desc:
+    d = Desc()
+    d.n = scn.n
+    for name in ("pred_mask", "cpu_us", "gpu_us", "xfer_us", "load_us", "vram_mib"):
+        arr = getattr(d, name)
+        for i, v in enumerate(getattr(scn, name)[:MAX_TOOLS]):
+            arr[i] = v
+    d.vram_budget_mib = scn.vram_budget_mib
+    for k, v in enumerate(scn.slowdown_q10[:MAX_TOOLS + 1]):
+        d.slowdown_q10[k] = v
+    return d
+
+
+def _result(r: CResult, n: int) -> Result:
+    return Result(int(r.index), int(r.makespan_us), bool(r.feasible), [int(r.mode[i]) for i in range(n)])
+
+
+def _stream_handle(stream) -> int:
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def validate_desc(scn: Scenario) -> None:
+    """Raise BfError(BF_EINVAL) if the scenario is outside the library's limits."""
+    d = to_desc(scn)
+    _check(load().bf_validate_desc(ctypes.byref(d)))
+
+
+class ScenarioHandle:
+    """An owned ``bf_scenario*``; released by :meth:`close` (or garbage collection)."""
+
+    def __init__(self, scn: Scenario):
+        self.scenario = scn
+        self._ptr = ctypes.c_void_p()
+        d = to_desc(scn)
+        _check(load().bf_create_scenario(ctypes.byref(d), ctypes.byref(self._ptr)))
+
+    @property
+    def ptr(self):
+        if not self._ptr:
+            raise ValueError("scenario handle is closed")
+        return self._ptr
+
+    def close(self):
+        if self._ptr:
+            ptr, self._ptr = self._ptr, ctypes.c_void_p()
+            _check(load().bf_destroy_scenario(ptr))
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *exc):
+        self.close()
+
+
+def create_scenario(scn: Scenario) -> ScenarioHandle:
+    return ScenarioHandle(scn)
+
+
+def destroy_scenario(handle: ScenarioHandle) -> None:
+    handle.close()
+
+
+def _handle(h: Union[ScenarioHandle, Scenario]) -> Tuple[ScenarioHandle, bool]:
+    if isinstance(h, ScenarioHandle):
+        return h, False
+    return ScenarioHandle(h), True
+
+
+def eval_mappings(h: Union[ScenarioHandle, Scenario], first: int, count: int, out_makespan=None,
+                  out_feasible=None, stream=None):
+    """Makespans (torch.int32 CUDA tensor holding u32 bit patterns) and feasibility
+    flags (torch.uint8) of mappings [first, first+count).  Asynchronous on ``stream``;
+    the scenario's tables travel by value with the launch, so a temporary handle
+    may be released as soon as the call returns."""
+    import torch
+    handle, owned = _handle(h)
+    try:
+        if out_makespan is None:
+            out_makespan = torch.empty(count, dtype=torch.int32, device="cuda")
+        if out_feasible is None:
+            out_feasible = torch.empty(count, dtype=torch.uint8, device="cuda")
+        assert out_makespan.is_cuda and out_feasible.is_cuda
+        assert out_makespan.numel() >= count and out_feasible.numel() >= count
+        assert out_makespan.element_size() == 4 and out_feasible.element_size() == 1
+        _check(load().bf_eval_mappings(handle.ptr, first, count, ctypes.c_void_p(out_makespan.data_ptr()),
+                                       ctypes.c_void_p(out_feasible.data_ptr()),
+                                       ctypes.c_void_p(_stream_handle(stream))))
+        return out_makespan, out_feasible
+    finally:
+        if owned:
+            handle.close()
+
+
+def search_best(h: Union[ScenarioHandle, Scenario], stream=None) -> Result:
+    """Optimal feasible mapping over all 3^n (ties to the lowest index)."""
+    handle, owned = _handle(h)
+    try:
+        r = CResult()
+        _check(load().bf_search_best(handle.ptr, ctypes.byref(r), ctypes.c_void_p(_stream_handle(stream))))
+        return _result(r, handle.scenario.n)
+    finally:
+        if owned:
+            handle.close()
+
+
+def search_range(h: Union[ScenarioHandle, Scenario], first: int, count: int, stream=None) -> Result:
+    """Best feasible mapping in [first, first+count) (feasible=False if none)."""
+    handle, owned = _handle(h)
+    try:
+        r = CResult()
+        _check(load().bf_search_range(handle.ptr, first, count, ctypes.byref(r),
+                                      ctypes.c_void_p(_stream_handle(stream))))
+        return _result(r, handle.scenario.n)
+    finally:
+        if owned:
+            handle.close()
+
+
+def search_batch(scns: Sequence[Scenario], stream=None) -> List[Result]:
+    """Full search of each scenario, one launch for the whole batch."""
+    count = len(scns)
+    descs = (Desc * max(count, 1))()
+    for i, s in enumerate(scns):
+        descs[i] = to_desc(s)
+    results = (CResult * max(count, 1))()
+    _check(load().bf_search_batch(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
+    return [_result(results[i], scns[i].n) for i in range(count)]

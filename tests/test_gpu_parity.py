@@ -1,0 +1,285 @@
+"""Parity of the CUDA search (through the C ABI) with the CPU oracle.
+
+Makespans, feasibility flags and argmin indices must match bit for bit.
+Small and mid-size cases are compared element by element with the oracle run
+in the test; full-size cases (3^19 mappings, 4096-scenario batch) against the
+oracle's results committed in golden/config_results.json, plus sampled
+chunks computed by the oracle here.
+"""
+import json
+import os
+
+import numpy as np
+import pytest
+
+import oracle
+import pins
+from paper_2607_22242_gb300 import bf
+from paper_2607_22242_gb300 import scenarios as S
+
+pytestmark = pytest.mark.gpu
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden")
+INF = 0xFFFFFFFF
+THREADS = oracle.default_threads()
+
+
+@pytest.fixture(scope="module", autouse=True)
+def cuda():
+    import torch
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    import __graft_entry__
+    __graft_entry__.build()
+    torch.cuda.set_device(0)
+    return torch
+
+
+@pytest.fixture(scope="module")
+def golden():
+    path = os.path.join(GOLDEN, "config_results.json")
+    with open(path) as fh:
+        return json.load(fh)["configs"]
+
+
+def gpu_eval(h, first, count):
+    import torch
+    ms, fe = bf.eval_mappings(h, first, count)
+    torch.cuda.synchronize()
+    return ms.cpu().numpy().view(np.uint32).astype(np.uint64), fe.cpu().numpy()
+
+
+def assert_same(h, scn, first, count):
+    g_ms, g_fe = gpu_eval(h, first, count)
+    o_ms, o_fe = oracle.eval_range(scn, first, count, THREADS)
+    bad = np.flatnonzero((g_ms != o_ms) | (g_fe != o_fe))
+    assert bad.size == 0, (f"{bad.size} mismatches, first at index {first + int(bad[0])}: "
+                           f"gpu {int(g_ms[bad[0]])}/{int(g_fe[bad[0]])} oracle {int(o_ms[bad[0]])}/{int(o_fe[bad[0]])}")
+
+
+# --------------------------------------------------------------------------- small cases
+
+def test_hand_examples():
+    for ex in pins._load("hand_examples.json")["examples"]:
+        scn = S.Scenario.from_dict(ex["scenario"])
+        with bf.create_scenario(scn) as h:
+            ms, fe = gpu_eval(h, 0, 3 ** scn.n)
+            for idx, want in ex["expected"].items():
+                assert int(ms[int(idx)]) == want, (ex["name"], idx)
+                assert bool(fe[int(idx)]) == (want != INF)
+            if "argmin" in ex:
+                r = bf.search_best(h)
+                assert [r.index, r.makespan_us] == ex["argmin"], ex["name"]
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_random_small_exhaustive(seed):
+    """Every mapping of small random DAGs: ties, VRAM-blocked queues, infeasible starts."""
+    rng = np.random.default_rng(1000 + seed)
+    for t in range(60):
+        n = int(rng.integers(1, 8))
+        scn = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.3, 0.7])), tight=bool(t % 3),
+                             contention=bool(t % 5), max_time=int(rng.choice([6, 30, 2000])))
+        with bf.create_scenario(scn) as h:
+            assert_same(h, scn, 0, 3 ** n)
+            r = bf.search_best(h)
+        assert (r.index, r.makespan_us) == oracle.search(scn)
+        assert r.modes == S.mapping_modes(r.index, n)
+
+
+@pytest.mark.parametrize("n", [1, 2, 9, 11, 13, 15, 17])
+def test_every_bucket_edge(n):
+    """Scenarios whose n sits at or just past a compiled bucket size, realistic magnitudes."""
+    rng = np.random.default_rng(50 + n)
+    base = S.random_small(rng, n, edge_p=0.3, tight=True, max_time=50)
+    scale = lambda v: [x * 997 + 1 for x in v]
+    scn = S.Scenario(n, base.pred_mask, scale(base.cpu_us), scale(base.gpu_us), scale(base.xfer_us),
+                     scale(base.load_us), [m * 300 for m in base.vram_mib], base.vram_budget_mib * 300,
+                     S.slowdown_linear())
+    total = 3 ** n
+    with bf.create_scenario(scn) as h:
+        count = min(total, 200_003)
+        assert_same(h, scn, 0, count)
+        assert_same(h, scn, total - min(total, 4099), min(total, 4099))
+        r = bf.search_best(h)
+    if total <= 2_000_000:
+        assert (r.index, r.makespan_us) == oracle.search(scn, THREADS)
+
+
+# --------------------------------------------------------------------------- standard workloads
+
+@pytest.mark.parametrize("cfg", [0, 1, 2])
+def test_config_full_arrays(cfg, golden):
+    scn = S.config(cfg)
+    assert S.sha256_of([scn]) == golden[str(cfg)]["sha256"]
+    with bf.create_scenario(scn) as h:
+        assert_same(h, scn, 0, 3 ** scn.n)
+        r = bf.search_best(h)
+    g = golden[str(cfg)]["summary"]
+    assert (r.index, r.makespan_us, r.feasible) == (g["best_index"], g["best_makespan"], True)
+
+
+def test_config3_argmin(golden):
+    """The full 3^19 search in the benchmark's launch configuration."""
+    scn = S.config3()
+    assert S.sha256_of([scn]) == golden["3"]["sha256"]
+    g = golden["3"]["summary"]
+    with bf.create_scenario(scn) as h:
+        for _ in range(2):
+            r = bf.search_best(h)
+            assert (r.index, r.makespan_us, r.feasible) == (g["best_index"], g["best_makespan"], True)
+        assert oracle.evaluate(scn, r.index) == r.makespan_us
+
+
+def test_config3_sampled_chunks():
+    scn = S.config3()
+    total = 3 ** scn.n
+    rng = np.random.default_rng(7)
+    starts = [0, total - 70_001] + [int(v) for v in rng.integers(0, total - 70_001, 10)]
+    with bf.create_scenario(scn) as h:
+        for s in starts:
+            assert_same(h, scn, s, 70_001)
+
+
+def test_config3_full_stream_summary(golden):
+    """Every makespan of the 3^19 stream, compared through the oracle's summary."""
+    import torch
+    scn = S.config3()
+    total = 3 ** scn.n
+    g = golden["3"]["summary"]
+    # torch's int64 products wrap modulo 2^64 like the oracle's uint64: check on a sample first.
+    sample = np.random.default_rng(3).integers(0, 2 ** 32, 1000, dtype=np.uint64)
+    t = torch.from_numpy(sample.astype(np.int64)).cuda()
+    idx = torch.arange(5, 1005, dtype=torch.int64, device="cuda")
+    th = int((t * (idx * 2654435761 + 1)).sum().item()) & (2 ** 64 - 1)
+    assert th == oracle.stream_hash(sample, 5)
+    piece = 1 << 27
+    feasible = ms_sum = hsum = 0
+    with bf.create_scenario(scn) as h:
+        ms = torch.empty(piece, dtype=torch.int32, device="cuda")
+        fe = torch.empty(piece, dtype=torch.uint8, device="cuda")
+        for first in range(0, total, piece):
+            cnt = min(piece, total - first)
+            bf.eval_mappings(h, first, cnt, ms, fe)
+            m64 = ms[:cnt].to(torch.int64) & 0xFFFFFFFF
+            f = fe[:cnt].to(torch.bool)
+            feasible += int(f.sum().item())
+            ms_sum += int(m64[f].sum().item())
+            idx = torch.arange(first, first + cnt, dtype=torch.int64, device="cuda")
+            hsum += int((m64 * (idx * 2654435761 + 1)).sum().item())
+    assert feasible == g["feasible"]
+    assert ms_sum == g["makespan_sum"]
+    assert hsum & (2 ** 64 - 1) == g["hash"]
+
+
+def test_config4_batch(golden):
+    batch = S.config4()
+    assert S.sha256_of(batch) == golden["4"]["sha256"]
+    res = bf.search_batch(batch)
+    want_i, want_m = golden["4"]["best_index"], golden["4"]["best_makespan"]
+    bad = [i for i, r in enumerate(res) if (r.index, r.makespan_us, r.feasible) != (want_i[i], want_m[i], True)]
+    assert not bad, f"{len(bad)} scenarios differ, first {bad[0]}: {res[bad[0]]} vs {(want_i[bad[0]], want_m[bad[0]])}"
+
+
+def test_batch_mixed_sizes():
+    rng = np.random.default_rng(77)
+    scns = [S.random_small(rng, int(rng.integers(1, 9)), max_time=int(rng.choice([8, 500]))) for _ in range(40)]
+    res = bf.search_batch(scns)
+    o_i, o_m = oracle.search_batch(scns, THREADS)
+    assert [(r.index, r.makespan_us) for r in res] == list(zip(o_i.tolist(), o_m.tolist()))
+
+
+# --------------------------------------------------------------------------- ranges and edge cases
+
+def test_search_ranges_compose():
+    scn = S.config2()
+    total = 3 ** scn.n
+    cuts = [0, 1, 12345, 3 ** 10, 20_000_000, total - 1, total]
+    with bf.create_scenario(scn) as h:
+        parts = [bf.search_range(h, a, b - a) for a, b in zip(cuts, cuts[1:])]
+        full = bf.search_best(h)
+    best = min((p.makespan_us, p.index) for p in parts if p.feasible)
+    assert best == (full.makespan_us, full.index)
+    for (a, b), p in zip(zip(cuts, cuts[1:]), parts):
+        if b - a <= 2_000_000:
+            oi, om = oracle.search_range(scn, a, b - a, THREADS)
+            assert (p.index, p.makespan_us) == ((oi, om) if oi >= 0 else (a, INF))
+
+
+def test_n20_sampled():
+    rng = np.random.default_rng(20)
+    base = S.random_small(rng, 20, edge_p=0.15, tight=True, max_time=60)
+    scn = S.Scenario(20, base.pred_mask, [c * 1000 for c in base.cpu_us], [g * 1000 for g in base.gpu_us],
+                     [x * 1000 for x in base.xfer_us], [l * 1000 for l in base.load_us],
+                     [m * 1000 for m in base.vram_mib], base.vram_budget_mib * 1000, S.slowdown_linear())
+    total = 3 ** 20
+    with bf.create_scenario(scn) as h:
+        for first in (0, total // 3, total - 50_000):
+            assert_same(h, scn, first, 50_000)
+        r = bf.search_range(h, total - 1_000_000, 1_000_000)
+    oi, om = oracle.search_range(scn, total - 1_000_000, 1_000_000, THREADS)
+    assert (r.index, r.makespan_us, r.feasible) == ((oi, om, True) if oi >= 0 else (total - 1_000_000, INF, False))
+
+
+def test_all_infeasible_range():
+    # a single tool larger than the budget: only the cpu mapping is feasible
+    scn = S.Scenario(1, [0], [50], [5], [0], [0], [10], 5, S.slowdown_flat())
+    with bf.create_scenario(scn) as h:
+        r = bf.search_range(h, 1, 2)
+        assert not r.feasible and r.makespan_us == INF and r.index == 1
+        r = bf.search_best(h)
+        assert (r.index, r.makespan_us, r.feasible) == (0, 50, True)
+        r = bf.search_range(h, 0, 0)
+        assert not r.feasible
+
+
+def test_range_errors():
+    scn = S.config0()
+    lib = bf.load()
+    with bf.create_scenario(scn) as h:
+        for first, count in ((0, 3 ** 8 + 1), (3 ** 8, 1), (3 ** 8 + 1, 0), (2 ** 63, 2 ** 63), (1, 2 ** 64 - 1)):
+            with pytest.raises(bf.BfError) as ei:
+                bf.search_range(h, first, count)
+            assert ei.value.code == bf.BF_ERANGE
+            # the range is checked before the output pointers
+            assert lib.bf_eval_mappings(h.ptr, first, count, None, None, None) == bf.BF_ERANGE
+        bf.eval_mappings(h, 3 ** 8, 0)  # empty range at the end is fine
+
+
+def test_ragged_eval_ranges():
+    scn = S.config1()
+    with bf.create_scenario(scn) as h:
+        for first, count in ((1, 255), (255, 257), (100_000, 1), (3 ** 12 - 513, 513), (7, 33_333)):
+            assert_same(h, scn, first, count)
+
+
+def test_non_default_stream():
+    import torch
+    scn = S.config1()
+    s = torch.cuda.Stream()
+    with bf.create_scenario(scn) as h:
+        with torch.cuda.stream(s):
+            r = bf.search_best(h, stream=s)
+            ms, fe = bf.eval_mappings(h, 0, 3 ** 12, stream=s)
+        s.synchronize()
+    assert (r.index, r.makespan_us) == oracle.search(scn, THREADS)
+    o_ms, _ = oracle.eval_range(scn, 0, 3 ** 12, THREADS)
+    assert np.array_equal(ms.cpu().numpy().view(np.uint32).astype(np.uint64), o_ms)
+
+
+def test_wait_timeout_is_reported():
+    """The host wait is bounded: a 1 ms limit on a ~0.1 s search returns BF_ETIMEOUT, the GPU
+    work finishes normally, and the library works afterwards."""
+    import torch
+    scn = S.config3()
+    with bf.create_scenario(scn) as h:
+        bf.set_wait_timeout_ms(1)
+        try:
+            with pytest.raises(bf.BfError) as ei:
+                bf.search_best(h)
+            assert ei.value.code == bf.BF_ETIMEOUT
+        finally:
+            bf.set_wait_timeout_ms(600000)
+            torch.cuda.synchronize()
+        r = bf.search_best(h)
+    assert r.feasible
