@@ -1,7 +1,7 @@
 """Build ``libbf.so`` in-tree with nvcc for sm_103a (GB300).
 
-Each tool-count bucket of ``csrc/bf_kernels.cu`` is its own translation unit
-(``-DBF_NT=<NT>``); the units compile in parallel and link with ``bf_capi.cu``
+Each window-width bucket of ``csrc/bf_kernels.cu`` is its own translation unit
+(``-DBF_NW=<slots>``); the units compile in parallel and link with ``bf_capi.cu``
 into ``paper_2607_22242_gb300/_build/libbf.so`` (CUDA runtime linked
 statically, so the library carries no path to a toolkit).
 """
@@ -18,7 +18,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(BUILD_DIR, "libbf.so")
-BUCKETS = (4, 6, 8, 10, 12, 14, 16, 18, 19, 20)
+BUCKETS = (4, 6, 8, 10, 12, 14, 16, 18, 19, 20)  # window widths (bf_launch.h)
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", f"-I{INCLUDE}"]
 
@@ -55,8 +55,8 @@ def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
     cc = nvcc()
     jobs = []
     for nt in BUCKETS:
-        obj = os.path.join(BUILD_DIR, f"bf_kernels_nt{nt}.o")
-        jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, f"-DBF_NT={nt}", "-c",
+        obj = os.path.join(BUILD_DIR, f"bf_kernels_nw{nt}.o")
+        jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, f"-DBF_NW={nt}", "-c",
                      os.path.join(CSRC, "bf_kernels.cu"), "-o", obj])
     capi_obj = os.path.join(BUILD_DIR, "bf_capi.o")
     jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, "bf_capi.cu"), "-o", capi_obj])

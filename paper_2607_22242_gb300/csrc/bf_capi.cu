@@ -14,16 +14,24 @@
 
 #include "../../include/bf.h"
 #include "bf_launch.h"
+#include "bf_plan.h"
 
 struct bf_scenario {
   bf_scenario_desc desc;
-  bfk::Tables tables;
+  bfk::Tables tables;   // all n tools
+  bfk::Tables window;   // tools [W0, n), renumbered from 0
+  uint32_t P, K, W0;    // index split and window start (see bfk::Plan)
   int device;
   unsigned long long* d_key;  // device scratch: one packed search key
   unsigned long long* h_key;  // pinned host copy of it
 };
 
 namespace {
+
+using bfk::host::build_tables;
+using bfk::host::make_plan;
+using bfk::host::pow3;
+using bfk::host::split_and_window;
 
 thread_local std::string g_error;
 uint32_t g_wait_timeout_ms = 600000;
@@ -65,12 +73,6 @@ cudaError_t lib_malloc_host(void** p, size_t bytes) {
   return cudaMallocHost(p, bytes);
 }
 
-uint64_t pow3(uint32_t n) {
-  uint64_t p = 1;
-  for (uint32_t i = 0; i < n; ++i) p *= 3;
-  return p;
-}
-
 int validate(const bf_scenario_desc* d, const char* who) {
   if (!d) return fail(BF_EINVAL, "%s: desc is NULL", who);
   const uint32_t n = d->n;
@@ -109,37 +111,6 @@ int validate(const bf_scenario_desc* d, const char* who) {
   return BF_OK;
 }
 
-void build_tables(const bf_scenario_desc* d, bfk::Tables* t) {
-  std::memset(t, 0, sizeof *t);
-  const uint32_t n = d->n;
-  t->n = n;
-  t->budget = d->vram_budget_mib;
-  t->all_mask = (n == 32) ? ~0u : ((1u << n) - 1u);
-  for (uint32_t v = 0; v < n; ++v) {
-    t->pred[v] = d->pred_mask[v];
-    for (uint32_t u = 0; u < v; ++u)
-      if (d->pred_mask[v] & (1u << u)) t->succ[u] |= 1u << v;
-    t->cpu[v] = d->cpu_us[v];
-    t->wnow[v] = (d->gpu_us[v] + d->xfer_us[v]) * 1024u;
-    t->wq[v] = (d->load_us[v] + d->gpu_us[v] + d->xfer_us[v]) * 1024u;
-    t->vram[v] = d->vram_mib[v];
-    if (d->vram_mib[v] > d->vram_budget_mib) t->big_mask |= 1u << v;
-  }
-  for (uint32_t k = 1; k <= BF_MAX_TOOLS; ++k) {
-    // Entries above n are never used; fill them with f[n] so every k is defined.
-    const uint32_t f = d->slowdown_q10[k <= n ? k : n];
-    uint32_t l = 0;
-    while ((1u << l) < f) ++l;  // ceil(log2 f)
-    if (l < 12) l = 12;
-    const unsigned __int128 num = (unsigned __int128)1 << (52 + l);
-    t->f[k] = f;
-    t->fshift[k] = l - 12;
-    t->fmagic[k] = (uint64_t)((num + f - 1) / f);
-  }
-  t->f[0] = 1024;
-  t->fmagic[0] = 1ull << 54;
-}
-
 int wait_stream(cudaStream_t st, const char* who) {
   const auto t0 = std::chrono::steady_clock::now();
   for (;;) {
@@ -175,14 +146,6 @@ void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* 
   }
 }
 
-// Consecutive mappings per thread in the search kernels: enough to amortise
-// the decode and the reductions, small enough to fill every SM for mid-size N.
-uint32_t search_chunk(uint64_t count) {
-  if (count >= (1ull << 26)) return 64;
-  if (count >= (1ull << 20)) return 16;
-  return 4;
-}
-
 #define BF_DISPATCH(NT_VAL, CALL)                         \
   switch (NT_VAL) {                                       \
     case 4: { e = bfk::CALL(4); } break;                  \
@@ -202,9 +165,9 @@ int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result
   cudaError_t e = cudaMemsetAsync(scn->d_key, 0xFF, sizeof(unsigned long long), st);
   if (e != cudaSuccess) return cuda_fail(e, who);
   if (count) {
-    const uint32_t per_thread = search_chunk(count);
-#define CALL(NT) launch_search_nt##NT(scn->tables, (uint32_t)first, count, per_thread, scn->d_key, st)
-    BF_DISPATCH(bfk::bucket_for(scn->desc.n), CALL)
+    const bfk::Plan plan = make_plan(scn->desc.n, scn->P, scn->K, scn->W0, first, count);
+#define CALL(NW) launch_search_nw##NW(scn->tables, scn->window, plan, scn->d_key, st)
+    BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
 #undef CALL
     if (e != cudaSuccess) return cuda_fail(e, who);
   }
@@ -231,6 +194,7 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   std::memset(s, 0, sizeof *s);
   s->desc = *desc;
   build_tables(desc, &s->tables);
+  split_and_window(s->tables, &s->P, &s->K, &s->W0, &s->window);
   cudaError_t e = cudaGetDevice(&s->device);
   if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_key), sizeof(unsigned long long));
   if (e == cudaSuccess) e = lib_malloc_host(reinterpret_cast<void**>(&s->h_key), sizeof(unsigned long long));
@@ -263,15 +227,11 @@ int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count, uin
                 (unsigned long long)first, (unsigned long long)first, (unsigned long long)count, scn->desc.n);
   if (count == 0) return BF_OK;
   if (!d_makespan || !d_feasible) return fail(BF_EINVAL, "bf_eval_mappings: NULL output buffer");
-  int sms = 0;
-  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, scn->device);
-  if (e != cudaSuccess) return cuda_fail(e, "bf_eval_mappings");
-  const uint64_t blocks_needed = (count + bfk::kThreads - 1) / bfk::kThreads;
-  const uint64_t cap = (uint64_t)sms * 16;
-  const int grid = (int)(blocks_needed < cap ? blocks_needed : cap);
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-#define CALL(NT) launch_eval_nt##NT(scn->tables, (uint32_t)first, count, d_makespan, d_feasible, grid, st)
-  BF_DISPATCH(bfk::bucket_for(scn->desc.n), CALL)
+  const bfk::Plan plan = make_plan(scn->desc.n, scn->P, scn->K, scn->W0, first, count);
+  cudaError_t e = cudaSuccess;
+#define CALL(NW) launch_eval_nw##NW(scn->tables, scn->window, plan, d_makespan, d_feasible, st)
+  BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
 #undef CALL
   if (e != cudaSuccess) return cuda_fail(e, "bf_eval_mappings");
   return BF_OK;
@@ -301,32 +261,39 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
     if (rc != BF_OK) return fail(rc, "bf_search_batch: descs[%u]: %s", i, g_error.c_str());
     if (descs[i].n > nmax) nmax = descs[i].n;
   }
-  std::vector<bfk::Tables> tables(count);
-  for (uint32_t i = 0; i < count; ++i) build_tables(descs + i, &tables[i]);
+  std::vector<bfk::BatchRecord> recs(count);
+  uint32_t wmax = 0, pmax = 0;
+  for (uint32_t i = 0; i < count; ++i) {
+    bfk::BatchRecord& r = recs[i];
+    std::memset(&r, 0, sizeof r);
+    build_tables(descs + i, &r.full);
+    uint32_t P, K, W0;
+    split_and_window(r.full, &P, &K, &W0, &r.window);
+    r.plan = make_plan(descs[i].n, P, K, W0, 0, pow3(descs[i].n));
+    if (r.window.n > wmax) wmax = r.window.n;
+    if (r.plan.pow3P > pmax) pmax = r.plan.pow3P;
+  }
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  bfk::Tables* d_tables = nullptr;
+  bfk::BatchRecord* d_recs = nullptr;
   unsigned long long* d_keys = nullptr;
   std::vector<unsigned long long> keys(count);
-  const size_t tbytes = sizeof(bfk::Tables) * count, kbytes = sizeof(unsigned long long) * count;
-  cudaError_t e = lib_malloc(reinterpret_cast<void**>(&d_tables), tbytes);
+  const size_t rbytes = sizeof(bfk::BatchRecord) * count, kbytes = sizeof(unsigned long long) * count;
+  cudaError_t e = lib_malloc(reinterpret_cast<void**>(&d_recs), rbytes);
   if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&d_keys), kbytes);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(d_tables, tables.data(), tbytes, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(d_recs, recs.data(), rbytes, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, kbytes, st);
   int rc = BF_OK;
   if (e == cudaSuccess) {
-    const uint64_t per_scn = pow3(nmax);
-    const uint32_t per_thread = per_scn >= 8192 ? 32 : 4;
-    const uint64_t threads = (per_scn + per_thread - 1) / per_thread;
-    const uint32_t bps = (uint32_t)((threads + bfk::kThreads - 1) / bfk::kThreads);
-#define CALL(NT) launch_batch_nt##NT(d_tables, count, per_thread, bps, d_keys, st)
-    BF_DISPATCH(bfk::bucket_for(nmax), CALL)
+    const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
+#define CALL(NW) launch_batch_nw##NW(d_recs, count, bps, d_keys, st)
+    BF_DISPATCH(bfk::bucket_for(wmax), CALL)
 #undef CALL
   }
   if (e == cudaSuccess) e = cudaMemcpyAsync(keys.data(), d_keys, kbytes, cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
   if (rc == BF_OK) rc = wait_stream(st, "bf_search_batch");
   if (rc != BF_ETIMEOUT) {  // on timeout the kernel may still use the scratch: leak it rather than free in-use memory
-    if (d_tables) cudaFree(d_tables);
+    if (d_recs) cudaFree(d_recs);
     if (d_keys) cudaFree(d_keys);
   }
   if (rc != BF_OK) return rc;

@@ -1,25 +1,34 @@
-// bf_kernels.cu -- the three search kernels, compiled once per tool-count
-// bucket (-DBF_NT=<NT>).  All integer ALU work; no tensor cores, no HBM
+// bf_kernels.cu -- the three search kernels, compiled once per window width
+// (-DBF_NW=<slots>).  All integer ALU work: no tensor cores, and no HBM
 // streaming beyond the eval kernel's 5 bytes of output per mapping.
 //
-//   eval   : one mapping per thread (grid-stride), coalesced stores of the
-//            makespan (u32) and feasibility flag (u8) -- §2.1's T_e2e per mapping.
-//   search : each thread walks a chunk of consecutive indices (decode once,
-//            then base-3 increment), keeps the smallest packed key
-//            (makespan << 32 | index), then warp shuffle-min -> block min ->
-//            one 64-bit atomicMin per block.  Ties go to the lowest index
-//            because the index is the key's low word.  This is the brute-force
-//            oracle of §2.3 / §4.1 under the integer model.
+// Work decomposition (the same in all three kernels).  A mapping index is
+// idx = p + 3^P * s.  Each warp owns one prefix p (the modes of tools
+// [0, P)); its 32 lanes simulate that prefix together -- identical control
+// flow -- until the first instant a suffix tool (index >= P) would become
+// ready, and lane 0 saves the state (restricted to the window [W0, n)) in
+// shared memory.  Then lane l resumes that state for suffixes s = l, l+32, ...
+// with a simulation only NW slots wide.  Every mapping's makespan is still
+// simulated event by event; only the common prefix of its history is shared.
+//
+//   eval   : writes the makespan (u32) and feasibility flag (u8) of every
+//            mapping in [first, last] -- §2.1's T_e2e per mapping.
+//   search : keeps the smallest packed key (makespan << 32 | index) per lane,
+//            then warp shuffle-min -> block min -> one 64-bit atomicMin per
+//            block.  Ties go to the lowest index (the key's low word).  This is
+//            the brute-force oracle of §2.3 / §4.1 under the integer model.
 //   batch  : as search, for many independent scenarios in one launch; each
-//            block stages its scenario's tables in shared memory.
+//            block stages its scenario's tables and plan in shared memory.
 #include "bf_launch.h"
 
-#ifndef BF_NT
-#error "compile with -DBF_NT=<tool-count bucket>"
+#ifndef BF_NW
+#error "compile with -DBF_NW=<window slot count>"
 #endif
 
 namespace bfk {
 namespace {
+
+constexpr int kWarps = kThreads / 32;
 
 __device__ __forceinline__ unsigned long long warp_min(unsigned long long v) {
 #pragma unroll
@@ -28,93 +37,137 @@ __device__ __forceinline__ unsigned long long warp_min(unsigned long long v) {
 }
 
 // Block-wide min of `v`, then one atomicMin into *dst from thread 0 (skipped
-// when the block saw no mapping).
+// when the block found nothing).
 __device__ __forceinline__ void block_min_to(unsigned long long v, unsigned long long* dst) {
-  __shared__ unsigned long long warp_best[kThreads / 32];
+  __shared__ unsigned long long warp_best[kWarps];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   v = warp_min(v);
   if (lane == 0) warp_best[warp] = v;
   __syncthreads();
   if (warp == 0) {
-    v = lane < (int)(blockDim.x >> 5) ? warp_best[lane] : ~0ull;
+    v = lane < kWarps ? warp_best[lane] : ~0ull;
     v = warp_min(v);
     if (lane == 0 && v != ~0ull) atomicMin(dst, v);
   }
 }
 
-template <int NT, typename TB>
-__device__ __forceinline__ unsigned long long search_chunk(const TB& tb, const SmemTables& sd,
-                                                           uint32_t idx, uint32_t cnt) {
-  unsigned long long best = ~0ull;
-  Digits dg = decode<NT>(idx);
-#pragma unroll 1
-  for (uint32_t j = 0; j < cnt; ++j) {
-    const uint32_t ms = simulate<NT>(tb, sd, dg);
-    best = min(best, ((unsigned long long)ms << 32) | (idx + j));
-    increment(dg);
+// Simulate prefix p once per warp and save its window state in `snap`.
+// Returns false (warp-uniformly) when every mapping with this prefix is
+// infeasible.
+template <typename TB>
+__device__ __forceinline__ bool prefix_phase(const TB& tb, const SmemTables& sd, const Plan& plan,
+                                             uint32_t p, Digits& dgp, Snapshot& snap) {
+  dgp = decode(p, plan.P);
+  bool ok = (dgp.que & tb.big_mask) == 0u;
+  if (ok) {
+    State<kMaxTools> s;
+    init_state(s, tb.all_mask);
+    const uint32_t suffix_mask = tb.all_mask & ~((1u << plan.P) - 1u);
+    ok = run<kMaxTools>(s, tb, sd, dgp, suffix_mask) == kRunStopped;
+    if (ok && (threadIdx.x & 31) == 0) save_window(s, plan.W0, tb.n - plan.W0, snap);
   }
-  return best;
+  __syncwarp();
+  return ok;
 }
 
-template <int NT>
+// Makespan of mapping (p, s) resumed from the warp's snapshot.
+template <typename TB>
+__device__ __forceinline__ uint32_t suffix_makespan(const TB& tw, const SmemTables& sdw, const Plan& plan,
+                                                    Digits dgp, uint32_t s, const Snapshot& snap) {
+  const Digits dgs = decode(s, plan.K);
+  const uint32_t sh = plan.P - plan.W0;
+  const Digits dw{(dgp.now >> plan.W0) | (dgs.now << sh), (dgp.que >> plan.W0) | (dgs.que << sh)};
+  if (dw.que & tw.big_mask) return kInfeasible;
+  State<BF_NW> w;
+  load_window(snap, w);
+  return run<BF_NW>(w, tw, sdw, dw, 0u) == kRunFinished ? w.T : kInfeasible;
+}
+
 __global__ void __launch_bounds__(kThreads) eval_kernel(const __grid_constant__ Tables tb,
-                                                        uint32_t first, uint64_t count,
+                                                        const __grid_constant__ Tables tw,
+                                                        const __grid_constant__ Plan plan,
                                                         uint32_t* __restrict__ ms_out,
                                                         uint8_t* __restrict__ fe_out) {
-  __shared__ SmemTables sd;
+  __shared__ SmemTables sd, sdw;
+  __shared__ Snapshot snap[kWarps];
   load_smem_tables(tb, sd);
+  load_smem_tables(tw, sdw);
   __syncthreads();
-  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
-  for (uint64_t j = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; j < count; j += stride) {
-    const uint32_t ms = simulate<NT>(tb, sd, decode<NT>(first + (uint32_t)j));
-    ms_out[j] = ms;
-    fe_out[j] = ms != kInfeasible;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint64_t p64 = (uint64_t)plan.p_lo + (uint64_t)blockIdx.x * kWarps + warp;
+  if (p64 > plan.p_hi) return;  // no block-level synchronisation follows
+  const uint32_t p = (uint32_t)p64;
+  Digits dgp;
+  const bool ok = prefix_phase(tb, sd, plan, p, dgp, snap[warp]);
+  for (uint32_t s = plan.s_lo + lane; s <= plan.s_hi; s += 32) {
+    const uint32_t idx = p + plan.pow3P * s;
+    if (idx < plan.first || idx > plan.last) continue;
+    const uint32_t ms = ok ? suffix_makespan(tw, sdw, plan, dgp, s, snap[warp]) : kInfeasible;
+    ms_out[idx - plan.first] = ms;
+    fe_out[idx - plan.first] = ms != kInfeasible;
   }
 }
 
-template <int NT>
 __global__ void __launch_bounds__(kThreads) search_kernel(const __grid_constant__ Tables tb,
-                                                          uint32_t first, uint64_t count,
-                                                          uint32_t per_thread,
+                                                          const __grid_constant__ Tables tw,
+                                                          const __grid_constant__ Plan plan,
                                                           unsigned long long* key) {
-  __shared__ SmemTables sd;
+  __shared__ SmemTables sd, sdw;
+  __shared__ Snapshot snap[kWarps];
   load_smem_tables(tb, sd);
+  load_smem_tables(tw, sdw);
   __syncthreads();
-  const uint64_t off = ((uint64_t)blockIdx.x * blockDim.x + threadIdx.x) * per_thread;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint64_t p64 = (uint64_t)plan.p_lo + (uint64_t)blockIdx.x * kWarps + warp;
   unsigned long long best = ~0ull;
-  if (off < count) {
-    const uint32_t cnt = (uint32_t)min((uint64_t)per_thread, count - off);
-    best = search_chunk<NT>(tb, sd, first + (uint32_t)off, cnt);
+  if (p64 <= plan.p_hi) {
+    const uint32_t p = (uint32_t)p64;
+    Digits dgp;
+    if (prefix_phase(tb, sd, plan, p, dgp, snap[warp])) {
+      for (uint32_t s = plan.s_lo + lane; s <= plan.s_hi; s += 32) {
+        const uint32_t idx = p + plan.pow3P * s;
+        if (idx < plan.first || idx > plan.last) continue;
+        const uint32_t ms = suffix_makespan(tw, sdw, plan, dgp, s, snap[warp]);
+        best = min(best, ((unsigned long long)ms << 32) | idx);
+      }
+    }
   }
   block_min_to(best, key);
 }
 
-template <int NT>
-__global__ void __launch_bounds__(kThreads) batch_kernel(const Tables* __restrict__ all,
-                                                         uint32_t per_thread,
+// One record per scenario of a batch: full tables, window tables and plan.
+__global__ void __launch_bounds__(kThreads) batch_kernel(const BatchRecord* __restrict__ recs,
                                                          uint32_t blocks_per_scenario,
                                                          unsigned long long* keys) {
-  __shared__ Tables tb;
-  __shared__ SmemTables sd;
-  const uint32_t s = blockIdx.x / blocks_per_scenario;
-  const uint32_t b = blockIdx.x - s * blocks_per_scenario;
+  __shared__ BatchRecord rec;
+  __shared__ SmemTables sd, sdw;
+  __shared__ Snapshot snap[kWarps];
+  const uint32_t sc = blockIdx.x / blocks_per_scenario;
+  const uint32_t b = blockIdx.x - sc * blocks_per_scenario;
   {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(all + s);
-    uint32_t* dst = reinterpret_cast<uint32_t*>(&tb);
-    for (uint32_t w = threadIdx.x; w < sizeof(Tables) / 4; w += blockDim.x) dst[w] = src[w];
+    const uint32_t* src = reinterpret_cast<const uint32_t*>(recs + sc);
+    uint32_t* dst = reinterpret_cast<uint32_t*>(&rec);
+    for (uint32_t w = threadIdx.x; w < sizeof(BatchRecord) / 4; w += blockDim.x) dst[w] = src[w];
   }
   __syncthreads();
-  load_smem_tables(tb, sd);
+  load_smem_tables(rec.full, sd);
+  load_smem_tables(rec.window, sdw);
   __syncthreads();
-  uint32_t total = 1;
-  for (uint32_t i = 0; i < tb.n; ++i) total *= 3u;
-  const uint64_t off = ((uint64_t)b * blockDim.x + threadIdx.x) * per_thread;
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const uint64_t p64 = (uint64_t)rec.plan.p_lo + (uint64_t)b * kWarps + warp;
   unsigned long long best = ~0ull;
-  if (off < total) {
-    const uint32_t cnt = (uint32_t)min((uint64_t)per_thread, (uint64_t)total - off);
-    best = search_chunk<NT>(tb, sd, (uint32_t)off, cnt);
+  if (p64 <= rec.plan.p_hi) {
+    const uint32_t p = (uint32_t)p64;
+    Digits dgp;
+    if (prefix_phase(rec.full, sd, rec.plan, p, dgp, snap[warp])) {
+      for (uint32_t s = rec.plan.s_lo + lane; s <= rec.plan.s_hi; s += 32) {
+        const uint32_t idx = p + rec.plan.pow3P * s;
+        const uint32_t ms = suffix_makespan(rec.window, sdw, rec.plan, dgp, s, snap[warp]);
+        best = min(best, ((unsigned long long)ms << 32) | idx);
+      }
+    }
   }
-  block_min_to(best, keys + s);
+  block_min_to(best, keys + sc);
 }
 
 }  // namespace
@@ -122,27 +175,28 @@ __global__ void __launch_bounds__(kThreads) batch_kernel(const Tables* __restric
 #define BF_PASTE2(a, b) a##b
 #define BF_PASTE(a, b) BF_PASTE2(a, b)
 
-cudaError_t BF_PASTE(launch_eval_nt, BF_NT)(const Tables& tb, uint32_t first, uint64_t count,
-                                            uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st) {
-  eval_kernel<BF_NT><<<grid, kThreads, 0, st>>>(tb, first, count, ms, fe);
+static unsigned blocks_for(const Plan& plan) {
+  const uint64_t warps = (uint64_t)plan.p_hi - plan.p_lo + 1;
+  return (unsigned)((warps + kWarps - 1) / kWarps);
+}
+
+cudaError_t BF_PASTE(launch_eval_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
+                                            uint32_t* ms, uint8_t* fe, cudaStream_t st) {
+  eval_kernel<<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, ms, fe);
   return cudaGetLastError();
 }
 
-cudaError_t BF_PASTE(launch_search_nt, BF_NT)(const Tables& tb, uint32_t first, uint64_t count,
-                                              uint32_t per_thread, unsigned long long* key,
-                                              cudaStream_t st) {
-  const uint64_t threads = (count + per_thread - 1) / per_thread;
-  const uint64_t blocks = (threads + kThreads - 1) / kThreads;
-  search_kernel<BF_NT><<<(unsigned)blocks, kThreads, 0, st>>>(tb, first, count, per_thread, key);
+cudaError_t BF_PASTE(launch_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
+                                              unsigned long long* key, cudaStream_t st) {
+  search_kernel<<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, key);
   return cudaGetLastError();
 }
 
-cudaError_t BF_PASTE(launch_batch_nt, BF_NT)(const Tables* d_tables, uint32_t count,
-                                             uint32_t per_thread, uint32_t blocks_per_scenario,
-                                             unsigned long long* keys, cudaStream_t st) {
+cudaError_t BF_PASTE(launch_batch_nw, BF_NW)(const BatchRecord* d_recs, uint32_t count,
+                                             uint32_t blocks_per_scenario, unsigned long long* keys,
+                                             cudaStream_t st) {
   const uint64_t blocks = (uint64_t)count * blocks_per_scenario;
-  batch_kernel<BF_NT><<<(unsigned)blocks, kThreads, 0, st>>>(d_tables, per_thread,
-                                                              blocks_per_scenario, keys);
+  batch_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(d_recs, blocks_per_scenario, keys);
   return cudaGetLastError();
 }
 

@@ -1,28 +1,38 @@
-// bf_sim.cuh -- device-side simulation of one mapping under the integer
-// latency model (version 1) declared in include/bf.h.
+// bf_sim.cuh -- device-side simulation of mappings under the integer latency
+// model (version 1) declared in include/bf.h.
 //
-// The model (paper §2.1 problem statement; Factor A/B of §2.3; Table 1's
-// gpu_queue = GPU + Load) is restated in bf.h.  This file is the GB300 form of
-// it: every per-tool quantity of one simulated mapping lives in registers
-// (fully unrolled loops over a compile-time tool count NT >= n), the tool
-// tables come from the kernel-parameter constant bank (or shared memory in
-// the batched kernel), and everything is 32-bit integer arithmetic except
-// two 32x32->64 products per event.
+// The model (paper §2.1 problem statement; Factors A and B of §2.3; Table 1's
+// gpu_queue = GPU + Load) is restated in bf.h.  This file is its GB300 form:
+// every per-tool quantity of a simulated mapping lives in registers (fully
+// unrolled loops over a compile-time slot count NT >= n), tool tables come
+// from the kernel-parameter constant bank (or shared memory in the batched
+// kernel), and all arithmetic is 32-bit integer except two 32x32->64
+// products per event.
 //
 // Representation (all exact):
 //   * Real time T and CPU end times: u32 microseconds (the scenario validator
 //     guarantees every event time fits).
-//   * Virtual GPU clock V and GPU end stamps `eg[i]`: kept modulo 2^32.  A
+//   * Virtual GPU clock V and GPU end stamps eg[i]: kept modulo 2^32.  A
 //     running GPU tool always has 0 <= vend - V < 2^32 (its whole work is
 //     < 2^32 units), so the u32 difference eg[i] - V is its exact remaining
-//     work and eg[i] == V exactly when it ends.
+//     work and eg[i] == V exactly when it ends.  `gmin` is the stamp of the
+//     running GPU tool that ends first; processor sharing runs every GPU tool
+//     at the same rate, so it only changes when GPU tools start or end.
 //   * The floor division of a CPU event, floor(dt * 2^20 / f[k]) with
-//     dt * 2^20 < 2^52, uses a per-k reciprocal (Granlund & Montgomery, "Division
-//     by invariant integers using multiplication", PLDI 1994, Thm 4.2):
-//     m = ceil(2^(52+l) / f), l = max(12, ceil(log2 f)); q = umulhi(m, n) >> (l-12).
+//     dt * 2^20 < 2^52, uses a per-k reciprocal (Granlund & Montgomery,
+//     "Division by invariant integers using multiplication", PLDI 1994,
+//     Thm 4.2): m = ceil(2^(52+l) / f), l = max(12, ceil(log2 f));
+//     q = umulhi(m, n) >> (l - 12).
 //   * A queued tool with m > M can never start, so such a mapping is rejected
-//     before simulating (the same verdict the model reaches when that tool
-//     becomes the queue head).
+//     before simulating (the verdict the model reaches when that tool becomes
+//     the queue head).
+//
+// Resumable runs.  run() can stop at the first admission at which a tool in
+// `stop_mask` would become ready, leaving the state exactly as it was after
+// that instant's retirements.  Until then no tool of stop_mask has started,
+// so the history does not depend on their modes: the search kernels simulate
+// the prefix tools once per warp up to that instant and resume from the saved
+// state for every combination of the remaining tools' modes.
 #pragma once
 
 #include <stdint.h>
@@ -31,13 +41,15 @@ namespace bfk {
 
 constexpr int kMaxTools = 20;
 constexpr uint32_t kInfeasible = 0xFFFFFFFFu;
-// Returned if the event loop ever exceeded its bound (each event retires at
+// Returned if a run ever exceeded its event bound (each event retires at
 // least one tool, so a correct simulation needs at most n events).  Scenario
 // validation keeps real makespans <= 0xFFFFFFFD, so this value never collides.
 constexpr uint32_t kStalled = 0xFFFFFFFEu;
 
-// Device-format scenario tables, passed by value as a __grid_constant__
-// kernel parameter (constant bank) or staged in shared memory.
+enum RunResult : uint32_t { kRunFinished = 0, kRunInfeasible = 1, kRunStopped = 2 };
+
+// Device-format scenario tables (per tool: index order), passed by value as a
+// __grid_constant__ kernel parameter (constant bank) or staged in shared memory.
 struct Tables {
   uint32_t n;
   uint32_t budget;       // M
@@ -52,6 +64,20 @@ struct Tables {
   uint32_t f[kMaxTools + 1];        // f[k]; f[0] unused
   uint32_t fshift[kMaxTools + 1];   // l - 12
   uint64_t fmagic[kMaxTools + 1];   // ceil(2^(52+l) / f[k])
+};
+
+// How a search splits the mapping index idx = p + 3^P * s:
+//   prefix p  -> the modes of tools [0, P), one per warp;
+//   suffix s  -> the modes of tools [P, n), spread over the warp's lanes.
+// Tools below W0 are done whenever the first suffix tool becomes ready (they
+// are ancestors of every suffix tool that can become ready first), so the
+// per-suffix simulation only carries the window [W0, n), renumbered from 0.
+struct Plan {
+  uint32_t P, K, W0;        // K = n - P
+  uint32_t pow3P, pow3K;
+  uint32_t p_lo, p_hi;      // prefixes this launch covers (inclusive)
+  uint32_t s_lo, s_hi;      // suffixes this launch covers (inclusive)
+  uint32_t first, last;     // canonical index range (inclusive)
 };
 
 // Tables read with a per-thread (dynamic) index, staged in shared memory:
@@ -79,72 +105,81 @@ struct Digits {
   uint32_t now, que;
 };
 
-template <int NT>
-__device__ __forceinline__ Digits decode(uint32_t idx) {
+// The low `digits` base-3 digits of v as masks (digits is a runtime count <= 20).
+__device__ __forceinline__ Digits decode(uint32_t v, uint32_t digits) {
   Digits d{0u, 0u};
 #pragma unroll
-  for (int i = 0; i < NT; ++i) {
-    const uint32_t q = idx / 3u;
-    const uint32_t r = idx - 3u * q;
+  for (uint32_t i = 0; i < (uint32_t)kMaxTools; ++i) {
+    if (i >= digits) break;
+    const uint32_t q = v / 3u;
+    const uint32_t r = v - 3u * q;
     d.now |= (r == 1u) ? (1u << i) : 0u;
     d.que |= (r == 2u) ? (1u << i) : 0u;
-    idx = q;
+    v = q;
   }
   return d;
 }
 
-// idx -> idx + 1 on the two masks: trailing 2-digits wrap to 0, the next digit
-// steps 0->1 or 1->2.
-__device__ __forceinline__ void increment(Digits& d) {
-  const uint32_t low = ~d.que & (d.que + 1u);  // lowest digit that is not 2
-  d.que &= ~(low - 1u);
-  const uint32_t had = d.now & low;
-  d.now ^= low;
-  d.que |= had;
-}
-
-// Makespan of one mapping (kInfeasible if infeasible).  `TB` is the tables'
-// storage (constant-bank parameter or shared memory).
-template <int NT, typename TB>
-__device__ __forceinline__ uint32_t simulate(const TB& tb, const SmemTables& sd, Digits dg) {
-  if (dg.que & tb.big_mask) return kInfeasible;
-  const uint32_t cpu_mask = tb.all_mask & ~(dg.now | dg.que);
-
-  uint32_t ec[NT];   // end time of a running CPU tool, else 0xFFFFFFFF
+// Simulation state over NT slots.
+template <int NT>
+struct State {
+  uint32_t ec[NT];   // running CPU tool: real end time; otherwise 0xFFFFFFFF
   uint32_t eg[NT];   // running GPU tool: virtual end stamp; waiting queued tool: ready time
+  uint32_t done;     // retired tools (slots >= n count as done)
+  uint32_t pend;     // not yet ready
+  uint32_t run_g;    // running GPU tools
+  uint32_t qwait;    // queued tools waiting
+  uint32_t qrun;     // the running queued tool (0 or one bit)
+  uint32_t cand;     // tools that may have become ready at T (successors of the last retirees)
+  uint32_t T, V, L, k;
+  uint32_t tc;       // earliest CPU end (0xFFFFFFFF if none)
+  uint32_t gmin;     // stamp of the first GPU tool to end (valid when k > 0)
+};
+
+template <int NT>
+__device__ __forceinline__ void init_state(State<NT>& s, uint32_t all_mask) {
 #pragma unroll
   for (int i = 0; i < NT; ++i) {
-    ec[i] = 0xFFFFFFFFu;
-    eg[i] = 0u;
+    s.ec[i] = 0xFFFFFFFFu;
+    s.eg[i] = 0u;
   }
-  uint32_t done = ~tb.all_mask;  // tools >= n count as done
-  uint32_t pend = tb.all_mask;   // not yet ready
-  uint32_t run_g = 0u;           // running GPU tools
-  uint32_t qwait = 0u;           // queued tools waiting
-  uint32_t qrun = 0u;            // the running queued tool (0 or one bit)
-  uint32_t T = 0u, V = 0u, L = 0u, k = 0u;
-  uint32_t tc = 0xFFFFFFFFu;     // earliest CPU end
+  s.done = ~all_mask;
+  s.pend = all_mask;
+  s.run_g = s.qwait = s.qrun = 0u;
+  s.cand = all_mask;  // at T = 0 every tool is a candidate
+  s.T = s.V = s.L = s.k = 0u;
+  s.tc = 0xFFFFFFFFu;
+  s.gmin = 0u;
+}
 
-  // Candidate tools for readiness are the successors of retired tools; at
-  // T = 0 every tool is a candidate.
-  uint32_t cand = tb.all_mask;
-
+// Advance `s` under modes `dg` until every tool is done (kRunFinished, the
+// makespan is s.T), the mapping proves infeasible (kRunInfeasible), or a tool
+// of `stop_mask` would become ready (kRunStopped, state left before that
+// admission).  A stalled run reports kRunFinished with s.T = kStalled.
+template <int NT, typename TB>
+__device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTables& sd, Digits dg,
+                                        uint32_t stop_mask) {
+  const uint32_t cpu_mask = tb.all_mask & ~(dg.now | dg.que);
 #pragma unroll 1
   for (uint32_t events = 0;; ++events) {
-    if (events > (uint32_t)NT) return kStalled;
-    // ---- admission at T -------------------------------------------------
+    if (events > (uint32_t)NT + 1u) {
+      s.T = kStalled;
+      return kRunFinished;
+    }
+    // ---- admission at T ---------------------------------------------------
     uint32_t ready = 0u;
     {
-      uint32_t c = cand & pend;
-      const uint32_t notdone = ~done;
+      uint32_t c = s.cand & s.pend;
+      const uint32_t notdone = ~s.done;
       while (c) {
         const int v = __ffs(c) - 1;
         c &= c - 1u;
         if ((sd.pred[v] & notdone) == 0u) ready |= 1u << v;
       }
     }
+    if (ready & stop_mask) return kRunStopped;
     if (ready) {
-      pend &= ~ready;
+      s.pend &= ~ready;
       const uint32_t rc = ready & cpu_mask;
       const uint32_t rg = ready & dg.now;
       const uint32_t rq = ready & dg.que;
@@ -152,112 +187,170 @@ __device__ __forceinline__ uint32_t simulate(const TB& tb, const SmemTables& sd,
 #pragma unroll
         for (int i = 0; i < NT; ++i) {
           if (rc & (1u << i)) {
-            ec[i] = T + tb.cpu[i];
-            tc = min(tc, ec[i]);
+            s.ec[i] = s.T + tb.cpu[i];
+            s.tc = min(s.tc, s.ec[i]);
           }
         }
       }
       if (rg) {
+        uint32_t wmin = 0xFFFFFFFFu;
 #pragma unroll
         for (int i = 0; i < NT; ++i) {
           if (rg & (1u << i)) {
-            eg[i] = V + tb.wnow[i];
-            L += tb.vram[i];
+            s.eg[i] = s.V + tb.wnow[i];
+            s.L += tb.vram[i];
+            wmin = min(wmin, tb.wnow[i]);
           }
         }
-        run_g |= rg;
-        k += __popc(rg);
-        if (L > tb.budget) return kInfeasible;
+        if (s.k == 0u || wmin < s.gmin - s.V) s.gmin = s.V + wmin;
+        s.run_g |= rg;
+        s.k += __popc(rg);
+        if (s.L > tb.budget) return kRunInfeasible;
       }
       if (rq) {
 #pragma unroll
         for (int i = 0; i < NT; ++i)
-          if (rq & (1u << i)) eg[i] = T;
-        qwait |= rq;
+          if (rq & (1u << i)) s.eg[i] = s.T;
+        s.qwait |= rq;
       }
     }
-    if (qwait && !qrun) {
+    if (s.qwait && !s.qrun) {
       // Queue head: earliest ready time, ties to the lower index.
       uint32_t best = 0xFFFFFFFFu, hm = 0u, hv = 0u, hw = 0u;
 #pragma unroll
       for (int i = 0; i < NT; ++i) {
-        if ((qwait & (1u << i)) && eg[i] < best) {
-          best = eg[i];
+        if ((s.qwait & (1u << i)) && s.eg[i] < best) {
+          best = s.eg[i];
           hm = 1u << i;
           hv = tb.vram[i];
           hw = tb.wq[i];
         }
       }
-      if (L + hv <= tb.budget) {
+      if (s.L + hv <= tb.budget) {
 #pragma unroll
         for (int i = 0; i < NT; ++i)
-          if (hm & (1u << i)) eg[i] = V + hw;
-        L += hv;
-        k += 1u;
-        run_g |= hm;
-        qrun = hm;
-        qwait &= ~hm;
+          if (hm & (1u << i)) s.eg[i] = s.V + hw;
+        if (s.k == 0u || hw < s.gmin - s.V) s.gmin = s.V + hw;
+        s.L += hv;
+        s.k += 1u;
+        s.run_g |= hm;
+        s.qrun = hm;
+        s.qwait &= ~hm;
       }
     }
-    if (done == 0xFFFFFFFFu) break;
+    if (s.done == 0xFFFFFFFFu) return kRunFinished;
 
-    // ---- next event -------------------------------------------------------
-    uint32_t rem = 0xFFFFFFFFu;  // remaining work of the first GPU tool to end
-#pragma unroll
-    for (int i = 0; i < NT; ++i)
-      if (run_g & (1u << i)) rem = min(rem, eg[i] - V);
-    const uint32_t kk = min(k, (uint32_t)kMaxTools);  // k <= n always; the clamp keeps indexing in bounds
-    uint64_t tg = 0xFFFFFFFFFFFFFFFFull;
-    if (k) {
-      const uint64_t prod = (uint64_t)rem * sd.f[kk];
-      tg = (uint64_t)T + ((prod + 0xFFFFFull) >> 20);
-    }
-    bool gpu_event;
-    if (tg <= (uint64_t)tc) {
-      T = (uint32_t)tg;
-      V += rem;
-      gpu_event = true;
+    // ---- next event ---------------------------------------------------------
+    const uint32_t kk = min(s.k, (uint32_t)kMaxTools);  // k <= n always; keeps indexing in bounds
+    bool gpu_event = false;
+    if (s.k) {
+      const uint32_t rem = s.gmin - s.V;
+      const uint64_t tg = (uint64_t)s.T + (((uint64_t)rem * sd.f[kk] + 0xFFFFFull) >> 20);
+      if (tg <= (uint64_t)s.tc) {
+        s.T = (uint32_t)tg;
+        s.V = s.gmin;
+        gpu_event = true;
+      } else {
+        const uint64_t num = (uint64_t)(s.tc - s.T) << 20;
+        s.V += (uint32_t)(__umul64hi(sd.magic[kk], num) >> sd.shift[kk]);
+        s.T = s.tc;
+      }
     } else {
-      if (k) {
-        const uint64_t num = (uint64_t)(tc - T) << 20;
-        V += (uint32_t)(__umul64hi(sd.magic[kk], num) >> sd.shift[kk]);
-      }
-      T = tc;
-      gpu_event = false;
+      s.T = s.tc;
     }
 
-    // ---- retire everything that ends at T ----------------------------------
-    cand = 0u;
-    if (tc == T) {
+    // ---- retire everything that ends at T ------------------------------------
+    s.cand = 0u;
+    if (s.tc == s.T) {
       uint32_t ntc = 0xFFFFFFFFu;
 #pragma unroll
       for (int i = 0; i < NT; ++i) {
-        if (ec[i] == T) {
-          ec[i] = 0xFFFFFFFFu;
-          done |= 1u << i;
-          cand |= tb.succ[i];
+        if (s.ec[i] == s.T) {
+          s.ec[i] = 0xFFFFFFFFu;
+          s.done |= 1u << i;
+          s.cand |= tb.succ[i];
         }
-        ntc = min(ntc, ec[i]);
+        ntc = min(ntc, s.ec[i]);
       }
-      tc = ntc;
+      s.tc = ntc;
     }
     if (gpu_event) {
-      uint32_t rg = 0u;
+      uint32_t rg = 0u, nrem = 0xFFFFFFFFu;
 #pragma unroll
       for (int i = 0; i < NT; ++i) {
-        if ((run_g & (1u << i)) && eg[i] == V) {
-          rg |= 1u << i;
-          L -= tb.vram[i];
-          cand |= tb.succ[i];
+        if (s.run_g & (1u << i)) {
+          if (s.eg[i] == s.V) {
+            rg |= 1u << i;
+            s.L -= tb.vram[i];
+            s.cand |= tb.succ[i];
+          } else {
+            nrem = min(nrem, s.eg[i] - s.V);
+          }
         }
       }
-      run_g &= ~rg;
-      done |= rg;
-      k -= __popc(rg);
-      if (rg & qrun) qrun = 0u;
+      s.run_g &= ~rg;
+      s.done |= rg;
+      s.k -= __popc(rg);
+      if (rg & s.qrun) s.qrun = 0u;
+      s.gmin = s.V + nrem;
     }
   }
-  return T;
+}
+
+// ---- saved state of a warp's prefix, restricted to the window [W0, n) --------
+// Stored once per warp in shared memory (every lane of the warp holds the same
+// prefix state) and reloaded by each lane for every suffix.
+struct Snapshot {
+  uint32_t ec[kMaxTools];
+  uint32_t eg[kMaxTools];
+  uint32_t done, pend, run_g, qwait, qrun, cand;
+  uint32_t T, V, L, k, tc, gmin;
+};
+
+// Save the window part of a full-width prefix state (slots >= W0, renumbered).
+template <int NT>
+__device__ __forceinline__ void save_window(const State<NT>& s, uint32_t W0, uint32_t nw, Snapshot& out) {
+#pragma unroll
+  for (int i = 0; i < NT; ++i) {
+    if ((uint32_t)i >= W0) {
+      out.ec[i - W0] = s.ec[i];
+      out.eg[i - W0] = s.eg[i];
+    }
+  }
+  const uint32_t wmask = (nw >= 32u) ? 0xFFFFFFFFu : ((1u << nw) - 1u);
+  out.done = (s.done >> W0) | ~wmask;
+  out.pend = (s.pend >> W0) & wmask;
+  out.run_g = s.run_g >> W0;
+  out.qwait = s.qwait >> W0;
+  out.qrun = s.qrun >> W0;
+  out.cand = (s.cand >> W0) & wmask;
+  out.T = s.T;
+  out.V = s.V;
+  out.L = s.L;
+  out.k = s.k;
+  out.tc = s.tc;
+  out.gmin = s.gmin;
+}
+
+template <int NW>
+__device__ __forceinline__ void load_window(const Snapshot& in, State<NW>& s) {
+#pragma unroll
+  for (int i = 0; i < NW; ++i) {
+    s.ec[i] = in.ec[i];
+    s.eg[i] = in.eg[i];
+  }
+  s.done = in.done;
+  s.pend = in.pend;
+  s.run_g = in.run_g;
+  s.qwait = in.qwait;
+  s.qrun = in.qrun;
+  s.cand = in.cand;
+  s.T = in.T;
+  s.V = in.V;
+  s.L = in.L;
+  s.k = in.k;
+  s.tc = in.tc;
+  s.gmin = in.gmin;
 }
 
 }  // namespace bfk

@@ -1,0 +1,66 @@
+"""Run one kernel of the search on a chosen range, for timing and profiling.
+
+  python -m paper_2607_22242_gb300.profile_case --kernel search --config 3 --count 67108864 --reps 3
+  python -m paper_2607_22242_gb300.profile_case --kernel eval --config 2 --count 16777216
+  python -m paper_2607_22242_gb300.profile_case --kernel batch --batch 1024
+
+Prints one line per repetition (CUDA-event time of the call and mappings/s).
+Sized so that a profiler capture of one launch stays short.
+"""
+from __future__ import annotations
+
+import argparse
+import os
+import sys
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--kernel", choices=("search", "eval", "batch"), default="search")
+    ap.add_argument("--config", type=int, default=3)
+    ap.add_argument("--first", type=int, default=0)
+    ap.add_argument("--count", type=int, default=1 << 26)
+    ap.add_argument("--batch", type=int, default=1024, help="scenarios for --kernel batch (config 4 prefix)")
+    ap.add_argument("--reps", type=int, default=3)
+    args = ap.parse_args()
+
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2607_22242_gb300 import bf
+    from paper_2607_22242_gb300 import scenarios as S
+
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream()
+    if args.kernel == "batch":
+        batch = S.config4(args.batch)
+        work = len(batch) * 3 ** 10
+        call = lambda: bf.search_batch(batch, stream)
+    else:
+        scn = S.config(args.config)
+        count = min(args.count, 3 ** scn.n - args.first)
+        work = count
+        h = bf.create_scenario(scn)
+        if args.kernel == "search":
+            call = lambda: bf.search_range(h, args.first, count, stream)
+        else:
+            ms = torch.empty(count, dtype=torch.int32, device="cuda")
+            fe = torch.empty(count, dtype=torch.uint8, device="cuda")
+            call = lambda: bf.eval_mappings(h, args.first, count, ms, fe, stream)
+    for rep in range(args.reps):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        out = call()
+        b.record(stream)
+        b.synchronize()
+        t = a.elapsed_time(b)
+        print(f"{args.kernel} rep {rep}: {t:.3f} ms, {work / (t / 1e3):.4g} mappings/s"
+              + (f", best {out.index}/{out.makespan_us}" if args.kernel == "search" else ""), flush=True)
+
+
+if __name__ == "__main__":
+    main()
