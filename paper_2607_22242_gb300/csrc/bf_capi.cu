@@ -20,7 +20,7 @@ struct bf_scenario {
   bf_scenario_desc desc;
   bfk::Tables tables;   // all n tools
   bfk::Tables window;   // tools [W0, n), renumbered from 0
-  uint32_t P, K, W0;    // index split and window start (see bfk::Plan)
+  bfk::Plan plan;       // enumeration split and window (see bfk::Plan), full range
   int device;
   unsigned long long* d_key;  // device scratch: one packed search key
   unsigned long long* h_key;  // pinned host copy of it
@@ -165,7 +165,7 @@ int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result
   cudaError_t e = cudaMemsetAsync(scn->d_key, 0xFF, sizeof(unsigned long long), st);
   if (e != cudaSuccess) return cuda_fail(e, who);
   if (count) {
-    const bfk::Plan plan = make_plan(scn->desc.n, scn->P, scn->K, scn->W0, first, count);
+    const bfk::Plan plan = make_plan(scn->plan, first, count);
 #define CALL(NW) launch_search_nw##NW(scn->tables, scn->window, plan, scn->d_key, st)
     BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
 #undef CALL
@@ -194,7 +194,7 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   std::memset(s, 0, sizeof *s);
   s->desc = *desc;
   build_tables(desc, &s->tables);
-  split_and_window(s->tables, &s->P, &s->K, &s->W0, &s->window);
+  split_and_window(s->tables, &s->plan, &s->window);
   cudaError_t e = cudaGetDevice(&s->device);
   if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_key), sizeof(unsigned long long));
   if (e == cudaSuccess) e = lib_malloc_host(reinterpret_cast<void**>(&s->h_key), sizeof(unsigned long long));
@@ -228,7 +228,7 @@ int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count, uin
   if (count == 0) return BF_OK;
   if (!d_makespan || !d_feasible) return fail(BF_EINVAL, "bf_eval_mappings: NULL output buffer");
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  const bfk::Plan plan = make_plan(scn->desc.n, scn->P, scn->K, scn->W0, first, count);
+  const bfk::Plan plan = make_plan(scn->plan, first, count);
   cudaError_t e = cudaSuccess;
 #define CALL(NW) launch_eval_nw##NW(scn->tables, scn->window, plan, d_makespan, d_feasible, st)
   BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
@@ -267,9 +267,9 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
     bfk::BatchRecord& r = recs[i];
     std::memset(&r, 0, sizeof r);
     build_tables(descs + i, &r.full);
-    uint32_t P, K, W0;
-    split_and_window(r.full, &P, &K, &W0, &r.window);
-    r.plan = make_plan(descs[i].n, P, K, W0, 0, pow3(descs[i].n));
+    bfk::Plan base;
+    split_and_window(r.full, &base, &r.window);
+    r.plan = make_plan(base, 0, pow3(descs[i].n));
     if (r.window.n > wmax) wmax = r.window.n;
     if (r.plan.pow3P > pmax) pmax = r.plan.pow3P;
   }

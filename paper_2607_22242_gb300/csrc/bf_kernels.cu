@@ -2,14 +2,16 @@
 // (-DBF_NW=<slots>).  All integer ALU work: no tensor cores, and no HBM
 // streaming beyond the eval kernel's 5 bytes of output per mapping.
 //
-// Work decomposition (the same in all three kernels).  A mapping index is
-// idx = p + 3^P * s.  Each warp owns one prefix p (the modes of tools
-// [0, P)); its 32 lanes simulate that prefix together -- identical control
-// flow -- until the first instant a suffix tool (index >= P) would become
+// Work decomposition (the same in all three kernels; see bfk::Plan).  A
+// mapping index is idx = p + 3^P * (m + 3^M * i).  Each warp owns one prefix
+// p (the modes of tools [0, P)); its 32 lanes simulate that prefix together --
+// identical control flow -- until the first instant a tool >= P would become
 // ready, and lane 0 saves the state (restricted to the window [W0, n)) in
-// shared memory.  Then lane l resumes that state for suffixes s = l, l+32, ...
-// with a simulation only NW slots wide.  Every mapping's makespan is still
-// simulated event by event; only the common prefix of its history is shared.
+// shared memory.  Lane l then resumes it for mid combinations m = l, l+32, ...
+// with a simulation only NW slots wide; with an inner level it saves its own
+// state again when the first inner tool would become ready and resumes that
+// for each inner combination i.  Every mapping's makespan is still simulated
+// event by event; only the common part of the histories is shared.
 //
 //   eval   : writes the makespan (u32) and feasibility flag (u8) of every
 //            mapping in [first, last] -- §2.1's T_e2e per mapping.
@@ -19,6 +21,7 @@
 //            the brute-force oracle of §2.3 / §4.1 under the integer model.
 //   batch  : as search, for many independent scenarios in one launch; each
 //            block stages its scenario's tables and plan in shared memory.
+#include "bf_enum.cuh"
 #include "bf_launch.h"
 
 #ifndef BF_NW
@@ -51,38 +54,6 @@ __device__ __forceinline__ void block_min_to(unsigned long long v, unsigned long
   }
 }
 
-// Simulate prefix p once per warp and save its window state in `snap`.
-// Returns false (warp-uniformly) when every mapping with this prefix is
-// infeasible.
-template <typename TB>
-__device__ __forceinline__ bool prefix_phase(const TB& tb, const SmemTables& sd, const Plan& plan,
-                                             uint32_t p, Digits& dgp, Snapshot& snap) {
-  dgp = decode(p, plan.P);
-  bool ok = (dgp.que & tb.big_mask) == 0u;
-  if (ok) {
-    State<kMaxTools> s;
-    init_state(s, tb.all_mask);
-    const uint32_t suffix_mask = tb.all_mask & ~((1u << plan.P) - 1u);
-    ok = run<kMaxTools>(s, tb, sd, dgp, suffix_mask) == kRunStopped;
-    if (ok && (threadIdx.x & 31) == 0) save_window(s, plan.W0, tb.n - plan.W0, snap);
-  }
-  __syncwarp();
-  return ok;
-}
-
-// Makespan of mapping (p, s) resumed from the warp's snapshot.
-template <typename TB>
-__device__ __forceinline__ uint32_t suffix_makespan(const TB& tw, const SmemTables& sdw, const Plan& plan,
-                                                    Digits dgp, uint32_t s, const Snapshot& snap) {
-  const Digits dgs = decode(s, plan.K);
-  const uint32_t sh = plan.P - plan.W0;
-  const Digits dw{(dgp.now >> plan.W0) | (dgs.now << sh), (dgp.que >> plan.W0) | (dgs.que << sh)};
-  if (dw.que & tw.big_mask) return kInfeasible;
-  State<BF_NW> w;
-  load_window(snap, w);
-  return run<BF_NW>(w, tw, sdw, dw, 0u) == kRunFinished ? w.T : kInfeasible;
-}
-
 __global__ void __launch_bounds__(kThreads) eval_kernel(const __grid_constant__ Tables tb,
                                                         const __grid_constant__ Tables tw,
                                                         const __grid_constant__ Plan plan,
@@ -90,22 +61,18 @@ __global__ void __launch_bounds__(kThreads) eval_kernel(const __grid_constant__ 
                                                         uint8_t* __restrict__ fe_out) {
   __shared__ SmemTables sd, sdw;
   __shared__ Snapshot snap[kWarps];
+  __shared__ uint32_t lane_state[LaneWords<BF_NW>::value * kThreads];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
   __syncthreads();
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int warp = threadIdx.x >> 5;
   const uint64_t p64 = (uint64_t)plan.p_lo + (uint64_t)blockIdx.x * kWarps + warp;
   if (p64 > plan.p_hi) return;  // no block-level synchronisation follows
   const uint32_t p = (uint32_t)p64;
   Digits dgp;
   const bool ok = prefix_phase(tb, sd, plan, p, dgp, snap[warp]);
-  for (uint32_t s = plan.s_lo + lane; s <= plan.s_hi; s += 32) {
-    const uint32_t idx = p + plan.pow3P * s;
-    if (idx < plan.first || idx > plan.last) continue;
-    const uint32_t ms = ok ? suffix_makespan(tw, sdw, plan, dgp, s, snap[warp]) : kInfeasible;
-    ms_out[idx - plan.first] = ms;
-    fe_out[idx - plan.first] = ms != kInfeasible;
-  }
+  StoreSink sink{plan.first, ms_out, fe_out};
+  lane_mappings<BF_NW>(tw, sdw, plan, p, ok, dgp, snap[warp], lane_state + threadIdx.x, kThreads, sink);
 }
 
 __global__ void __launch_bounds__(kThreads) search_kernel(const __grid_constant__ Tables tb,
@@ -114,34 +81,29 @@ __global__ void __launch_bounds__(kThreads) search_kernel(const __grid_constant_
                                                           unsigned long long* key) {
   __shared__ SmemTables sd, sdw;
   __shared__ Snapshot snap[kWarps];
+  __shared__ uint32_t lane_state[LaneWords<BF_NW>::value * kThreads];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
   __syncthreads();
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int warp = threadIdx.x >> 5;
   const uint64_t p64 = (uint64_t)plan.p_lo + (uint64_t)blockIdx.x * kWarps + warp;
-  unsigned long long best = ~0ull;
+  MinKeySink sink;
   if (p64 <= plan.p_hi) {
     const uint32_t p = (uint32_t)p64;
     Digits dgp;
-    if (prefix_phase(tb, sd, plan, p, dgp, snap[warp])) {
-      for (uint32_t s = plan.s_lo + lane; s <= plan.s_hi; s += 32) {
-        const uint32_t idx = p + plan.pow3P * s;
-        if (idx < plan.first || idx > plan.last) continue;
-        const uint32_t ms = suffix_makespan(tw, sdw, plan, dgp, s, snap[warp]);
-        best = min(best, ((unsigned long long)ms << 32) | idx);
-      }
-    }
+    if (prefix_phase(tb, sd, plan, p, dgp, snap[warp])) lane_mappings<BF_NW>(tw, sdw, plan, p, true, dgp, snap[warp], lane_state + threadIdx.x, kThreads, sink);
   }
-  block_min_to(best, key);
+  block_min_to(sink.best, key);
 }
 
 // One record per scenario of a batch: full tables, window tables and plan.
-__global__ void __launch_bounds__(kThreads) batch_kernel(const BatchRecord* __restrict__ recs,
+__global__ void __launch_bounds__(kThreads, 2) batch_kernel(const BatchRecord* __restrict__ recs,
                                                          uint32_t blocks_per_scenario,
                                                          unsigned long long* keys) {
   __shared__ BatchRecord rec;
   __shared__ SmemTables sd, sdw;
   __shared__ Snapshot snap[kWarps];
+  __shared__ uint32_t lane_state[LaneWords<BF_NW>::value * kThreads];
   const uint32_t sc = blockIdx.x / blocks_per_scenario;
   const uint32_t b = blockIdx.x - sc * blocks_per_scenario;
   {
@@ -153,21 +115,17 @@ __global__ void __launch_bounds__(kThreads) batch_kernel(const BatchRecord* __re
   load_smem_tables(rec.full, sd);
   load_smem_tables(rec.window, sdw);
   __syncthreads();
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  const int warp = threadIdx.x >> 5;
   const uint64_t p64 = (uint64_t)rec.plan.p_lo + (uint64_t)b * kWarps + warp;
-  unsigned long long best = ~0ull;
+  MinKeySink sink;
   if (p64 <= rec.plan.p_hi) {
     const uint32_t p = (uint32_t)p64;
     Digits dgp;
-    if (prefix_phase(rec.full, sd, rec.plan, p, dgp, snap[warp])) {
-      for (uint32_t s = rec.plan.s_lo + lane; s <= rec.plan.s_hi; s += 32) {
-        const uint32_t idx = p + rec.plan.pow3P * s;
-        const uint32_t ms = suffix_makespan(rec.window, sdw, rec.plan, dgp, s, snap[warp]);
-        best = min(best, ((unsigned long long)ms << 32) | idx);
-      }
-    }
+    if (prefix_phase(rec.full, sd, rec.plan, p, dgp, snap[warp]))
+      lane_mappings<BF_NW>(rec.window, sdw, rec.plan, p, true, dgp, snap[warp], lane_state + threadIdx.x,
+                           kThreads, sink);
   }
-  block_min_to(best, keys + sc);
+  block_min_to(sink.best, keys + sc);
 }
 
 }  // namespace

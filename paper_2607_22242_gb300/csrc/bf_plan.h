@@ -52,35 +52,64 @@ inline void build_tables(const bf_scenario_desc* d, bfk::Tables* t) {
   t->fmagic[0] = 1ull << 54;
 }
 
-// Number of suffix tools K (their modes vary across a warp's lanes): large
+// Number of mid tools M (their modes vary across a warp's lanes): large
 // enough to keep 32 lanes busy, small enough to leave many prefixes (warps).
-inline uint32_t suffix_tools(uint32_t n) {
-  if (n >= 13) return 6;   // 729 suffixes: 23 rounds of 32 lanes, 1% idle
-  if (n >= 9) return 5;    // 243 suffixes
-  if (n >= 4) return 4;    // 81 suffixes
+inline uint32_t mid_tools(uint32_t n) {
+  if (n >= 13) return 6;   // 729 combinations: 23 rounds of 32 lanes, 1% idle
+  if (n >= 9) return 5;    // 243 combinations
+  if (n >= 4) return 4;    // 81 combinations
   return n;
 }
 
-// Split the tools at P = n - K and find the window start W0: the tools that
-// every "suffix source" (a tool >= P whose predecessors are all < P) depends
-// on, transitively, are done by the time the first suffix tool becomes ready
-// (that tool is a suffix source).  W0 is the lowest tool outside that set.
-inline void split_and_window(const bfk::Tables& t, uint32_t* P, uint32_t* K, uint32_t* W0, bfk::Tables* w) {
+// Tools that are certainly done when the first tool of [from, n) becomes
+// ready: the common ancestors of the "sources" of that range (tools >= from
+// whose predecessors are all < from); the first tool of the range to become
+// ready is one of them.
+inline uint32_t done_when_first_ready(const uint32_t* anc, const bfk::Tables& t, uint32_t from) {
+  const uint32_t below = (from >= 32) ? ~0u : ((1u << from) - 1u);
+  uint32_t done = below;
+  for (uint32_t v = from; v < t.n; ++v)
+    if ((t.pred[v] & ~below) == 0u) done &= anc[v];
+  return done;
+}
+
+// Choose P, M, I and the window start W0 for a scenario, and fill the window
+// tables (tools [W0, n) renumbered from 0).
+inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
   const uint32_t n = t.n;
-  *K = suffix_tools(n);
-  *P = n - *K;
-  const uint32_t prefix_mask = (*P >= 32) ? ~0u : ((1u << *P) - 1u);
   uint32_t anc[BF_MAX_TOOLS];
-  uint32_t done_at_split = prefix_mask;
   for (uint32_t v = 0; v < n; ++v) {
     anc[v] = t.pred[v];
     for (uint32_t u = 0; u < v; ++u)
       if (t.pred[v] & (1u << u)) anc[v] |= anc[u];
-    if (v >= *P && (t.pred[v] & ~prefix_mask) == 0u) done_at_split &= anc[v];
   }
+  const uint32_t M = mid_tools(n);
+  uint32_t I = 0;
+  if (n >= M + 1) {
+    // One inner tool pays off when most of the window is done before it can
+    // start: then each lane's second snapshot saves most of the events.
+    const uint32_t P1 = n - M - 1, Q = n - 1;
+    const uint32_t d0 = done_when_first_ready(anc, t, P1);
+    uint32_t w0 = 0;
+    while (w0 < P1 && (d0 & (1u << w0))) ++w0;
+    const uint32_t dq = done_when_first_ready(anc, t, Q);
+    const uint32_t span = Q - w0;
+    const uint32_t span_mask = ((Q >= 32) ? ~0u : ((1u << Q) - 1u)) & ~((1u << w0) - 1u);
+    const uint32_t saved = (uint32_t)__builtin_popcount(dq & span_mask);
+    if (saved >= 2 && 2 * saved >= span) I = 1;
+  }
+  const uint32_t P = n - M - I;
+  const uint32_t d = done_when_first_ready(anc, t, P);
   uint32_t w0 = 0;
-  while (w0 < *P && (done_at_split & (1u << w0))) ++w0;
-  *W0 = w0;
+  while (w0 < P && (d & (1u << w0))) ++w0;
+  std::memset(pl, 0, sizeof *pl);
+  pl->P = P;
+  pl->M = M;
+  pl->I = I;
+  pl->W0 = w0;
+  pl->pow3P = (uint32_t)pow3(P);
+  pl->pow3M = (uint32_t)pow3(M);
+  pl->pow3I = (uint32_t)pow3(I);
   std::memset(w, 0, sizeof *w);
   const uint32_t nw = n - w0;
   w->n = nw;
@@ -102,28 +131,23 @@ inline void split_and_window(const bfk::Tables& t, uint32_t* P, uint32_t* K, uin
   }
 }
 
-// Plan covering canonical indices [first, first+count), count >= 1.
-inline bfk::Plan make_plan(uint32_t n, uint32_t P, uint32_t K, uint32_t W0, uint64_t first, uint64_t count) {
-  bfk::Plan pl;
-  std::memset(&pl, 0, sizeof pl);
-  pl.P = P;
-  pl.K = K;
-  pl.W0 = W0;
-  pl.pow3P = (uint32_t)pow3(P);
-  pl.pow3K = (uint32_t)pow3(K);
+// Restrict a scenario's plan to canonical indices [first, first+count), count >= 1.
+inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count) {
+  bfk::Plan pl = base;
   const uint64_t last = first + count - 1;
   pl.first = (uint32_t)first;
   pl.last = (uint32_t)last;
-  pl.s_lo = (uint32_t)(first / pl.pow3P);
-  pl.s_hi = (uint32_t)(last / pl.pow3P);
-  if (pl.s_lo == pl.s_hi) {
+  const uint64_t pm = (uint64_t)pl.pow3P * pl.pow3M;
+  pl.i_lo = (uint32_t)(first / pm);
+  pl.i_hi = (uint32_t)(last / pm);
+  const uint64_t s_lo = first / pl.pow3P, s_hi = last / pl.pow3P;
+  if (s_lo == s_hi) {
     pl.p_lo = (uint32_t)(first % pl.pow3P);
     pl.p_hi = (uint32_t)(last % pl.pow3P);
   } else {
     pl.p_lo = 0;
     pl.p_hi = pl.pow3P - 1;
   }
-  (void)n;
   return pl;
 }
 

@@ -66,17 +66,21 @@ struct Tables {
   uint64_t fmagic[kMaxTools + 1];   // ceil(2^(52+l) / f[k])
 };
 
-// How a search splits the mapping index idx = p + 3^P * s:
-//   prefix p  -> the modes of tools [0, P), one per warp;
-//   suffix s  -> the modes of tools [P, n), spread over the warp's lanes.
-// Tools below W0 are done whenever the first suffix tool becomes ready (they
-// are ancestors of every suffix tool that can become ready first), so the
-// per-suffix simulation only carries the window [W0, n), renumbered from 0.
+// How a search enumerates the mapping index idx = p + 3^P * (m + 3^M * i):
+//   prefix p -> the modes of tools [0, P), one per warp;
+//   mid m    -> the modes of tools [P, P+M), spread over the warp's lanes;
+//   inner i  -> the modes of the last I tools [Q, n), Q = P+M, walked by each lane.
+// The warp simulates its prefix once, up to the first instant a tool >= P
+// would become ready.  Tools below W0 are done by then (they are ancestors of
+// every tool >= P that can become ready first), so everything after that is
+// simulated over the window [W0, n) only, renumbered from 0.  With I > 0 each
+// lane saves its state again at the first instant an inner tool would become
+// ready and resumes it for every inner combination.
 struct Plan {
-  uint32_t P, K, W0;        // K = n - P
-  uint32_t pow3P, pow3K;
+  uint32_t P, M, I, W0;
+  uint32_t pow3P, pow3M, pow3I;
   uint32_t p_lo, p_hi;      // prefixes this launch covers (inclusive)
-  uint32_t s_lo, s_hi;      // suffixes this launch covers (inclusive)
+  uint32_t i_lo, i_hi;      // inner combinations this launch covers (inclusive)
   uint32_t first, last;     // canonical index range (inclusive)
 };
 
@@ -351,6 +355,58 @@ __device__ __forceinline__ void load_window(const Snapshot& in, State<NW>& s) {
   s.k = in.k;
   s.tc = in.tc;
   s.gmin = in.gmin;
+}
+
+// Per-lane copy of a window state in shared memory, one word per row of a
+// [word][thread] array (`stride` = threads per block), so that a warp's
+// accesses to the same word hit 32 different banks.
+template <int NW>
+struct LaneWords {
+  static constexpr int value = 2 * NW + 12;
+};
+
+template <int NW>
+__device__ __forceinline__ void save_lane(const State<NW>& s, uint32_t* slot, uint32_t stride) {
+#pragma unroll
+  for (int i = 0; i < NW; ++i) {
+    slot[(2 * i) * stride] = s.ec[i];
+    slot[(2 * i + 1) * stride] = s.eg[i];
+  }
+  uint32_t* t = slot + (2 * NW) * stride;
+  t[0 * stride] = s.done;
+  t[1 * stride] = s.pend;
+  t[2 * stride] = s.run_g;
+  t[3 * stride] = s.qwait;
+  t[4 * stride] = s.qrun;
+  t[5 * stride] = s.cand;
+  t[6 * stride] = s.T;
+  t[7 * stride] = s.V;
+  t[8 * stride] = s.L;
+  t[9 * stride] = s.k;
+  t[10 * stride] = s.tc;
+  t[11 * stride] = s.gmin;
+}
+
+template <int NW>
+__device__ __forceinline__ void load_lane(const uint32_t* slot, uint32_t stride, State<NW>& s) {
+#pragma unroll
+  for (int i = 0; i < NW; ++i) {
+    s.ec[i] = slot[(2 * i) * stride];
+    s.eg[i] = slot[(2 * i + 1) * stride];
+  }
+  const uint32_t* t = slot + (2 * NW) * stride;
+  s.done = t[0 * stride];
+  s.pend = t[1 * stride];
+  s.run_g = t[2 * stride];
+  s.qwait = t[3 * stride];
+  s.qrun = t[4 * stride];
+  s.cand = t[5 * stride];
+  s.T = t[6 * stride];
+  s.V = t[7 * stride];
+  s.L = t[8 * stride];
+  s.k = t[9 * stride];
+  s.tc = t[10 * stride];
+  s.gmin = t[11 * stride];
 }
 
 }  // namespace bfk
