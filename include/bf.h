@@ -152,6 +152,26 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
 int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                     void* cuda_stream);
 
+/* Largest batch bf_search_batch_noalloc accepts. */
+#define BF_NOALLOC_MAX_SCENARIOS 1024
+
+/* The batched search of bf_search_batch without any memory allocation.  The
+ * paper has no counterpart: this exists for callers that cannot allocate
+ * device memory at the moment they search -- e.g. a scheduler loop whose
+ * process has handed all GPU memory to another allocator's pool, or one that
+ * must not let cudaMalloc/cudaFree synchronise the device between rounds.
+ * The caller passes the inputs (descs) and outputs (out) as for
+ * bf_search_batch; the scratch (packed scenario records and one key per
+ * scenario, about 1.7 MiB for BF_NOALLOC_MAX_SCENARIOS) is a fixed array in
+ * the library's device image, held on every GPU that loads the library until
+ * the process exits.  count > BF_NOALLOC_MAX_SCENARIOS fails with BF_EINVAL.
+ * The first call on a device resolves that array's device address; make it
+ * before any stream capture.  All calls share the one array, so calls whose
+ * GPU work overlaps (other threads, other streams) race and must be
+ * serialised by the caller.  Blocks until the results are on the host. */
+int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
+                            void* cuda_stream);
+
 /* Time limit of blocking waits, in milliseconds (default 600000; 0 = none).
  * Process-wide. */
 void bf_set_wait_timeout_ms(uint32_t ms);

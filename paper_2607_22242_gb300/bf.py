@@ -5,7 +5,7 @@ CUDA kernels.  PyTorch supplies device buffers (``eval_mappings`` outputs) and
 streams (``torch.cuda.current_stream()`` by default).  The functions mirror
 the C entry points without their ``bf_`` prefix: ``validate_desc``,
 ``create_scenario``, ``destroy_scenario``, ``eval_mappings``, ``search_best``,
-``search_range``, ``search_batch``, ``set_wait_timeout_ms``, ``last_error``,
+``search_range``, ``search_batch``, ``search_batch_noalloc``, ``set_wait_timeout_ms``, ``last_error``,
 ``version``.
 
 There is no CPU fallback: if ``libbf.so`` has not been built, or no CUDA
@@ -26,8 +26,9 @@ BF_OK, BF_EINVAL, BF_ERANGE, BF_ENOMEM, BF_ECUDA, BF_ETIMEOUT = range(6)
 STATUS_NAMES = {0: "BF_OK", 1: "BF_EINVAL", 2: "BF_ERANGE", 3: "BF_ENOMEM", 4: "BF_ECUDA", 5: "BF_ETIMEOUT"}
 INFEASIBLE = 0xFFFFFFFF
 EXPORTED = ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
-            "bf_search_best", "bf_search_range", "bf_search_batch", "bf_set_wait_timeout_ms",
-            "bf_last_error", "bf_version")
+            "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc",
+            "bf_set_wait_timeout_ms", "bf_last_error", "bf_version")
+NOALLOC_MAX_SCENARIOS = 1024
 
 
 class BfError(RuntimeError):
@@ -80,8 +81,9 @@ def load(path: str = LIB_PATH):
     lib.bf_search_best.argtypes = [vp, ctypes.POINTER(CResult), vp]
     lib.bf_search_range.argtypes = [vp, u64, u64, ctypes.POINTER(CResult), vp]
     lib.bf_search_batch.argtypes = [ctypes.POINTER(Desc), u32, ctypes.POINTER(CResult), vp]
+    lib.bf_search_batch_noalloc.argtypes = [ctypes.POINTER(Desc), u32, ctypes.POINTER(CResult), vp]
     for name in ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
-                 "bf_search_best", "bf_search_range", "bf_search_batch"):
+                 "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc"):
         getattr(lib, name).restype = ctypes.c_int
     lib.bf_set_wait_timeout_ms.argtypes = [u32]
     lib.bf_set_wait_timeout_ms.restype = None
@@ -243,4 +245,22 @@ def search_batch(scns: Sequence[Scenario], stream=None) -> List[Result]:
         descs[i] = to_desc(s)
     results = (CResult * max(count, 1))()
     _check(load().bf_search_batch(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
+    return [_result(results[i], scns[i].n) for i in range(count)]
+
+
+def search_batch_noalloc(scns: Sequence[Scenario], stream=None) -> List[Result]:
+    """As :func:`search_batch`, but the library allocates no memory for the call.
+
+    For callers that cannot allocate device memory while they search (their GPU
+    memory belongs to another allocator's pool, or a cudaMalloc/cudaFree pair
+    would synchronise the device inside a latency-critical loop).  The scratch is
+    a fixed array in the library's device image; at most NOALLOC_MAX_SCENARIOS
+    scenarios per call, and calls that overlap on the GPU must not be issued.
+    """
+    count = len(scns)
+    descs = (Desc * max(count, 1))()
+    for i, s in enumerate(scns):
+        descs[i] = to_desc(s)
+    results = (CResult * max(count, 1))()
+    _check(load().bf_search_batch_noalloc(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
     return [_result(results[i], scns[i].n) for i in range(count)]

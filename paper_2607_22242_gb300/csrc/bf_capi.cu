@@ -3,6 +3,7 @@
 // runs in the kernels (bf_kernels.cu, bf_sim.cuh); this file only marshals.
 #include <cuda_runtime.h>
 
+#include <atomic>
 #include <chrono>
 #include <cstdarg>
 #include <cstdio>
@@ -298,6 +299,118 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
   }
   if (rc != BF_OK) return rc;
   for (uint32_t i = 0; i < count; ++i) fill_result(keys[i], descs[i].n, 0, out + i);
+  return BF_OK;
+}
+
+// ---------------------------------------------------------------------------
+// bf_search_batch_noalloc: the batched search with no allocation at all.
+//
+// Its scratch (the packed per-scenario records and one result key per
+// scenario) lives in the file-scope device array below instead of memory
+// obtained from cudaMalloc.  The array is part of this library's module, so
+// every GPU that loads the library holds it until the process exits.
+// ---------------------------------------------------------------------------
+}  // extern "C"
+
+namespace {
+
+constexpr size_t kNoAllocRecordBytes = sizeof(bfk::BatchRecord) * BF_NOALLOC_MAX_SCENARIOS;
+constexpr size_t kNoAllocKeyOffset = (kNoAllocRecordBytes + 255) / 256 * 256;
+constexpr size_t kNoAllocBytes = kNoAllocKeyOffset + sizeof(unsigned long long) * BF_NOALLOC_MAX_SCENARIOS;
+
+}  // namespace
+
+static __device__ __align__(256) unsigned char bf_noalloc_scratch[kNoAllocBytes];
+
+namespace {
+
+constexpr int kNoAllocMaxDevices = 64;
+std::atomic<unsigned char*> g_noalloc_base[kNoAllocMaxDevices];
+
+// Device address of bf_noalloc_scratch on the current device.  In host code
+// the array's name only stands in for it; the address is resolved once per
+// device, with that device current.
+int noalloc_scratch(unsigned char** base, const char* who) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  if (dev < 0 || dev >= kNoAllocMaxDevices)
+    return fail(BF_EINVAL, "%s: device %d is beyond the %d devices this entry point supports", who, dev,
+                kNoAllocMaxDevices);
+  unsigned char* p = g_noalloc_base[dev].load(std::memory_order_acquire);
+  if (!p) {
+    void* addr = nullptr;
+    e = cudaGetSymbolAddress(&addr, bf_noalloc_scratch);
+    if (e != cudaSuccess) return cuda_fail(e, who);
+    p = static_cast<unsigned char*>(addr);
+    g_noalloc_base[dev].store(p, std::memory_order_release);
+  }
+  *base = p;
+  return BF_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
+  const char* who = "bf_search_batch_noalloc";
+  if (count == 0) return BF_OK;
+  if (!descs || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
+  if (count > BF_NOALLOC_MAX_SCENARIOS)
+    return fail(BF_EINVAL, "%s: %u scenarios exceed this entry point's fixed scratch of %d scenarios; split the "
+                "batch or use bf_search_batch", who, count, BF_NOALLOC_MAX_SCENARIOS);
+  for (uint32_t i = 0; i < count; ++i) {
+    const int rc = validate(descs + i, who);
+    if (rc != BF_OK) return fail(rc, "%s: descs[%u]: %s", who, i, g_error.c_str());
+  }
+  unsigned char* base = nullptr;
+  int rc = noalloc_scratch(&base, who);
+  if (rc != BF_OK) return rc;
+  bfk::BatchRecord* d_recs = reinterpret_cast<bfk::BatchRecord*>(base);
+  unsigned long long* d_keys = reinterpret_cast<unsigned long long*>(base + kNoAllocKeyOffset);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+
+  // Pack the records a few at a time through a stack buffer (a copy from
+  // pageable memory has left the buffer when cudaMemcpyAsync returns).
+  constexpr uint32_t kChunk = 8;
+  bfk::BatchRecord chunk[kChunk];
+  uint32_t wmax = 0, pmax = 0;
+  cudaError_t e = cudaSuccess;
+  for (uint32_t i0 = 0; i0 < count && e == cudaSuccess; i0 += kChunk) {
+    const uint32_t nrec = (count - i0 < kChunk) ? (count - i0) : kChunk;
+    for (uint32_t j = 0; j < nrec; ++j) {
+      bfk::BatchRecord& r = chunk[j];
+      std::memset(&r, 0, sizeof r);
+      build_tables(descs + i0 + j, &r.full);
+      bfk::Plan plan;
+      split_and_window(r.full, &plan, &r.window);
+      r.plan = make_plan(plan, 0, pow3(descs[i0 + j].n));
+      if (r.window.n > wmax) wmax = r.window.n;
+      if (r.plan.pow3P > pmax) pmax = r.plan.pow3P;
+    }
+    e = cudaMemcpyAsync(d_recs + i0, chunk, sizeof(bfk::BatchRecord) * nrec, cudaMemcpyHostToDevice, st);
+  }
+  // The keys keep the previous call's values: reset them to "nothing found".
+  if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, sizeof(unsigned long long) * count, st);
+  if (e == cudaSuccess) {
+    const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
+#define CALL(NW) launch_batch_nw##NW(d_recs, count, bps, d_keys, st)
+    BF_DISPATCH(bfk::bucket_for(wmax), CALL)
+#undef CALL
+  }
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  rc = wait_stream(st, who);
+  if (rc != BF_OK) return rc;
+  constexpr uint32_t kKeyChunk = 256;
+  unsigned long long keys[kKeyChunk];
+  for (uint32_t i0 = 0; i0 < count; i0 += kKeyChunk) {
+    const uint32_t nk = (count - i0 < kKeyChunk) ? (count - i0) : kKeyChunk;
+    e = cudaMemcpyAsync(keys, d_keys + i0, sizeof(unsigned long long) * nk, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) return cuda_fail(e, who);
+    for (uint32_t j = 0; j < nk; ++j) fill_result(keys[j], descs[i0 + j].n, 0, out + i0 + j);
+  }
   return BF_OK;
 }
 
