@@ -44,6 +44,23 @@ OPS_PER_MAPPING = 2 * N_TOOLS * N_TOOLS
 INT_LANES_PER_SM = 128  # 4 SMSPs x 32 lanes issue one integer op each per clock
 
 
+PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "search_kernel_config3_n19.md")
+
+
+def profiled_traffic():
+    """DRAM bytes per launch of the search kernel from the committed ncu summary,
+    or None when the kernel sources changed since that capture."""
+    from paper_2607_22242_gb300 import _build
+    try:
+        text = open(PROFILE_SUMMARY).read()
+    except OSError:
+        return None
+    fields = dict(line.split(": ", 1) for line in text.splitlines() if line.startswith(("source_fingerprint: ", "dram_bytes_per_launch: ")))
+    if fields.get("source_fingerprint", "").strip() != _build._fingerprint(()):
+        return None
+    return int(fields["dram_bytes_per_launch"])
+
+
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
     world = int(os.environ.get("WORLD_SIZE", "1"))
@@ -243,7 +260,7 @@ def run_gpu(args):
     peak_ops = sm_count * INT_LANES_PER_SM * clk_mhz * 1e6
     achieved_ops = OPS_PER_MAPPING * total / (mean_ms / 1e3)
     roofline = {"bound": "alu", "achieved": achieved_ops / 1e12, "peak": peak_ops / 1e12, "unit": "Tops/s",
-                "frac": achieved_ops / peak_ops, "traffic": None,
+                "frac": achieved_ops / peak_ops, "traffic": profiled_traffic(),
                 "peak_basis": f"{sm_count} SMs x {INT_LANES_PER_SM} int lanes x "
                               f"{clk_mhz:.0f} MHz ({'sampled median under load' if clocks['sm_mhz'] else 'max clock, no samples'})",
                 "ops_per_mapping": OPS_PER_MAPPING}
