@@ -15,6 +15,7 @@ from __future__ import annotations
 
 import ctypes
 import dataclasses
+import itertools
 import os
 from typing import List, Optional, Sequence, Tuple, Union
 
@@ -121,6 +122,37 @@ def to_desc(scn: Scenario) -> Desc:
     for k, v in enumerate(scn.slowdown_q10[:MAX_TOOLS + 1]):
         d.slowdown_q10[k] = v
     return d
+
+
+DESC_WORDS = ctypes.sizeof(Desc) // 4
+
+
+def pack_descs(scns: Sequence[Scenario]):
+    """Pack scenarios into a contiguous (count, DESC_WORDS) uint32 array laid out as bf_scenario_desc[]."""
+    import numpy as np
+    count = len(scns)
+    arr = np.zeros((count, DESC_WORDS), dtype=np.uint32)
+    if count == 0:
+        return arr
+    cols = ("pred_mask", "cpu_us", "gpu_us", "xfer_us", "load_us", "vram_mib")
+    sizes = {sc.n for sc in scns}
+    if len(sizes) == 1:  # one tool count: fill whole columns at once
+        n = sizes.pop()
+        arr[:, 0] = n
+        flat = lambda rows, width: np.fromiter(itertools.chain.from_iterable(rows), dtype=np.uint32,
+                                               count=count * width).reshape(count, width)
+        for j, name in enumerate(cols):
+            arr[:, 1 + MAX_TOOLS * j: 1 + MAX_TOOLS * j + n] = flat((getattr(sc, name)[:n] for sc in scns), n)
+        arr[:, 1 + 6 * MAX_TOOLS] = np.fromiter((sc.vram_budget_mib for sc in scns), dtype=np.uint32, count=count)
+        arr[:, 2 + 6 * MAX_TOOLS:] = flat((sc.slowdown_q10[:MAX_TOOLS + 1] for sc in scns), MAX_TOOLS + 1)
+        return arr
+    for r, sc in enumerate(scns):
+        arr[r, 0] = sc.n
+        for j, name in enumerate(cols):
+            arr[r, 1 + MAX_TOOLS * j: 1 + MAX_TOOLS * j + sc.n] = getattr(sc, name)[:sc.n]
+        arr[r, 1 + 6 * MAX_TOOLS] = sc.vram_budget_mib
+        arr[r, 2 + 6 * MAX_TOOLS:] = sc.slowdown_q10[:MAX_TOOLS + 1]
+    return arr
 
 
 def _result(r: CResult, n: int) -> Result:
@@ -237,15 +269,18 @@ def search_range(h: Union[ScenarioHandle, Scenario], first: int, count: int, str
             handle.close()
 
 
+def _batch_call(fn, scns: Sequence[Scenario], stream) -> List[Result]:
+    count = len(scns)
+    packed = pack_descs(scns) if count else None
+    descs = packed.ctypes.data_as(ctypes.POINTER(Desc)) if count else None
+    results = (CResult * max(count, 1))()
+    _check(fn(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
+    return [_result(results[i], scns[i].n) for i in range(count)]
+
+
 def search_batch(scns: Sequence[Scenario], stream=None) -> List[Result]:
     """Full search of each scenario, one launch for the whole batch."""
-    count = len(scns)
-    descs = (Desc * max(count, 1))()
-    for i, s in enumerate(scns):
-        descs[i] = to_desc(s)
-    results = (CResult * max(count, 1))()
-    _check(load().bf_search_batch(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
-    return [_result(results[i], scns[i].n) for i in range(count)]
+    return _batch_call(load().bf_search_batch, scns, stream)
 
 
 def search_batch_noalloc(scns: Sequence[Scenario], stream=None) -> List[Result]:
@@ -257,10 +292,4 @@ def search_batch_noalloc(scns: Sequence[Scenario], stream=None) -> List[Result]:
     a fixed array in the library's device image; at most NOALLOC_MAX_SCENARIOS
     scenarios per call, and calls that overlap on the GPU must not be issued.
     """
-    count = len(scns)
-    descs = (Desc * max(count, 1))()
-    for i, s in enumerate(scns):
-        descs[i] = to_desc(s)
-    results = (CResult * max(count, 1))()
-    _check(load().bf_search_batch_noalloc(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
-    return [_result(results[i], scns[i].n) for i in range(count)]
+    return _batch_call(load().bf_search_batch_noalloc, scns, stream)

@@ -286,7 +286,7 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
   int rc = BF_OK;
   if (e == cudaSuccess) {
     const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
-#define CALL(NW) launch_batch_nw##NW(d_recs, count, bps, d_keys, st)
+#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, bps, d_keys, st)
     BF_DISPATCH(bfk::bucket_for(wmax), CALL)
 #undef CALL
   }
@@ -360,9 +360,11 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
   if (count > BF_NOALLOC_MAX_SCENARIOS)
     return fail(BF_EINVAL, "%s: %u scenarios exceed this entry point's fixed scratch of %d scenarios; split the "
                 "batch or use bf_search_batch", who, count, BF_NOALLOC_MAX_SCENARIOS);
+  uint32_t nmax = 0;
   for (uint32_t i = 0; i < count; ++i) {
     const int rc = validate(descs + i, who);
     if (rc != BF_OK) return fail(rc, "%s: descs[%u]: %s", who, i, g_error.c_str());
+    if (descs[i].n > nmax) nmax = descs[i].n;
   }
   unsigned char* base = nullptr;
   int rc = noalloc_scratch(&base, who);
@@ -395,7 +397,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, sizeof(unsigned long long) * count, st);
   if (e == cudaSuccess) {
     const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
-#define CALL(NW) launch_batch_nw##NW(d_recs, count, bps, d_keys, st)
+#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, bps, d_keys, st)
     BF_DISPATCH(bfk::bucket_for(wmax), CALL)
 #undef CALL
   }

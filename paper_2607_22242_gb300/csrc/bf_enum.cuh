@@ -10,16 +10,17 @@ namespace bfk {
 // Simulate prefix p once per warp and save its window state in `snap`.
 // Returns false (warp-uniformly) when every mapping with this prefix is
 // infeasible.
-template <typename TB>
+// NP >= n is the slot count of the prefix simulation.
+template <int NP, typename TB>
 __device__ __forceinline__ bool prefix_phase(const TB& tb, const SmemTables& sd, const Plan& plan,
                                              uint32_t p, Digits& dgp, Snapshot& snap) {
   dgp = decode(p, plan.P);
   bool ok = (dgp.que & tb.big_mask) == 0u;
   if (ok) {
-    State<kMaxTools> s;
+    State<NP> s;
     init_state(s, tb.all_mask);
     const uint32_t later = tb.all_mask & ~((1u << plan.P) - 1u);
-    ok = run<kMaxTools>(s, tb, sd, dgp, later) == kRunStopped;
+    ok = run<NP>(s, tb, sd, dgp, later) == kRunStopped;
     if (ok && (threadIdx.x & 31) == 0) save_window(s, plan.W0, tb.n - plan.W0, snap);
   }
   __syncwarp();

@@ -28,6 +28,23 @@
 #error "compile with -DBF_NW=<window slot count>"
 #endif
 
+// Minimum resident blocks per SM requested from the compiler, which caps the
+// registers per thread (measured on GB300: 4 blocks of 256 threads is fastest
+// for windows of up to 8 slots, 3 up to 16, 2 above; 2 for the batch kernel,
+// whose tables sit in shared memory).
+#ifndef BF_MIN_BLOCKS
+#if BF_NW <= 8
+#define BF_MIN_BLOCKS 4
+#elif BF_NW <= 16
+#define BF_MIN_BLOCKS 3
+#else
+#define BF_MIN_BLOCKS 2
+#endif
+#endif
+#ifndef BF_MIN_BLOCKS_BATCH
+#define BF_MIN_BLOCKS_BATCH 2
+#endif
+
 namespace bfk {
 namespace {
 
@@ -54,7 +71,8 @@ __device__ __forceinline__ void block_min_to(unsigned long long v, unsigned long
   }
 }
 
-__global__ void __launch_bounds__(kThreads) eval_kernel(const __grid_constant__ Tables tb,
+template <int NP>
+__global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) eval_kernel(const __grid_constant__ Tables tb,
                                                         const __grid_constant__ Tables tw,
                                                         const __grid_constant__ Plan plan,
                                                         uint32_t* __restrict__ ms_out,
@@ -70,12 +88,13 @@ __global__ void __launch_bounds__(kThreads) eval_kernel(const __grid_constant__ 
   if (p64 > plan.p_hi) return;  // no block-level synchronisation follows
   const uint32_t p = (uint32_t)p64;
   Digits dgp;
-  const bool ok = prefix_phase(tb, sd, plan, p, dgp, snap[warp]);
+  const bool ok = prefix_phase<NP>(tb, sd, plan, p, dgp, snap[warp]);
   StoreSink sink{plan.first, ms_out, fe_out};
   lane_mappings<BF_NW>(tw, sdw, plan, p, ok, dgp, snap[warp], lane_state + threadIdx.x, kThreads, sink);
 }
 
-__global__ void __launch_bounds__(kThreads) search_kernel(const __grid_constant__ Tables tb,
+template <int NP>
+__global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) search_kernel(const __grid_constant__ Tables tb,
                                                           const __grid_constant__ Tables tw,
                                                           const __grid_constant__ Plan plan,
                                                           unsigned long long* key) {
@@ -91,13 +110,14 @@ __global__ void __launch_bounds__(kThreads) search_kernel(const __grid_constant_
   if (p64 <= plan.p_hi) {
     const uint32_t p = (uint32_t)p64;
     Digits dgp;
-    if (prefix_phase(tb, sd, plan, p, dgp, snap[warp])) lane_mappings<BF_NW>(tw, sdw, plan, p, true, dgp, snap[warp], lane_state + threadIdx.x, kThreads, sink);
+    if (prefix_phase<NP>(tb, sd, plan, p, dgp, snap[warp])) lane_mappings<BF_NW>(tw, sdw, plan, p, true, dgp, snap[warp], lane_state + threadIdx.x, kThreads, sink);
   }
   block_min_to(sink.best, key);
 }
 
 // One record per scenario of a batch: full tables, window tables and plan.
-__global__ void __launch_bounds__(kThreads, 2) batch_kernel(const BatchRecord* __restrict__ recs,
+template <int NP>
+__global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(const BatchRecord* __restrict__ recs,
                                                          uint32_t blocks_per_scenario,
                                                          unsigned long long* keys) {
   __shared__ BatchRecord rec;
@@ -121,7 +141,7 @@ __global__ void __launch_bounds__(kThreads, 2) batch_kernel(const BatchRecord* _
   if (p64 <= rec.plan.p_hi) {
     const uint32_t p = (uint32_t)p64;
     Digits dgp;
-    if (prefix_phase(rec.full, sd, rec.plan, p, dgp, snap[warp]))
+    if (prefix_phase<NP>(rec.full, sd, rec.plan, p, dgp, snap[warp]))
       lane_mappings<BF_NW>(rec.window, sdw, rec.plan, p, true, dgp, snap[warp], lane_state + threadIdx.x,
                            kThreads, sink);
   }
@@ -138,23 +158,34 @@ static unsigned blocks_for(const Plan& plan) {
   return (unsigned)((warps + kWarps - 1) / kWarps);
 }
 
+// The prefix simulation runs BF_NW slots wide when the scenario fits (n <= BF_NW),
+// else kMaxTools wide.
 cudaError_t BF_PASTE(launch_eval_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                             uint32_t* ms, uint8_t* fe, cudaStream_t st) {
-  eval_kernel<<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, ms, fe);
+  if (tb.n <= (uint32_t)BF_NW)
+    eval_kernel<BF_NW><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, ms, fe);
+  else
+    eval_kernel<kMaxTools><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, ms, fe);
   return cudaGetLastError();
 }
 
 cudaError_t BF_PASTE(launch_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                               unsigned long long* key, cudaStream_t st) {
-  search_kernel<<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, key);
+  if (tb.n <= (uint32_t)BF_NW)
+    search_kernel<BF_NW><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, key);
+  else
+    search_kernel<kMaxTools><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, key);
   return cudaGetLastError();
 }
 
-cudaError_t BF_PASTE(launch_batch_nw, BF_NW)(const BatchRecord* d_recs, uint32_t count,
+cudaError_t BF_PASTE(launch_batch_nw, BF_NW)(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,
                                              uint32_t blocks_per_scenario, unsigned long long* keys,
                                              cudaStream_t st) {
   const uint64_t blocks = (uint64_t)count * blocks_per_scenario;
-  batch_kernel<<<(unsigned)blocks, kThreads, 0, st>>>(d_recs, blocks_per_scenario, keys);
+  if (nmax <= (uint32_t)BF_NW)
+    batch_kernel<BF_NW><<<(unsigned)blocks, kThreads, 0, st>>>(d_recs, blocks_per_scenario, keys);
+  else
+    batch_kernel<kMaxTools><<<(unsigned)blocks, kThreads, 0, st>>>(d_recs, blocks_per_scenario, keys);
   return cudaGetLastError();
 }
 

@@ -311,7 +311,9 @@ struct Snapshot {
   uint32_t T, V, L, k, tc, gmin;
 };
 
-// Save the window part of a full-width prefix state (slots >= W0, renumbered).
+// Save the window part of a prefix state (slots >= W0, renumbered).  Window
+// slots beyond the prefix state's last slot are written as unused slots (no
+// CPU end, stamp 0), so every slot a window simulation reads is defined.
 template <int NT>
 __device__ __forceinline__ void save_window(const State<NT>& s, uint32_t W0, uint32_t nw, Snapshot& out) {
 #pragma unroll
@@ -320,6 +322,10 @@ __device__ __forceinline__ void save_window(const State<NT>& s, uint32_t W0, uin
       out.ec[i - W0] = s.ec[i];
       out.eg[i - W0] = s.eg[i];
     }
+  }
+  for (uint32_t j = (uint32_t)NT - W0; j < (uint32_t)kMaxTools; ++j) {
+    out.ec[j] = 0xFFFFFFFFu;
+    out.eg[j] = 0u;
   }
   const uint32_t wmask = (nw >= 32u) ? 0xFFFFFFFFu : ((1u << nw) - 1u);
   out.done = (s.done >> W0) | ~wmask;
