@@ -34,6 +34,10 @@ using bfk::host::make_plan;
 using bfk::host::pow3;
 using bfk::host::split_and_window;
 
+// Warp tasks a single-scenario launch is split into (several waves of the
+// GPU's resident warps, so that uneven tasks even out).
+constexpr uint64_t kSearchTasks = 32768;
+
 thread_local std::string g_error;
 uint32_t g_wait_timeout_ms = 600000;
 
@@ -166,7 +170,7 @@ int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result
   cudaError_t e = cudaMemsetAsync(scn->d_key, 0xFF, sizeof(unsigned long long), st);
   if (e != cudaSuccess) return cuda_fail(e, who);
   if (count) {
-    const bfk::Plan plan = make_plan(scn->plan, first, count);
+    const bfk::Plan plan = make_plan(scn->plan, first, count, kSearchTasks);
 #define CALL(NW) launch_search_nw##NW(scn->tables, scn->window, plan, scn->d_key, st)
     BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
 #undef CALL
@@ -229,7 +233,7 @@ int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count, uin
   if (count == 0) return BF_OK;
   if (!d_makespan || !d_feasible) return fail(BF_EINVAL, "bf_eval_mappings: NULL output buffer");
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  const bfk::Plan plan = make_plan(scn->plan, first, count);
+  const bfk::Plan plan = make_plan(scn->plan, first, count, kSearchTasks);
   cudaError_t e = cudaSuccess;
 #define CALL(NW) launch_eval_nw##NW(scn->tables, scn->window, plan, d_makespan, d_feasible, st)
   BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
@@ -263,16 +267,18 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
     if (descs[i].n > nmax) nmax = descs[i].n;
   }
   std::vector<bfk::BatchRecord> recs(count);
-  uint32_t wmax = 0, pmax = 0;
+  uint32_t wmax = 0, pmax = 0, any_inner = 0;
   for (uint32_t i = 0; i < count; ++i) {
     bfk::BatchRecord& r = recs[i];
     std::memset(&r, 0, sizeof r);
     build_tables(descs + i, &r.full);
     bfk::Plan base;
     split_and_window(r.full, &base, &r.window);
-    r.plan = make_plan(base, 0, pow3(descs[i].n));
+    r.plan = make_plan(base, 0, pow3(descs[i].n), 1);
     if (r.window.n > wmax) wmax = r.window.n;
-    if (r.plan.pow3P > pmax) pmax = r.plan.pow3P;
+    const uint32_t tasks = r.plan.groups * r.plan.m_parts;
+    if (tasks > pmax) pmax = tasks;
+    any_inner |= r.plan.I;
   }
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   bfk::BatchRecord* d_recs = nullptr;
@@ -286,7 +292,7 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
   int rc = BF_OK;
   if (e == cudaSuccess) {
     const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
-#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, bps, d_keys, st)
+#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, any_inner, bps, d_keys, st)
     BF_DISPATCH(bfk::bucket_for(wmax), CALL)
 #undef CALL
   }
@@ -377,7 +383,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
   // pageable memory has left the buffer when cudaMemcpyAsync returns).
   constexpr uint32_t kChunk = 8;
   bfk::BatchRecord chunk[kChunk];
-  uint32_t wmax = 0, pmax = 0;
+  uint32_t wmax = 0, pmax = 0, any_inner = 0;
   cudaError_t e = cudaSuccess;
   for (uint32_t i0 = 0; i0 < count && e == cudaSuccess; i0 += kChunk) {
     const uint32_t nrec = (count - i0 < kChunk) ? (count - i0) : kChunk;
@@ -387,9 +393,11 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
       build_tables(descs + i0 + j, &r.full);
       bfk::Plan plan;
       split_and_window(r.full, &plan, &r.window);
-      r.plan = make_plan(plan, 0, pow3(descs[i0 + j].n));
+      r.plan = make_plan(plan, 0, pow3(descs[i0 + j].n), 1);
       if (r.window.n > wmax) wmax = r.window.n;
-      if (r.plan.pow3P > pmax) pmax = r.plan.pow3P;
+      const uint32_t tasks = r.plan.groups * r.plan.m_parts;
+      if (tasks > pmax) pmax = tasks;
+      any_inner |= r.plan.I;
     }
     e = cudaMemcpyAsync(d_recs + i0, chunk, sizeof(bfk::BatchRecord) * nrec, cudaMemcpyHostToDevice, st);
   }
@@ -397,7 +405,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, sizeof(unsigned long long) * count, st);
   if (e == cudaSuccess) {
     const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
-#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, bps, d_keys, st)
+#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, any_inner, bps, d_keys, st)
     BF_DISPATCH(bfk::bucket_for(wmax), CALL)
 #undef CALL
   }

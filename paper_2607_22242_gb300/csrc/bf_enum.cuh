@@ -1,65 +1,82 @@
-// bf_enum.cuh -- how a warp enumerates its share of the mapping space (see
-// bfk::Plan): the shared prefix simulation and each lane's mid/inner walk.
-// Used by the kernels in bf_kernels.cu; sinks receive (index, makespan).
+// bf_enum.cuh -- one warp task of the enumeration (see bfk::Plan): 32
+// consecutive prefixes, one per lane, times a chunk of mid combinations, each
+// with its inner combinations.  Used by the kernels in bf_kernels.cu; the
+// sink receives (canonical index, makespan) for every mapping of the task
+// that lies inside [plan.first, plan.last].
 #pragma once
 
 #include "bf_sim.cuh"
 
 namespace bfk {
 
-// Simulate prefix p once per warp and save its window state in `snap`.
-// Returns false (warp-uniformly) when every mapping with this prefix is
-// infeasible.
-// NP >= n is the slot count of the prefix simulation.
-template <int NP, typename TB>
-__device__ __forceinline__ bool prefix_phase(const TB& tb, const SmemTables& sd, const Plan& plan,
-                                             uint32_t p, Digits& dgp, Snapshot& snap) {
-  dgp = decode(p, plan.P);
-  bool ok = (dgp.que & tb.big_mask) == 0u;
-  if (ok) {
-    State<NP> s;
-    init_state(s, tb.all_mask);
-    const uint32_t later = tb.all_mask & ~((1u << plan.P) - 1u);
-    ok = run<NP>(s, tb, sd, dgp, later) == kRunStopped;
-    if (ok && (threadIdx.x & 31) == 0) save_window(s, plan.W0, tb.n - plan.W0, snap);
+// Inner combinations [*lo, *hi] of (p, m) that fall inside [first, last];
+// returns false when there is none.  base = p + 3^P * m.
+__device__ __forceinline__ bool inner_range(const Plan& plan, uint64_t base, uint64_t stride_i, uint32_t* lo,
+                                            uint32_t* hi) {
+  uint32_t a = plan.i_lo, b = plan.i_hi;
+  while (a <= b && base + stride_i * a < plan.first) ++a;
+  while (a <= b && base + stride_i * b > plan.last) {
+    if (b == 0u) return false;
+    --b;
   }
-  __syncwarp();
-  return ok;
+  *lo = a;
+  *hi = b;
+  return a <= b;
 }
 
-// Every mapping (p, m, i) of this lane, in window form, handed to
-// sink(idx, makespan).  `ok` is the prefix verdict; the prefix digits dgp and
-// the warp's snapshot come from prefix_phase.  `slot`/`stride` is this lane's
-// shared-memory area of LaneWords<NW>::value words for the inner-level state.
-template <int NW, typename TB, typename Sink>
-__device__ __forceinline__ void lane_mappings(const TB& tw, const SmemTables& sdw, const Plan& plan,
-                                              uint32_t p, bool ok, Digits dgp, const Snapshot& snap,
-                                              uint32_t* slot, uint32_t stride, Sink& sink) {
-  const uint32_t lane = threadIdx.x & 31;
-  const uint32_t shm = plan.P - plan.W0;          // first mid tool, window numbering
-  const uint32_t shi = shm + plan.M;              // first inner tool, window numbering
+// Run one warp task: prefix group `g` (prefix p_lo + 32 g + lane) and mid chunk
+// `part`.  NP >= n is the prefix simulation's slot count, NW >= the window's.
+// slotA / slotB are this lane's shared-memory areas of LaneWords<NW> words
+// (stride `stride`) for the state at the prefix checkpoint and at the inner
+// checkpoint.
+template <int NP, int NW, typename TBF, typename TBW, typename Sink>
+__device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, const TBW& tw,
+                                          const SmemTables& sdw, const Plan& plan, uint32_t g, uint32_t part,
+                                          uint32_t* slotA, uint32_t* slotB, uint32_t stride, Sink& sink) {
+  const uint32_t lane = threadIdx.x & 31u;
+  const uint64_t p64 = (uint64_t)plan.p_lo + 32ull * g + lane;
+  const bool p_valid = p64 <= plan.p_hi;
+  const uint32_t p = (uint32_t)p64;
+
+  // ---- this lane's prefix, up to the first instant a tool >= P is ready ----
+  Digits dgp{0u, 0u};
+  bool ok = false;
+  if (p_valid) {
+    dgp = decode(p, plan.P);
+    ok = (dgp.que & tb.big_mask) == 0u;
+    if (ok) {
+      State<NP> s;
+      init_state(s, tb.all_mask);
+      const uint32_t later = tb.all_mask & ~((1u << plan.P) - 1u);
+      ok = run<NP>(s, tb, sd, dgp, later) == kRunStopped;
+      if (ok) save_prefix_window<NP, NW>(s, plan.W0, tb.n - plan.W0, slotA, stride);
+    }
+  }
+
+  // ---- the task's mid combinations, in lockstep across the warp -----------
+  const uint32_t shm = plan.P - plan.W0;  // first mid tool, window numbering
+  const uint32_t shi = shm + plan.M;      // first inner tool, window numbering
   const uint32_t inner_mask = tw.all_mask & ~((1u << shi) - 1u);
   const uint64_t stride_i = (uint64_t)plan.pow3P * plan.pow3M;
-  for (uint32_t m = lane; m < plan.pow3M; m += 32) {
-    // Inner combinations of (p, m) inside [first, last].
+  const Digits dgw{dgp.now >> plan.W0, dgp.que >> plan.W0};
+  const uint32_t m0 = plan.m_lo + part * plan.m_chunk;
+  const uint32_t m1 = min(m0 + plan.m_chunk - 1u, plan.m_hi);
+  for (uint32_t m = m0; m <= m1; ++m) {
     const uint64_t base = (uint64_t)p + (uint64_t)plan.pow3P * m;
-    uint32_t i_lo = plan.i_lo, i_hi = plan.i_hi;
-    while (i_lo <= i_hi && base + stride_i * i_lo < plan.first) ++i_lo;
-    while (i_hi >= i_lo && base + stride_i * i_hi > plan.last) {
-      if (i_hi == 0) { i_lo = 1; break; }
-      --i_hi;
-    }
-    if (i_lo > i_hi) continue;
-    if (!ok) {
+    uint32_t i_lo, i_hi;
+    if (!p_valid || !inner_range(plan, base, stride_i, &i_lo, &i_hi)) continue;
+    if (!ok) {  // every mapping with this prefix is infeasible
       for (uint32_t i = i_lo; i <= i_hi; ++i) sink((uint32_t)(base + stride_i * i), kInfeasible);
       continue;
     }
     const Digits dm = decode(m, plan.M);
-    const Digits dmid{(dgp.now >> plan.W0) | (dm.now << shm), (dgp.que >> plan.W0) | (dm.que << shm)};
+    const Digits dmid{dgw.now | (dm.now << shm), dgw.que | (dm.que << shm)};
     State<NW> w;
-    load_window(snap, w);
     uint32_t r = kRunInfeasible;
-    if ((dmid.que & tw.big_mask) == 0u) r = run<NW>(w, tw, sdw, dmid, inner_mask);
+    if ((dmid.que & tw.big_mask) == 0u) {
+      load_lane(slotA, stride, w);
+      r = run<NW>(w, tw, sdw, dmid, inner_mask);
+    }
     if (plan.I == 0u) {  // no inner level: the run went to the end
       sink((uint32_t)base, r == kRunFinished ? w.T : kInfeasible);
       continue;
@@ -68,13 +85,13 @@ __device__ __forceinline__ void lane_mappings(const TB& tw, const SmemTables& sd
       for (uint32_t i = i_lo; i <= i_hi; ++i) sink((uint32_t)(base + stride_i * i), kInfeasible);
       continue;
     }
-    save_lane(w, slot, stride);
+    save_lane(w, slotB, stride);
     for (uint32_t i = i_lo; i <= i_hi; ++i) {
       const Digits di = decode(i, plan.I);
       const Digits dg{dmid.now | (di.now << shi), dmid.que | (di.que << shi)};
       uint32_t ms = kInfeasible;
       if ((dg.que & tw.big_mask) == 0u) {
-        if (i != i_lo) load_lane(slot, stride, w);
+        if (i != i_lo) load_lane(slotB, stride, w);
         ms = run<NW>(w, tw, sdw, dg, 0u) == kRunFinished ? w.T : kInfeasible;
       }
       sink((uint32_t)(base + stride_i * i), ms);

@@ -29,13 +29,12 @@
 #endif
 
 // Minimum resident blocks per SM requested from the compiler, which caps the
-// registers per thread (measured on GB300: 4 blocks of 256 threads is fastest
-// for windows of up to 8 slots, 3 up to 16, 2 above; 2 for the batch kernel,
-// whose tables sit in shared memory).
+// registers per thread.  Each thread keeps up to two saved window states of
+// 2*NW+12 words in shared memory, so wider windows fit fewer blocks per SM.
 #ifndef BF_MIN_BLOCKS
-#if BF_NW <= 8
+#if BF_NW <= 6
 #define BF_MIN_BLOCKS 4
-#elif BF_NW <= 16
+#elif BF_NW <= 12
 #define BF_MIN_BLOCKS 3
 #else
 #define BF_MIN_BLOCKS 2
@@ -71,59 +70,57 @@ __device__ __forceinline__ void block_min_to(unsigned long long v, unsigned long
   }
 }
 
+// Dynamic shared memory of every kernel: one saved window state per thread for
+// the prefix checkpoint, and a second one for the inner checkpoint when the
+// plan has an inner level; [word][thread] layout.
+constexpr int kLaneWords = LaneWords<BF_NW>::value;
+constexpr size_t kDynSmemBytes = sizeof(uint32_t) * 2 * kLaneWords * kThreads;
+inline size_t dyn_smem_bytes(uint32_t inner_levels) { return inner_levels ? kDynSmemBytes : kDynSmemBytes / 2; }
+
 template <int NP>
 __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) eval_kernel(const __grid_constant__ Tables tb,
-                                                        const __grid_constant__ Tables tw,
-                                                        const __grid_constant__ Plan plan,
-                                                        uint32_t* __restrict__ ms_out,
-                                                        uint8_t* __restrict__ fe_out) {
+                                                                       const __grid_constant__ Tables tw,
+                                                                       const __grid_constant__ Plan plan,
+                                                                       uint32_t* __restrict__ ms_out,
+                                                                       uint8_t* __restrict__ fe_out) {
+  extern __shared__ uint32_t lane_state[];
   __shared__ SmemTables sd, sdw;
-  __shared__ Snapshot snap[kWarps];
-  __shared__ uint32_t lane_state[LaneWords<BF_NW>::value * kThreads];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
   __syncthreads();
-  const int warp = threadIdx.x >> 5;
-  const uint64_t p64 = (uint64_t)plan.p_lo + (uint64_t)blockIdx.x * kWarps + warp;
-  if (p64 > plan.p_hi) return;  // no block-level synchronisation follows
-  const uint32_t p = (uint32_t)p64;
-  Digits dgp;
-  const bool ok = prefix_phase<NP>(tb, sd, plan, p, dgp, snap[warp]);
+  const uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  if (task >= plan.groups * plan.m_parts) return;  // no block-level synchronisation follows
   StoreSink sink{plan.first, ms_out, fe_out};
-  lane_mappings<BF_NW>(tw, sdw, plan, p, ok, dgp, snap[warp], lane_state + threadIdx.x, kThreads, sink);
+  warp_task<NP, BF_NW>(tb, sd, tw, sdw, plan, task / plan.m_parts, task % plan.m_parts, lane_state + threadIdx.x,
+                       lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
 }
 
 template <int NP>
 __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) search_kernel(const __grid_constant__ Tables tb,
-                                                          const __grid_constant__ Tables tw,
-                                                          const __grid_constant__ Plan plan,
-                                                          unsigned long long* key) {
+                                                                         const __grid_constant__ Tables tw,
+                                                                         const __grid_constant__ Plan plan,
+                                                                         unsigned long long* key) {
+  extern __shared__ uint32_t lane_state[];
   __shared__ SmemTables sd, sdw;
-  __shared__ Snapshot snap[kWarps];
-  __shared__ uint32_t lane_state[LaneWords<BF_NW>::value * kThreads];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
   __syncthreads();
-  const int warp = threadIdx.x >> 5;
-  const uint64_t p64 = (uint64_t)plan.p_lo + (uint64_t)blockIdx.x * kWarps + warp;
+  const uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5);
   MinKeySink sink;
-  if (p64 <= plan.p_hi) {
-    const uint32_t p = (uint32_t)p64;
-    Digits dgp;
-    if (prefix_phase<NP>(tb, sd, plan, p, dgp, snap[warp])) lane_mappings<BF_NW>(tw, sdw, plan, p, true, dgp, snap[warp], lane_state + threadIdx.x, kThreads, sink);
-  }
+  if (task < plan.groups * plan.m_parts)
+    warp_task<NP, BF_NW>(tb, sd, tw, sdw, plan, task / plan.m_parts, task % plan.m_parts, lane_state + threadIdx.x,
+                         lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
   block_min_to(sink.best, key);
 }
 
 // One record per scenario of a batch: full tables, window tables and plan.
 template <int NP>
 __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(const BatchRecord* __restrict__ recs,
-                                                         uint32_t blocks_per_scenario,
-                                                         unsigned long long* keys) {
+                                                                              uint32_t blocks_per_scenario,
+                                                                              unsigned long long* keys) {
+  extern __shared__ uint32_t lane_state[];
   __shared__ BatchRecord rec;
   __shared__ SmemTables sd, sdw;
-  __shared__ Snapshot snap[kWarps];
-  __shared__ uint32_t lane_state[LaneWords<BF_NW>::value * kThreads];
   const uint32_t sc = blockIdx.x / blocks_per_scenario;
   const uint32_t b = blockIdx.x - sc * blocks_per_scenario;
   {
@@ -135,17 +132,21 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
   load_smem_tables(rec.full, sd);
   load_smem_tables(rec.window, sdw);
   __syncthreads();
-  const int warp = threadIdx.x >> 5;
-  const uint64_t p64 = (uint64_t)rec.plan.p_lo + (uint64_t)b * kWarps + warp;
+  const uint32_t task = b * kWarps + (threadIdx.x >> 5);
   MinKeySink sink;
-  if (p64 <= rec.plan.p_hi) {
-    const uint32_t p = (uint32_t)p64;
-    Digits dgp;
-    if (prefix_phase<NP>(rec.full, sd, rec.plan, p, dgp, snap[warp]))
-      lane_mappings<BF_NW>(rec.window, sdw, rec.plan, p, true, dgp, snap[warp], lane_state + threadIdx.x,
-                           kThreads, sink);
-  }
+  if (task < rec.plan.groups * rec.plan.m_parts)
+    warp_task<NP, BF_NW>(rec.full, sd, rec.window, sdw, rec.plan, task / rec.plan.m_parts, task % rec.plan.m_parts,
+                         lane_state + threadIdx.x, lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
   block_min_to(sink.best, keys + sc);
+}
+
+// Allow the kernel more than the default 48 KB of dynamic shared memory (once per kernel).
+template <typename K>
+static cudaError_t allow_dyn_smem(K kernel, bool* done) {
+  if (*done) return cudaSuccess;
+  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDynSmemBytes);
+  if (e == cudaSuccess) *done = true;
+  return e;
 }
 
 }  // namespace
@@ -154,39 +155,40 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
 #define BF_PASTE(a, b) BF_PASTE2(a, b)
 
 static unsigned blocks_for(const Plan& plan) {
-  const uint64_t warps = (uint64_t)plan.p_hi - plan.p_lo + 1;
-  return (unsigned)((warps + kWarps - 1) / kWarps);
+  const uint64_t tasks = (uint64_t)plan.groups * plan.m_parts;
+  return (unsigned)((tasks + kWarps - 1) / kWarps);
 }
 
-// The prefix simulation runs BF_NW slots wide when the scenario fits (n <= BF_NW),
-// else kMaxTools wide.
+// Each launcher picks the prefix width (BF_NW when the scenario fits, else 20).
+#define BF_LAUNCH(KERNEL, FITS, INNER, GRID, ...)                                            \
+  do {                                                                                       \
+    static bool ready_narrow = false, ready_wide = false;                                    \
+    cudaError_t e_ = (FITS) ? allow_dyn_smem(KERNEL<BF_NW>, &ready_narrow)                  \
+                            : allow_dyn_smem(KERNEL<kMaxTools>, &ready_wide);                \
+    if (e_ != cudaSuccess) return e_;                                                        \
+    const size_t smem_ = dyn_smem_bytes(INNER);                                              \
+    if (FITS)                                                                                \
+      KERNEL<BF_NW><<<(GRID), kThreads, smem_, st>>>(__VA_ARGS__);                           \
+    else                                                                                     \
+      KERNEL<kMaxTools><<<(GRID), kThreads, smem_, st>>>(__VA_ARGS__);                       \
+    return cudaGetLastError();                                                               \
+  } while (0)
+
 cudaError_t BF_PASTE(launch_eval_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                             uint32_t* ms, uint8_t* fe, cudaStream_t st) {
-  if (tb.n <= (uint32_t)BF_NW)
-    eval_kernel<BF_NW><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, ms, fe);
-  else
-    eval_kernel<kMaxTools><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, ms, fe);
-  return cudaGetLastError();
+  BF_LAUNCH(eval_kernel, tb.n <= (uint32_t)BF_NW, plan.I, blocks_for(plan), tb, tw, plan, ms, fe);
 }
 
 cudaError_t BF_PASTE(launch_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                               unsigned long long* key, cudaStream_t st) {
-  if (tb.n <= (uint32_t)BF_NW)
-    search_kernel<BF_NW><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, key);
-  else
-    search_kernel<kMaxTools><<<blocks_for(plan), kThreads, 0, st>>>(tb, tw, plan, key);
-  return cudaGetLastError();
+  BF_LAUNCH(search_kernel, tb.n <= (uint32_t)BF_NW, plan.I, blocks_for(plan), tb, tw, plan, key);
 }
 
 cudaError_t BF_PASTE(launch_batch_nw, BF_NW)(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,
-                                             uint32_t blocks_per_scenario, unsigned long long* keys,
-                                             cudaStream_t st) {
-  const uint64_t blocks = (uint64_t)count * blocks_per_scenario;
-  if (nmax <= (uint32_t)BF_NW)
-    batch_kernel<BF_NW><<<(unsigned)blocks, kThreads, 0, st>>>(d_recs, blocks_per_scenario, keys);
-  else
-    batch_kernel<kMaxTools><<<(unsigned)blocks, kThreads, 0, st>>>(d_recs, blocks_per_scenario, keys);
-  return cudaGetLastError();
+                                             uint32_t any_inner, uint32_t blocks_per_scenario,
+                                             unsigned long long* keys, cudaStream_t st) {
+  const unsigned blocks = (unsigned)((uint64_t)count * blocks_per_scenario);
+  BF_LAUNCH(batch_kernel, nmax <= (uint32_t)BF_NW, any_inner, blocks, d_recs, blocks_per_scenario, keys);
 }
 
 }  // namespace bfk

@@ -36,8 +36,8 @@ inline int bucket_for(uint32_t w) {
   cudaError_t launch_search_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan,             \
                                    unsigned long long* key, cudaStream_t st);                        \
   cudaError_t launch_batch_nw##NW(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,           \
-                                  uint32_t blocks_per_scenario, unsigned long long* keys,            \
-                                  cudaStream_t st);
+                                  uint32_t any_inner, uint32_t blocks_per_scenario,                  \
+                                  unsigned long long* keys, cudaStream_t st);
 BF_FOR_EACH_BUCKET(BF_DECLARE_BUCKET)
 #undef BF_DECLARE_BUCKET
 

@@ -131,8 +131,12 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
   }
 }
 
-// Restrict a scenario's plan to canonical indices [first, first+count), count >= 1.
-inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count) {
+// Restrict a scenario's plan to canonical indices [first, first+count),
+// count >= 1, and split its work into warp tasks: prefix groups of 32 times
+// chunks of mid combinations, about `target_tasks` tasks in all (each task
+// covers at least 16 mid combinations when there are that many, so that a
+// lane's prefix simulation is shared by enough mappings).
+inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count, uint64_t target_tasks) {
   bfk::Plan pl = base;
   const uint64_t last = first + count - 1;
   pl.first = (uint32_t)first;
@@ -140,7 +144,7 @@ inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count
   const uint64_t pm = (uint64_t)pl.pow3P * pl.pow3M;
   pl.i_lo = (uint32_t)(first / pm);
   pl.i_hi = (uint32_t)(last / pm);
-  const uint64_t s_lo = first / pl.pow3P, s_hi = last / pl.pow3P;
+  const uint64_t s_lo = first / pl.pow3P, s_hi = last / pl.pow3P;  // s = m + 3^M i
   if (s_lo == s_hi) {
     pl.p_lo = (uint32_t)(first % pl.pow3P);
     pl.p_hi = (uint32_t)(last % pl.pow3P);
@@ -148,6 +152,22 @@ inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count
     pl.p_lo = 0;
     pl.p_hi = pl.pow3P - 1;
   }
+  if (s_lo / pl.pow3M == s_hi / pl.pow3M) {
+    pl.m_lo = (uint32_t)(s_lo % pl.pow3M);
+    pl.m_hi = (uint32_t)(s_hi % pl.pow3M);
+  } else {
+    pl.m_lo = 0;
+    pl.m_hi = pl.pow3M - 1;
+  }
+  pl.groups = (pl.p_hi - pl.p_lo) / 32 + 1;
+  const uint64_t num_m = (uint64_t)pl.m_hi - pl.m_lo + 1;
+  uint64_t parts = (target_tasks + pl.groups - 1) / pl.groups;
+  const uint64_t min_chunk = num_m < 16 ? num_m : 16;
+  const uint64_t max_parts = (num_m + min_chunk - 1) / min_chunk;
+  if (parts > max_parts) parts = max_parts;
+  if (parts < 1) parts = 1;
+  pl.m_chunk = (uint32_t)((num_m + parts - 1) / parts);
+  pl.m_parts = (uint32_t)((num_m + pl.m_chunk - 1) / pl.m_chunk);
   return pl;
 }
 

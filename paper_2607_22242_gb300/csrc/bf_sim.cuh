@@ -31,8 +31,8 @@
 // `stop_mask` would become ready, leaving the state exactly as it was after
 // that instant's retirements.  Until then no tool of stop_mask has started,
 // so the history does not depend on their modes: the search kernels simulate
-// the prefix tools once per warp up to that instant and resume from the saved
-// state for every combination of the remaining tools' modes.
+// a prefix once up to that instant and resume from the saved state for every
+// combination of the remaining tools' modes.
 #pragma once
 
 #include <stdint.h>
@@ -67,21 +67,30 @@ struct Tables {
 };
 
 // How a search enumerates the mapping index idx = p + 3^P * (m + 3^M * i):
-//   prefix p -> the modes of tools [0, P), one per warp;
-//   mid m    -> the modes of tools [P, P+M), spread over the warp's lanes;
-//   inner i  -> the modes of the last I tools [Q, n), Q = P+M, walked by each lane.
-// The warp simulates its prefix once, up to the first instant a tool >= P
-// would become ready.  Tools below W0 are done by then (they are ancestors of
-// every tool >= P that can become ready first), so everything after that is
-// simulated over the window [W0, n) only, renumbered from 0.  With I > 0 each
-// lane saves its state again at the first instant an inner tool would become
-// ready and resumes it for every inner combination.
+//   prefix p -> the modes of tools [0, P);
+//   mid m    -> the modes of tools [P, P+M);
+//   inner i  -> the modes of the last I tools [Q, n), Q = P+M.
+// A warp task is 32 consecutive prefixes (one per lane) times a chunk of mid
+// combinations.  Each lane simulates its own prefix once, up to the first
+// instant a tool >= P would become ready, and saves that state.  Tools below
+// W0 are done by then (they are ancestors of every tool >= P that can become
+// ready first), so everything after it is simulated over the window [W0, n)
+// only, renumbered from 0.  The warp then walks its mid combinations (and each
+// one's inner combinations) in lockstep: the lanes differ only in the early
+// tools of their prefixes, so their window simulations mostly follow the same
+// control flow.  With I > 0 each lane saves its state again at the first
+// instant an inner tool would become ready and resumes it for every inner
+// combination.
 struct Plan {
   uint32_t P, M, I, W0;
   uint32_t pow3P, pow3M, pow3I;
   uint32_t p_lo, p_hi;      // prefixes this launch covers (inclusive)
+  uint32_t m_lo, m_hi;      // mid combinations this launch covers (inclusive)
   uint32_t i_lo, i_hi;      // inner combinations this launch covers (inclusive)
   uint32_t first, last;     // canonical index range (inclusive)
+  uint32_t groups;          // ceil((p_hi - p_lo + 1) / 32) prefix groups
+  uint32_t m_chunk;         // mid combinations per warp task
+  uint32_t m_parts;         // warp tasks per prefix group
 };
 
 // Tables read with a per-thread (dynamic) index, staged in shared memory:
@@ -301,68 +310,6 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
   }
 }
 
-// ---- saved state of a warp's prefix, restricted to the window [W0, n) --------
-// Stored once per warp in shared memory (every lane of the warp holds the same
-// prefix state) and reloaded by each lane for every suffix.
-struct Snapshot {
-  uint32_t ec[kMaxTools];
-  uint32_t eg[kMaxTools];
-  uint32_t done, pend, run_g, qwait, qrun, cand;
-  uint32_t T, V, L, k, tc, gmin;
-};
-
-// Save the window part of a prefix state (slots >= W0, renumbered).  Window
-// slots beyond the prefix state's last slot are written as unused slots (no
-// CPU end, stamp 0), so every slot a window simulation reads is defined.
-template <int NT>
-__device__ __forceinline__ void save_window(const State<NT>& s, uint32_t W0, uint32_t nw, Snapshot& out) {
-#pragma unroll
-  for (int i = 0; i < NT; ++i) {
-    if ((uint32_t)i >= W0) {
-      out.ec[i - W0] = s.ec[i];
-      out.eg[i - W0] = s.eg[i];
-    }
-  }
-  for (uint32_t j = (uint32_t)NT - W0; j < (uint32_t)kMaxTools; ++j) {
-    out.ec[j] = 0xFFFFFFFFu;
-    out.eg[j] = 0u;
-  }
-  const uint32_t wmask = (nw >= 32u) ? 0xFFFFFFFFu : ((1u << nw) - 1u);
-  out.done = (s.done >> W0) | ~wmask;
-  out.pend = (s.pend >> W0) & wmask;
-  out.run_g = s.run_g >> W0;
-  out.qwait = s.qwait >> W0;
-  out.qrun = s.qrun >> W0;
-  out.cand = (s.cand >> W0) & wmask;
-  out.T = s.T;
-  out.V = s.V;
-  out.L = s.L;
-  out.k = s.k;
-  out.tc = s.tc;
-  out.gmin = s.gmin;
-}
-
-template <int NW>
-__device__ __forceinline__ void load_window(const Snapshot& in, State<NW>& s) {
-#pragma unroll
-  for (int i = 0; i < NW; ++i) {
-    s.ec[i] = in.ec[i];
-    s.eg[i] = in.eg[i];
-  }
-  s.done = in.done;
-  s.pend = in.pend;
-  s.run_g = in.run_g;
-  s.qwait = in.qwait;
-  s.qrun = in.qrun;
-  s.cand = in.cand;
-  s.T = in.T;
-  s.V = in.V;
-  s.L = in.L;
-  s.k = in.k;
-  s.tc = in.tc;
-  s.gmin = in.gmin;
-}
-
 // Per-lane copy of a window state in shared memory, one word per row of a
 // [word][thread] array (`stride` = threads per block), so that a warp's
 // accesses to the same word hit 32 different banks.
@@ -413,6 +360,40 @@ __device__ __forceinline__ void load_lane(const uint32_t* slot, uint32_t stride,
   s.k = t[9 * stride];
   s.tc = t[10 * stride];
   s.gmin = t[11 * stride];
+}
+
+// Save the window part [W0, n) of a prefix state (NP slots) as a window state
+// of NW slots.  Window slots past the prefix state's last slot are written as
+// unused (no CPU end, stamp 0), so every slot a window run reads is defined.
+template <int NP, int NW>
+__device__ __forceinline__ void save_prefix_window(const State<NP>& s, uint32_t W0, uint32_t nw, uint32_t* slot,
+                                                   uint32_t stride) {
+#pragma unroll
+  for (int i = 0; i < NP; ++i) {
+    const uint32_t j = (uint32_t)i - W0;
+    if ((uint32_t)i >= W0 && j < (uint32_t)NW) {
+      slot[(2 * j) * stride] = s.ec[i];
+      slot[(2 * j + 1) * stride] = s.eg[i];
+    }
+  }
+  for (uint32_t j = (uint32_t)NP - W0; j < (uint32_t)NW; ++j) {
+    slot[(2 * j) * stride] = 0xFFFFFFFFu;
+    slot[(2 * j + 1) * stride] = 0u;
+  }
+  const uint32_t wmask = (nw >= 32u) ? 0xFFFFFFFFu : ((1u << nw) - 1u);
+  uint32_t* t = slot + (2 * NW) * stride;
+  t[0 * stride] = (s.done >> W0) | ~wmask;
+  t[1 * stride] = (s.pend >> W0) & wmask;
+  t[2 * stride] = s.run_g >> W0;
+  t[3 * stride] = s.qwait >> W0;
+  t[4 * stride] = s.qrun >> W0;
+  t[5 * stride] = (s.cand >> W0) & wmask;
+  t[6 * stride] = s.T;
+  t[7 * stride] = s.V;
+  t[8 * stride] = s.L;
+  t[9 * stride] = s.k;
+  t[10 * stride] = s.tc;
+  t[11 * stride] = s.gmin;
 }
 
 }  // namespace bfk
