@@ -61,15 +61,16 @@ __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, c
   const Digits dgw{dgp.now >> plan.W0, dgp.que >> plan.W0};
   const uint32_t m0 = plan.m_lo + part * plan.m_chunk;
   const uint32_t m1 = min(m0 + plan.m_chunk - 1u, plan.m_hi);
-  for (uint32_t m = m0; m <= m1; ++m) {
+  Digits dm = decode(m0, plan.M);
+  for (uint32_t m = m0; m <= m1; ++m, increment(dm)) {
     const uint64_t base = (uint64_t)p + (uint64_t)plan.pow3P * m;
-    uint32_t i_lo, i_hi;
-    if (!p_valid || !inner_range(plan, base, stride_i, &i_lo, &i_hi)) continue;
+    uint32_t i_lo = 0u, i_hi = plan.pow3I - 1u;
+    if (!p_valid) continue;
+    if (!plan.full && !inner_range(plan, base, stride_i, &i_lo, &i_hi)) continue;
     if (!ok) {  // every mapping with this prefix is infeasible
       for (uint32_t i = i_lo; i <= i_hi; ++i) sink((uint32_t)(base + stride_i * i), kInfeasible);
       continue;
     }
-    const Digits dm = decode(m, plan.M);
     const Digits dmid{dgw.now | (dm.now << shm), dgw.que | (dm.que << shm)};
     State<NW> w;
     uint32_t r = kRunInfeasible;

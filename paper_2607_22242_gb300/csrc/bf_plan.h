@@ -168,6 +168,7 @@ inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count
   if (parts < 1) parts = 1;
   pl.m_chunk = (uint32_t)((num_m + parts - 1) / parts);
   pl.m_parts = (uint32_t)((num_m + pl.m_chunk - 1) / pl.m_chunk);
+  pl.full = (first == 0 && last + 1 == (uint64_t)pl.pow3P * pl.pow3M * pl.pow3I) ? 1u : 0u;
   return pl;
 }
 

@@ -91,6 +91,7 @@ struct Plan {
   uint32_t groups;          // ceil((p_hi - p_lo + 1) / 32) prefix groups
   uint32_t m_chunk;         // mid combinations per warp task
   uint32_t m_parts;         // warp tasks per prefix group
+  uint32_t full;            // 1 if [first, last] is all of [0, 3^n)
 };
 
 // Tables read with a per-thread (dynamic) index, staged in shared memory:
@@ -133,6 +134,16 @@ __device__ __forceinline__ Digits decode(uint32_t v, uint32_t digits) {
   return d;
 }
 
+// v -> v + 1 on the two digit masks: trailing 2-digits wrap to 0, the next
+// digit steps 0 -> 1 or 1 -> 2.
+__device__ __forceinline__ void increment(Digits& d) {
+  const uint32_t low = ~d.que & (d.que + 1u);  // lowest digit that is not 2
+  d.que &= ~(low - 1u);
+  const uint32_t had = d.now & low;
+  d.now ^= low;
+  d.que |= had;
+}
+
 // Simulation state over NT slots.
 template <int NT>
 struct State {
@@ -143,7 +154,8 @@ struct State {
   uint32_t run_g;    // running GPU tools
   uint32_t qwait;    // queued tools waiting
   uint32_t qrun;     // the running queued tool (0 or one bit)
-  uint32_t cand;     // tools that may have become ready at T (successors of the last retirees)
+  uint32_t cand;     // tools that may have become ready at T (successors of the last
+                     // retirees); maintained by runs wider than 12 slots only
   uint32_t T, V, L, k;
   uint32_t tc;       // earliest CPU end (0xFFFFFFFF if none)
   uint32_t gmin;     // stamp of the first GPU tool to end (valid when k > 0)
@@ -173,6 +185,9 @@ template <int NT, typename TB>
 __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTables& sd, Digits dg,
                                         uint32_t stop_mask) {
   const uint32_t cpu_mask = tb.all_mask & ~(dg.now | dg.que);
+  // Narrow states test every pending slot for readiness at each admission;
+  // wide ones only test the successors of the tools that just retired (cand).
+  constexpr bool kScanReady = NT <= 12;
 #pragma unroll 1
   for (uint32_t events = 0;; ++events) {
     if (events > (uint32_t)NT + 1u) {
@@ -181,9 +196,13 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
     }
     // ---- admission at T ---------------------------------------------------
     uint32_t ready = 0u;
-    {
+    const uint32_t notdone = ~s.done;
+    if constexpr (kScanReady) {
+#pragma unroll
+      for (int i = 0; i < NT; ++i)
+        if ((s.pend & (1u << i)) && (tb.pred[i] & notdone) == 0u) ready |= 1u << i;
+    } else {
       uint32_t c = s.cand & s.pend;
-      const uint32_t notdone = ~s.done;
       while (c) {
         const int v = __ffs(c) - 1;
         c &= c - 1u;
@@ -281,7 +300,7 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
         if (s.ec[i] == s.T) {
           s.ec[i] = 0xFFFFFFFFu;
           s.done |= 1u << i;
-          s.cand |= tb.succ[i];
+          if constexpr (!kScanReady) s.cand |= tb.succ[i];
         }
         ntc = min(ntc, s.ec[i]);
       }
@@ -295,7 +314,7 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
           if (s.eg[i] == s.V) {
             rg |= 1u << i;
             s.L -= tb.vram[i];
-            s.cand |= tb.succ[i];
+            if constexpr (!kScanReady) s.cand |= tb.succ[i];
           } else {
             nrem = min(nrem, s.eg[i] - s.V);
           }
