@@ -233,9 +233,8 @@ def run_gpu(args):
     mean_ms = statistics.mean(step_ms)
     worst_ms = mean_ms
     if world > 1:
-        t = torch.tensor([mean_ms], device="cuda")
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        worst_ms = float(t.item())
+        from paper_2607_22242_gb300 import shard
+        worst_ms = shard.max_over_ranks(mean_ms)
     value = world * total / (worst_ms / 1e3)
     clocks = sampler.summary()
 

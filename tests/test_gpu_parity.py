@@ -283,3 +283,17 @@ def test_wait_timeout_is_reported():
             torch.cuda.synchronize()
         r = bf.search_best(h)
     assert r.feasible
+
+
+def test_shards_combine_to_full_search(golden):
+    """The per-rank pieces of a sharded search (shard.gpu_search_range on each
+    rank's range), combined by packed key, give the full N=19 optimum."""
+    from paper_2607_22242_gb300 import shard
+    scn = S.config3()
+    total = 3 ** scn.n
+    g = golden["3"]["summary"]
+    with bf.create_scenario(scn) as h:
+        search = shard.gpu_search_range(h)
+        for world in (2, 3, 8):
+            keys = [shard.pack_key(*search(*shard.shard_range(total, r, world))) for r in range(world)]
+            assert shard.unpack_key(min(keys)) == (g["best_index"], g["best_makespan"], True)
