@@ -46,6 +46,8 @@
  *     copied).  Device pointers are caller-owned CUDA device memory on the
  *     current device.  `cuda_stream` is a cudaStream_t (NULL = legacy default
  *     stream); work is ordered on it.
+ *   - A handle's scratch (search key, what-if list) is shared by the calls that
+ *     use it: calls on one handle must not overlap in time.
  *   - Blocking calls wait with a time limit (bf_set_wait_timeout_ms) and
  *     return BF_ETIMEOUT if it passes; the GPU work is then still in flight,
  *     and the scenario must not be destroyed until the stream has finished.
@@ -151,6 +153,40 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
  * scenario) per call.  Blocks until the results are on the host. */
 int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                     void* cuda_stream);
+
+/* Makespans and feasibility of an arbitrary list of mappings: d_makespan[j] and
+ * d_feasible[j] for mapping d_indices[j] (all three caller-owned device arrays
+ * of >= count elements).  An index >= 3^n yields makespan 0xFFFFFFFF and
+ * d_feasible = 0xFF.  Asynchronous on `cuda_stream`; count == 0 is a no-op.
+ * Used to score neighbourhoods of a mapping (bf_whatif) or any caller-chosen
+ * candidate set. */
+int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t count,
+                    uint32_t* d_makespan, uint8_t* d_feasible, void* cuda_stream);
+
+/* One probe of the runtime monitor's bounded what-if exploration. */
+typedef struct bf_probe {
+  uint64_t index;        /* canonical index of the probed mapping */
+  uint32_t makespan_us;  /* 0xFFFFFFFF if infeasible */
+  uint32_t feasible;     /* 0 = exceeds the VRAM budget ("exceed") */
+  uint8_t kind;          /* 0 = single-tool reprobe, 1 = swap reprobe */
+  uint8_t tool;          /* i: the tool moved (swap: the tool moved to gpu_now) */
+  uint8_t mode;          /* the new mode of tool i (bf_mode) */
+  uint8_t other;         /* swap: j, the gpu_now tool moved to gpu_queue; single: 0xFF */
+} bf_probe;
+
+#define BF_MAX_PROBES (2 * BF_MAX_TOOLS + BF_MAX_TOOLS * BF_MAX_TOOLS)
+
+/* The what-if probes of Algorithm 1 (lines 4-13, §3.2) around mapping
+ * base_index, scored on the model in one launch: for each tool i in index
+ * order and each alternative mode a != d_i (in the order cpu, gpu_now,
+ * gpu_queue), the single-tool reprobe d[i := a]; when that reprobe moves i to
+ * gpu_now and exceeds the budget (infeasible), then for each tool j on
+ * gpu_now in d (index order) the swap reprobe d[i := gpu_now, j := gpu_queue].
+ * Writes the probes in that order to out[0 .. *count) (at most
+ * BF_MAX_PROBES); BF_EINVAL if capacity is smaller than the number of probes,
+ * BF_ERANGE if base_index >= 3^n.  Blocks until the results are on the host. */
+int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32_t capacity,
+              uint32_t* count, void* cuda_stream);
 
 /* Largest batch bf_search_batch_noalloc accepts. */
 #define BF_NOALLOC_MAX_SCENARIOS 1024

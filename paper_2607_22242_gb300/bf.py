@@ -5,7 +5,8 @@ CUDA kernels.  PyTorch supplies device buffers (``eval_mappings`` outputs) and
 streams (``torch.cuda.current_stream()`` by default).  The functions mirror
 the C entry points without their ``bf_`` prefix: ``validate_desc``,
 ``create_scenario``, ``destroy_scenario``, ``eval_mappings``, ``search_best``,
-``search_range``, ``search_batch``, ``search_batch_noalloc``, ``set_wait_timeout_ms``, ``last_error``,
+``search_range``, ``search_batch``, ``search_batch_noalloc``, ``eval_indices``,
+``whatif``, ``set_wait_timeout_ms``, ``last_error``,
 ``version``.
 
 There is no CPU fallback: if ``libbf.so`` has not been built, or no CUDA
@@ -28,7 +29,8 @@ STATUS_NAMES = {0: "BF_OK", 1: "BF_EINVAL", 2: "BF_ERANGE", 3: "BF_ENOMEM", 4: "
 INFEASIBLE = 0xFFFFFFFF
 EXPORTED = ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
             "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc",
-            "bf_set_wait_timeout_ms", "bf_last_error", "bf_version")
+            "bf_eval_indices", "bf_whatif", "bf_set_wait_timeout_ms", "bf_last_error", "bf_version")
+MAX_PROBES = 2 * MAX_TOOLS + MAX_TOOLS * MAX_TOOLS
 NOALLOC_MAX_SCENARIOS = 1024
 
 
@@ -53,6 +55,26 @@ class CResult(ctypes.Structure):
     """``bf_result``."""
     _fields_ = [("index", ctypes.c_uint64), ("makespan_us", ctypes.c_uint32), ("feasible", ctypes.c_uint32),
                 ("mode", ctypes.c_uint8 * MAX_TOOLS)]
+
+
+class CProbe(ctypes.Structure):
+    """``bf_probe``."""
+    _fields_ = [("index", ctypes.c_uint64), ("makespan_us", ctypes.c_uint32), ("feasible", ctypes.c_uint32),
+                ("kind", ctypes.c_uint8), ("tool", ctypes.c_uint8), ("mode", ctypes.c_uint8),
+                ("other", ctypes.c_uint8)]
+
+
+@dataclasses.dataclass
+class Probe:
+    """One what-if probe of Algorithm 1: kind 'single' (tool -> mode) or 'swap'
+    (tool -> gpu_now, other -> gpu_queue)."""
+    kind: str
+    tool: int
+    mode: int
+    other: Optional[int]
+    index: int
+    makespan_us: int
+    feasible: bool
 
 
 @dataclasses.dataclass
@@ -83,8 +105,11 @@ def load(path: str = LIB_PATH):
     lib.bf_search_range.argtypes = [vp, u64, u64, ctypes.POINTER(CResult), vp]
     lib.bf_search_batch.argtypes = [ctypes.POINTER(Desc), u32, ctypes.POINTER(CResult), vp]
     lib.bf_search_batch_noalloc.argtypes = [ctypes.POINTER(Desc), u32, ctypes.POINTER(CResult), vp]
+    lib.bf_eval_indices.argtypes = [vp, vp, u64, vp, vp, vp]
+    lib.bf_whatif.argtypes = [vp, u64, ctypes.POINTER(CProbe), u32, ctypes.POINTER(u32), vp]
     for name in ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
-                 "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc"):
+                 "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc",
+                 "bf_eval_indices", "bf_whatif"):
         getattr(lib, name).restype = ctypes.c_int
     lib.bf_set_wait_timeout_ms.argtypes = [u32]
     lib.bf_set_wait_timeout_ms.restype = None
@@ -293,3 +318,40 @@ def search_batch_noalloc(scns: Sequence[Scenario], stream=None) -> List[Result]:
     scenarios per call, and calls that overlap on the GPU must not be issued.
     """
     return _batch_call(load().bf_search_batch_noalloc, scns, stream)
+
+
+def eval_indices(h: Union[ScenarioHandle, Scenario], indices, out_makespan=None, out_feasible=None, stream=None):
+    """Makespans (torch.int32, u32 bit patterns) and flags (torch.uint8; 0xFF for an
+    index outside [0, 3^n)) of the mappings in `indices` (a CUDA int64 tensor)."""
+    import torch
+    handle, owned = _handle(h)
+    try:
+        assert indices.is_cuda and indices.dtype == torch.int64 and indices.is_contiguous()
+        count = indices.numel()
+        if out_makespan is None:
+            out_makespan = torch.empty(count, dtype=torch.int32, device=indices.device)
+        if out_feasible is None:
+            out_feasible = torch.empty(count, dtype=torch.uint8, device=indices.device)
+        _check(load().bf_eval_indices(handle.ptr, ctypes.c_void_p(indices.data_ptr()), count,
+                                      ctypes.c_void_p(out_makespan.data_ptr()),
+                                      ctypes.c_void_p(out_feasible.data_ptr()),
+                                      ctypes.c_void_p(_stream_handle(stream))))
+        return out_makespan, out_feasible
+    finally:
+        if owned:
+            handle.close()
+
+
+def whatif(h: Union[ScenarioHandle, Scenario], base_index: int, stream=None) -> List[Probe]:
+    """The single-tool and swap reprobes of Algorithm 1 around `base_index`, scored on the GPU."""
+    handle, owned = _handle(h)
+    try:
+        out = (CProbe * MAX_PROBES)()
+        count = ctypes.c_uint32(0)
+        _check(load().bf_whatif(handle.ptr, base_index, out, MAX_PROBES, ctypes.byref(count),
+                                ctypes.c_void_p(_stream_handle(stream))))
+        return [Probe("swap" if p.kind else "single", p.tool, p.mode, None if p.kind == 0 else p.other,
+                      p.index, p.makespan_us, bool(p.feasible)) for p in out[:count.value]]
+    finally:
+        if owned:
+            handle.close()

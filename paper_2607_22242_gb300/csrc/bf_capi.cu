@@ -17,14 +17,25 @@
 #include "bf_launch.h"
 #include "bf_plan.h"
 
+// Per-handle scratch, one block on the device and a pinned mirror on the host:
+// the packed search key and the what-if probe list with its results.
+struct bf_scratch {
+  unsigned long long key;
+  uint64_t idx[BF_MAX_PROBES];
+  uint32_t ms[BF_MAX_PROBES];
+  uint8_t fe[BF_MAX_PROBES];
+};
+
 struct bf_scenario {
   bf_scenario_desc desc;
   bfk::Tables tables;   // all n tools
   bfk::Tables window;   // tools [W0, n), renumbered from 0
   bfk::Plan plan;       // enumeration split and window (see bfk::Plan), full range
   int device;
-  unsigned long long* d_key;  // device scratch: one packed search key
-  unsigned long long* h_key;  // pinned host copy of it
+  bf_scratch* d_scratch;      // device scratch
+  bf_scratch* h_scratch;      // pinned host mirror
+  unsigned long long* d_key;  // &d_scratch->key
+  unsigned long long* h_key;  // &h_scratch->key
 };
 
 namespace {
@@ -201,22 +212,24 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   build_tables(desc, &s->tables);
   split_and_window(s->tables, &s->plan, &s->window);
   cudaError_t e = cudaGetDevice(&s->device);
-  if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_key), sizeof(unsigned long long));
-  if (e == cudaSuccess) e = lib_malloc_host(reinterpret_cast<void**>(&s->h_key), sizeof(unsigned long long));
+  if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_scratch), sizeof(bf_scratch));
+  if (e == cudaSuccess) e = lib_malloc_host(reinterpret_cast<void**>(&s->h_scratch), sizeof(bf_scratch));
   if (e != cudaSuccess) {
     const int code = cuda_fail(e, "bf_create_scenario");
-    if (s->d_key) cudaFree(s->d_key);
+    if (s->d_scratch) cudaFree(s->d_scratch);
     delete s;
     return code;
   }
+  s->d_key = &s->d_scratch->key;
+  s->h_key = &s->h_scratch->key;
   *out = s;
   return BF_OK;
 }
 
 int bf_destroy_scenario(bf_scenario* scn) {
   if (!scn) return BF_OK;
-  cudaError_t e1 = scn->d_key ? cudaFree(scn->d_key) : cudaSuccess;
-  cudaError_t e2 = scn->h_key ? cudaFreeHost(scn->h_key) : cudaSuccess;
+  cudaError_t e1 = scn->d_scratch ? cudaFree(scn->d_scratch) : cudaSuccess;
+  cudaError_t e2 = scn->h_scratch ? cudaFreeHost(scn->h_scratch) : cudaSuccess;
   delete scn;
   if (e1 != cudaSuccess) return cuda_fail(e1, "bf_destroy_scenario");
   if (e2 != cudaSuccess) return cuda_fail(e2, "bf_destroy_scenario");
@@ -255,6 +268,114 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count, bf_r
     return fail(BF_ERANGE, "bf_search_range: [%llu, %llu+%llu) is outside [0, 3^%u)",
                 (unsigned long long)first, (unsigned long long)first, (unsigned long long)count, scn->desc.n);
   return run_search(scn, first, count, out, static_cast<cudaStream_t>(cuda_stream), "bf_search_range");
+}
+
+int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t count, uint32_t* d_makespan,
+                    uint8_t* d_feasible, void* cuda_stream) {
+  if (!scn) return fail(BF_EINVAL, "bf_eval_indices: scenario is NULL");
+  if (count == 0) return BF_OK;
+  if (!d_indices || !d_makespan || !d_feasible) return fail(BF_EINVAL, "bf_eval_indices: NULL buffer");
+  int sms = 0;
+  cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, scn->device);
+  if (e != cudaSuccess) return cuda_fail(e, "bf_eval_indices");
+  const uint64_t need = (count + bfk::kThreads - 1) / bfk::kThreads, cap = (uint64_t)sms * 16;
+  const int grid = (int)(need < cap ? need : cap);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  const uint64_t total = pow3(scn->desc.n);
+#define CALL(NW) launch_list_nw##NW(scn->tables, total, d_indices, count, d_makespan, d_feasible, grid, st)
+  BF_DISPATCH(bfk::bucket_for(scn->desc.n), CALL)
+#undef CALL
+  if (e != cudaSuccess) return cuda_fail(e, "bf_eval_indices");
+  return BF_OK;
+}
+
+int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32_t capacity, uint32_t* count,
+              void* cuda_stream) {
+  const char* who = "bf_whatif";
+  if (!scn || !out || !count) return fail(BF_EINVAL, "%s: NULL argument", who);
+  const uint32_t n = scn->desc.n;
+  const uint64_t total = pow3(n);
+  if (base_index >= total)
+    return fail(BF_ERANGE, "%s: base index %llu is outside [0, 3^%u)", who, (unsigned long long)base_index, n);
+  uint32_t d[BF_MAX_TOOLS];
+  uint64_t p3[BF_MAX_TOOLS];
+  {
+    uint64_t v = base_index, p = 1;
+    for (uint32_t i = 0; i < n; ++i, p *= 3) {
+      d[i] = (uint32_t)(v % 3);
+      v /= 3;
+      p3[i] = p;
+    }
+  }
+  // Candidates: every single-tool reprobe, then every swap that Algorithm 1
+  // could run (i not on gpu_now, j on gpu_now); which swaps it runs depends on
+  // the single reprobes' outcomes, so all are scored in the same launch.
+  bf_scratch* h = scn->h_scratch;
+  uint32_t nc = 0;
+  for (uint32_t i = 0; i < n; ++i)
+    for (uint32_t a = 0; a < 3; ++a)
+      if (a != d[i]) h->idx[nc++] = base_index - d[i] * p3[i] + a * p3[i];
+  const uint32_t n_single = nc;
+  for (uint32_t i = 0; i < n; ++i) {
+    if (d[i] == BF_MODE_GPU_NOW) continue;
+    for (uint32_t j = 0; j < n; ++j)
+      if (d[j] == BF_MODE_GPU_NOW)
+        h->idx[nc++] = base_index - d[i] * p3[i] + BF_MODE_GPU_NOW * p3[i] + (BF_MODE_GPU_QUEUE - BF_MODE_GPU_NOW) * p3[j];
+  }
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  bf_scratch* dv = scn->d_scratch;
+  cudaError_t e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) {
+#define CALL(NW) launch_list_nw##NW(scn->tables, total, dv->idx, nc, dv->ms, dv->fe, 1 + (int)(nc / bfk::kThreads), st)
+    BF_DISPATCH(bfk::bucket_for(n), CALL)
+#undef CALL
+  }
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h->ms, dv->ms, sizeof(uint32_t) * nc, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h->fe, dv->fe, nc, cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  const int rc = wait_stream(st, who);
+  if (rc != BF_OK) return rc;
+  // Assemble in Algorithm 1's order.
+  uint32_t k = 0, c = 0, sw = n_single;
+  bf_probe probes[BF_MAX_PROBES];
+  for (uint32_t i = 0; i < n; ++i) {
+    const uint32_t first_swap = sw;
+    uint32_t n_now = 0;
+    for (uint32_t j = 0; j < n; ++j) n_now += (d[j] == BF_MODE_GPU_NOW);
+    if (d[i] != BF_MODE_GPU_NOW) sw += n_now;
+    for (uint32_t a = 0; a < 3; ++a) {
+      if (a == d[i]) continue;
+      bf_probe& pr = probes[k++];
+      pr.index = h->idx[c];
+      pr.makespan_us = h->ms[c];
+      pr.feasible = h->fe[c] == 1;
+      pr.kind = 0;
+      pr.tool = (uint8_t)i;
+      pr.mode = (uint8_t)a;
+      pr.other = 0xFF;
+      const bool exceed = h->fe[c] != 1;
+      ++c;
+      if (exceed && a == BF_MODE_GPU_NOW) {
+        uint32_t s = first_swap;
+        for (uint32_t j = 0; j < n; ++j) {
+          if (d[j] != BF_MODE_GPU_NOW) continue;
+          bf_probe& q = probes[k++];
+          q.index = h->idx[s];
+          q.makespan_us = h->ms[s];
+          q.feasible = h->fe[s] == 1;
+          q.kind = 1;
+          q.tool = (uint8_t)i;
+          q.mode = BF_MODE_GPU_NOW;
+          q.other = (uint8_t)j;
+          ++s;
+        }
+      }
+    }
+  }
+  if (k > capacity) return fail(BF_EINVAL, "%s: %u probes do not fit in capacity %u", who, k, capacity);
+  std::memcpy(out, probes, sizeof(bf_probe) * k);
+  *count = k;
+  return BF_OK;
 }
 
 int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {

@@ -140,6 +140,34 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
   block_min_to(sink.best, keys + sc);
 }
 
+// Index-list evaluation: one mapping per thread (grid-stride), simulated from
+// the start over NP >= n slots.  Indices >= total are flagged 0xFF.
+template <int NP>
+__global__ void __launch_bounds__(kThreads) list_kernel(const __grid_constant__ Tables tb, uint64_t total,
+                                                        const uint64_t* __restrict__ idx, uint64_t count,
+                                                        uint32_t* __restrict__ ms_out, uint8_t* __restrict__ fe_out) {
+  __shared__ SmemTables sd;
+  load_smem_tables(tb, sd);
+  __syncthreads();
+  const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
+  for (uint64_t j = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; j < count; j += stride) {
+    const uint64_t x = idx[j];
+    uint32_t ms = kInfeasible;
+    uint8_t fe = 0xFFu;
+    if (x < total) {
+      const Digits d = decode((uint32_t)x, tb.n);
+      if ((d.que & tb.big_mask) == 0u) {
+        State<NP> s;
+        init_state(s, tb.all_mask);
+        if (run<NP>(s, tb, sd, d, 0u) == kRunFinished) ms = s.T;
+      }
+      fe = ms != kInfeasible;
+    }
+    ms_out[j] = ms;
+    fe_out[j] = fe;
+  }
+}
+
 // Allow the kernel more than the default 48 KB of dynamic shared memory (once per kernel).
 template <typename K>
 static cudaError_t allow_dyn_smem(K kernel, bool* done) {
@@ -182,6 +210,13 @@ cudaError_t BF_PASTE(launch_eval_nw, BF_NW)(const Tables& tb, const Tables& tw, 
 cudaError_t BF_PASTE(launch_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                               unsigned long long* key, cudaStream_t st) {
   BF_LAUNCH(search_kernel, tb.n <= (uint32_t)BF_NW, plan.I, blocks_for(plan), tb, tw, plan, key);
+}
+
+// Index lists run the whole scenario in one simulation: this unit handles n <= BF_NW.
+cudaError_t BF_PASTE(launch_list_nw, BF_NW)(const Tables& tb, uint64_t total, const uint64_t* idx, uint64_t count,
+                                            uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st) {
+  list_kernel<BF_NW><<<grid, kThreads, 0, st>>>(tb, total, idx, count, ms, fe);
+  return cudaGetLastError();
 }
 
 cudaError_t BF_PASTE(launch_batch_nw, BF_NW)(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,

@@ -37,7 +37,9 @@ inline int bucket_for(uint32_t w) {
                                    unsigned long long* key, cudaStream_t st);                        \
   cudaError_t launch_batch_nw##NW(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,           \
                                   uint32_t any_inner, uint32_t blocks_per_scenario,                  \
-                                  unsigned long long* keys, cudaStream_t st);
+                                  unsigned long long* keys, cudaStream_t st);                        \
+  cudaError_t launch_list_nw##NW(const Tables& tb, uint64_t total, const uint64_t* idx, uint64_t count, \
+                                 uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st);
 BF_FOR_EACH_BUCKET(BF_DECLARE_BUCKET)
 #undef BF_DECLARE_BUCKET
 

@@ -270,3 +270,35 @@ ALL_CHECKS = [
     check_contention_monotone, check_against_pysim, check_rational_bound,
     check_table1_speedups, check_table3_feasibility, check_fig7_probes,
 ]
+
+
+def check_fig7_whatif(lib):
+    """Figure 7's what-if block: around round 2's mapping (A:GN B:GN C:GQ D:CPU)
+    Algorithm 1 reprobes C -> gpu_now, which exceeds 1100 MB, and then swaps C
+    with each gpu_now tool; every probe printed there appears with its status
+    and, for swaps, the printed full mapping."""
+    from oracle import whatif as W
+    f7 = _load("paper_fig7.json")
+    tools = [dict(cpu_ms=t["cpu"], gpu_ms=t["gpu"], load_ms=t["load"], vram_mb=t["mem"]) for t in f7["tools"]]
+    scn = _fanout(tools, f7["budget_mb"])
+    base = S.mapping_index([GPU_NOW, GPU_NOW, GPU_QUEUE, CPU])
+    probes = W.whatif(scn, base, evaluate=lib.evaluate)
+    singles = {(p[1], p[2]): p for p in probes if p[0] == "single"}
+    swaps = {(p[1], p[3]): p for p in probes if p[0] == "swap"}
+    A, B, C, D = range(4)
+    assert len(singles) == 8
+    for (tool, mode), feasible in (((A, CPU), True), ((B, CPU), True), ((C, GPU_NOW), False), ((D, GPU_QUEUE), True)):
+        assert singles[(tool, mode)][6] == feasible, (tool, mode)
+    for (i, j), full in (((C, A), [GPU_QUEUE, GPU_NOW, GPU_NOW, CPU]), ((C, B), [GPU_NOW, GPU_QUEUE, GPU_NOW, CPU])):
+        p = swaps[(i, j)]
+        assert p[4] == S.mapping_index(full) and p[6], (i, j)
+    # Algorithm 1 swaps exactly the blocked tools with each tool on gpu_now.
+    blocked = [t for (t, m), p in singles.items() if m == GPU_NOW and not p[6]]
+    assert set(swaps) == {(i, j) for i in blocked for j in (A, B)}
+    # the swaps follow their single reprobe in the list
+    pos = {(p[0], p[1], p[2], p[3]): k for k, p in enumerate(probes)}
+    for i, j in swaps:
+        assert pos[("swap", i, GPU_NOW, j)] > pos[("single", i, GPU_NOW, None)]
+
+
+ALL_CHECKS.append(check_fig7_whatif)

@@ -297,3 +297,66 @@ def test_shards_combine_to_full_search(golden):
         for world in (2, 3, 8):
             keys = [shard.pack_key(*search(*shard.shard_range(total, r, world))) for r in range(world)]
             assert shard.unpack_key(min(keys)) == (g["best_index"], g["best_makespan"], True)
+
+
+# --------------------------------------------------------------------------- what-if and index lists
+
+def _same_probes(got, want):
+    return [(p.kind, p.tool, p.mode, p.other, p.index, p.makespan_us, p.feasible) for p in got] == want
+
+
+def test_whatif_matches_algorithm1_oracle():
+    from oracle import whatif as W
+    rng = np.random.default_rng(314)
+    for t in range(80):
+        n = int(rng.integers(1, 9))
+        scn = S.random_small(rng, n, tight=bool(t % 2), max_time=int(rng.choice([9, 900])))
+        with bf.create_scenario(scn) as h:
+            for base in rng.integers(0, 3 ** n, 4):
+                assert _same_probes(bf.whatif(h, int(base)), W.whatif(scn, int(base))), (scn, int(base))
+
+
+def test_whatif_fig7_and_config3():
+    from oracle import whatif as W
+    f7 = pins._load("paper_fig7.json")
+    tools = [dict(cpu_ms=t["cpu"], gpu_ms=t["gpu"], load_ms=t["load"], vram_mb=t["mem"]) for t in f7["tools"]]
+    scn = pins._fanout(tools, f7["budget_mb"])
+    base = S.mapping_index([1, 1, 2, 0])
+    with bf.create_scenario(scn) as h:
+        assert _same_probes(bf.whatif(h, base), W.whatif(scn, base))
+    scn = S.config3()
+    rng = np.random.default_rng(3)
+    with bf.create_scenario(scn) as h:
+        for base in [575638191, 0, 3 ** 19 - 1] + [int(v) for v in rng.integers(0, 3 ** 19, 5)]:
+            got = bf.whatif(h, base)
+            assert len(got) <= bf.MAX_PROBES
+            assert _same_probes(got, W.whatif(scn, base)), base
+
+
+def test_eval_indices_matches_oracle():
+    import torch
+    rng = np.random.default_rng(99)
+    for cfg in (1, 2, 3):
+        scn = S.config(cfg)
+        total = 3 ** scn.n
+        idx = rng.integers(0, total, 20_000).astype(np.int64)
+        idx[:3] = [0, total - 1, total]          # includes one index past the end
+        with bf.create_scenario(scn) as h:
+            ms, fe = bf.eval_indices(h, torch.from_numpy(idx).cuda())
+            torch.cuda.synchronize()
+        ms = ms.cpu().numpy().view(np.uint32)
+        fe = fe.cpu().numpy()
+        assert fe[2] == 0xFF and ms[2] == INF
+        for j in list(range(3)) + [int(v) for v in rng.integers(3, idx.size, 400)]:
+            if idx[j] >= total:
+                continue
+            want = oracle.evaluate(scn, int(idx[j]))
+            assert (int(ms[j]), int(fe[j])) == (want, int(want != INF)), (cfg, int(idx[j]))
+
+
+def test_whatif_range_error():
+    scn = S.config0()
+    with bf.create_scenario(scn) as h:
+        with pytest.raises(bf.BfError) as ei:
+            bf.whatif(h, 3 ** 8)
+        assert ei.value.code == bf.BF_ERANGE
