@@ -153,10 +153,10 @@ struct State {
   uint32_t pend;     // not yet ready
   uint32_t run_g;    // running GPU tools
   uint32_t qwait;    // queued tools waiting
-  uint32_t qrun;     // the running queued tool (0 or one bit)
   uint32_t cand;     // tools that may have become ready at T (successors of the last
                      // retirees); maintained by runs wider than 12 slots only
-  uint32_t T, V, L, k;
+  uint32_t T, V, L;  // (k, the number of running GPU tools, is popc(run_g); the running
+                     // queued tool, if any, is run_g & the gpu_queue digits)
   uint32_t tc;       // earliest CPU end (0xFFFFFFFF if none)
   uint32_t gmin;     // stamp of the first GPU tool to end (valid when k > 0)
 };
@@ -170,9 +170,9 @@ __device__ __forceinline__ void init_state(State<NT>& s, uint32_t all_mask) {
   }
   s.done = ~all_mask;
   s.pend = all_mask;
-  s.run_g = s.qwait = s.qrun = 0u;
+  s.run_g = s.qwait = 0u;
   s.cand = all_mask;  // at T = 0 every tool is a candidate
-  s.T = s.V = s.L = s.k = 0u;
+  s.T = s.V = s.L = 0u;
   s.tc = 0xFFFFFFFFu;
   s.gmin = 0u;
 }
@@ -234,9 +234,8 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
             wmin = min(wmin, tb.wnow[i]);
           }
         }
-        if (s.k == 0u || wmin < s.gmin - s.V) s.gmin = s.V + wmin;
+        if (s.run_g == 0u || wmin < s.gmin - s.V) s.gmin = s.V + wmin;
         s.run_g |= rg;
-        s.k += __popc(rg);
         if (s.L > tb.budget) return kRunInfeasible;
       }
       if (rq) {
@@ -246,7 +245,7 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
         s.qwait |= rq;
       }
     }
-    if (s.qwait && !s.qrun) {
+    if (s.qwait && !(s.run_g & dg.que)) {
       // Queue head: earliest ready time, ties to the lower index.
       uint32_t best = 0xFFFFFFFFu, hm = 0u, hv = 0u, hw = 0u;
 #pragma unroll
@@ -262,20 +261,19 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
 #pragma unroll
         for (int i = 0; i < NT; ++i)
           if (hm & (1u << i)) s.eg[i] = s.V + hw;
-        if (s.k == 0u || hw < s.gmin - s.V) s.gmin = s.V + hw;
+        if (s.run_g == 0u || hw < s.gmin - s.V) s.gmin = s.V + hw;
         s.L += hv;
-        s.k += 1u;
         s.run_g |= hm;
-        s.qrun = hm;
         s.qwait &= ~hm;
       }
     }
     if (s.done == 0xFFFFFFFFu) return kRunFinished;
 
     // ---- next event ---------------------------------------------------------
-    const uint32_t kk = min(s.k, (uint32_t)kMaxTools);  // k <= n always; keeps indexing in bounds
+    const uint32_t k = __popc(s.run_g);
+    const uint32_t kk = min(k, (uint32_t)kMaxTools);  // k <= n always; keeps indexing in bounds
     bool gpu_event = false;
-    if (s.k) {
+    if (k) {
       const uint32_t rem = s.gmin - s.V;
       const uint64_t tg = (uint64_t)s.T + (((uint64_t)rem * sd.f[kk] + 0xFFFFFull) >> 20);
       if (tg <= (uint64_t)s.tc) {
@@ -322,8 +320,6 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
       }
       s.run_g &= ~rg;
       s.done |= rg;
-      s.k -= __popc(rg);
-      if (rg & s.qrun) s.qrun = 0u;
       s.gmin = s.V + nrem;
     }
   }
@@ -334,7 +330,7 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
 // accesses to the same word hit 32 different banks.
 template <int NW>
 struct LaneWords {
-  static constexpr int value = 2 * NW + 12;
+  static constexpr int value = 2 * NW + 10;
 };
 
 template <int NW>
@@ -349,14 +345,12 @@ __device__ __forceinline__ void save_lane(const State<NW>& s, uint32_t* slot, ui
   t[1 * stride] = s.pend;
   t[2 * stride] = s.run_g;
   t[3 * stride] = s.qwait;
-  t[4 * stride] = s.qrun;
-  t[5 * stride] = s.cand;
-  t[6 * stride] = s.T;
-  t[7 * stride] = s.V;
-  t[8 * stride] = s.L;
-  t[9 * stride] = s.k;
-  t[10 * stride] = s.tc;
-  t[11 * stride] = s.gmin;
+  t[4 * stride] = s.cand;
+  t[5 * stride] = s.T;
+  t[6 * stride] = s.V;
+  t[7 * stride] = s.L;
+  t[8 * stride] = s.tc;
+  t[9 * stride] = s.gmin;
 }
 
 template <int NW>
@@ -371,14 +365,12 @@ __device__ __forceinline__ void load_lane(const uint32_t* slot, uint32_t stride,
   s.pend = t[1 * stride];
   s.run_g = t[2 * stride];
   s.qwait = t[3 * stride];
-  s.qrun = t[4 * stride];
-  s.cand = t[5 * stride];
-  s.T = t[6 * stride];
-  s.V = t[7 * stride];
-  s.L = t[8 * stride];
-  s.k = t[9 * stride];
-  s.tc = t[10 * stride];
-  s.gmin = t[11 * stride];
+  s.cand = t[4 * stride];
+  s.T = t[5 * stride];
+  s.V = t[6 * stride];
+  s.L = t[7 * stride];
+  s.tc = t[8 * stride];
+  s.gmin = t[9 * stride];
 }
 
 // Save the window part [W0, n) of a prefix state (NP slots) as a window state
@@ -405,14 +397,12 @@ __device__ __forceinline__ void save_prefix_window(const State<NP>& s, uint32_t 
   t[1 * stride] = (s.pend >> W0) & wmask;
   t[2 * stride] = s.run_g >> W0;
   t[3 * stride] = s.qwait >> W0;
-  t[4 * stride] = s.qrun >> W0;
-  t[5 * stride] = (s.cand >> W0) & wmask;
-  t[6 * stride] = s.T;
-  t[7 * stride] = s.V;
-  t[8 * stride] = s.L;
-  t[9 * stride] = s.k;
-  t[10 * stride] = s.tc;
-  t[11 * stride] = s.gmin;
+  t[4 * stride] = (s.cand >> W0) & wmask;
+  t[5 * stride] = s.T;
+  t[6 * stride] = s.V;
+  t[7 * stride] = s.L;
+  t[8 * stride] = s.tc;
+  t[9 * stride] = s.gmin;
 }
 
 }  // namespace bfk

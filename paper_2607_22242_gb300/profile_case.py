@@ -3,6 +3,8 @@
   python -m paper_2607_22242_gb300.profile_case --kernel search --config 3 --count 67108864 --reps 3
   python -m paper_2607_22242_gb300.profile_case --kernel eval --config 2 --count 16777216
   python -m paper_2607_22242_gb300.profile_case --kernel batch --batch 1024
+  python -m paper_2607_22242_gb300.profile_case --kernel list --config 3 --count 16777216
+  python -m paper_2607_22242_gb300.profile_case --kernel whatif --config 3 --reps 20
 
 Prints one line per repetition (CUDA-event time of the call and mappings/s).
 Sized so that a profiler capture of one launch stays short.
@@ -20,7 +22,7 @@ if ROOT not in sys.path:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=("search", "eval", "batch"), default="search")
+    ap.add_argument("--kernel", choices=("search", "eval", "batch", "list", "whatif"), default="search")
     ap.add_argument("--config", type=int, default=3)
     ap.add_argument("--first", type=int, default=0)
     ap.add_argument("--count", type=int, default=1 << 26)
@@ -47,6 +49,16 @@ def main():
         h = bf.create_scenario(scn)
         if args.kernel == "search":
             call = lambda: bf.search_range(h, args.first, count, stream)
+        elif args.kernel == "list":  # uniformly random mapping indices of the whole space
+            g = torch.Generator(device="cuda").manual_seed(1)
+            idx = torch.randint(0, 3 ** scn.n, (count,), device="cuda", generator=g, dtype=torch.int64)
+            ms = torch.empty(count, dtype=torch.int32, device="cuda")
+            fe = torch.empty(count, dtype=torch.uint8, device="cuda")
+            call = lambda: bf.eval_indices(h, idx, ms, fe, stream)
+        elif args.kernel == "whatif":  # around the optimum of the scenario
+            base = bf.search_best(h, stream).index
+            work = len(bf.whatif(h, base, stream))
+            call = lambda: bf.whatif(h, base, stream)
         else:
             ms = torch.empty(count, dtype=torch.int32, device="cuda")
             fe = torch.empty(count, dtype=torch.uint8, device="cuda")
