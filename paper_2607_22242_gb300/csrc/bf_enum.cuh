@@ -29,10 +29,13 @@ __device__ __forceinline__ bool inner_range(const Plan& plan, uint64_t base, uin
 // slotA / slotB are this lane's shared-memory areas of LaneWords<NW> words
 // (stride `stride`) for the state at the prefix checkpoint and at the inner
 // checkpoint.
+// rt / rtw are the readiness tables of the full and window tables (used when
+// NP / NW <= kReadyTableSlots).
 template <int NP, int NW, typename TBF, typename TBW, typename Sink>
-__device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, const TBW& tw,
-                                          const SmemTables& sdw, const Plan& plan, uint32_t g, uint32_t part,
-                                          uint32_t* slotA, uint32_t* slotB, uint32_t stride, Sink& sink) {
+__device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, const uint32_t* rt, const TBW& tw,
+                                          const SmemTables& sdw, const uint32_t* rtw, const Plan& plan, uint32_t g,
+                                          uint32_t part, uint32_t* slotA, uint32_t* slotB, uint32_t stride,
+                                          Sink& sink) {
   const uint32_t lane = threadIdx.x & 31u;
   const uint64_t p64 = (uint64_t)plan.p_lo + 32ull * g + lane;
   const bool p_valid = p64 <= plan.p_hi;
@@ -48,7 +51,7 @@ __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, c
       State<NP> s;
       init_state(s, tb.all_mask);
       const uint32_t later = tb.all_mask & ~((1u << plan.P) - 1u);
-      ok = run<NP>(s, tb, sd, dgp, later) == kRunStopped;
+      ok = run<NP>(s, tb, sd, rt, dgp, later) == kRunStopped;
       if (ok) save_prefix_window<NP, NW>(s, plan.W0, tb.n - plan.W0, slotA, stride);
     }
   }
@@ -76,7 +79,7 @@ __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, c
     uint32_t r = kRunInfeasible;
     if ((dmid.que & tw.big_mask) == 0u) {
       load_lane(slotA, stride, w);
-      r = run<NW>(w, tw, sdw, dmid, inner_mask);
+      r = run<NW>(w, tw, sdw, rtw, dmid, inner_mask);
     }
     if (plan.I == 0u) {  // no inner level: the run went to the end
       sink((uint32_t)base, r == kRunFinished ? w.T : kInfeasible);
@@ -93,7 +96,7 @@ __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, c
       uint32_t ms = kInfeasible;
       if ((dg.que & tw.big_mask) == 0u) {
         if (i != i_lo) load_lane(slotB, stride, w);
-        ms = run<NW>(w, tw, sdw, dg, 0u) == kRunFinished ? w.T : kInfeasible;
+        ms = run<NW>(w, tw, sdw, rtw, dg, 0u) == kRunFinished ? w.T : kInfeasible;
       }
       sink((uint32_t)(base + stride_i * i), ms);
     }

@@ -85,14 +85,17 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) eval_kernel(const __g
                                                                        uint8_t* __restrict__ fe_out) {
   extern __shared__ uint32_t lane_state[];
   __shared__ SmemTables sd, sdw;
+  __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
+  fill_ready_table<NP>(tb, rt);
+  fill_ready_table<BF_NW>(tw, rtw);
   __syncthreads();
   const uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (task >= plan.groups * plan.m_parts) return;  // no block-level synchronisation follows
   StoreSink sink{plan.first, ms_out, fe_out};
-  warp_task<NP, BF_NW>(tb, sd, tw, sdw, plan, task / plan.m_parts, task % plan.m_parts, lane_state + threadIdx.x,
-                       lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
+  warp_task<NP, BF_NW>(tb, sd, rt, tw, sdw, rtw, plan, task / plan.m_parts, task % plan.m_parts,
+                       lane_state + threadIdx.x, lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
 }
 
 template <int NP>
@@ -102,14 +105,17 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) search_kernel(const _
                                                                          unsigned long long* key) {
   extern __shared__ uint32_t lane_state[];
   __shared__ SmemTables sd, sdw;
+  __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
+  fill_ready_table<NP>(tb, rt);
+  fill_ready_table<BF_NW>(tw, rtw);
   __syncthreads();
   const uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5);
   MinKeySink sink;
   if (task < plan.groups * plan.m_parts)
-    warp_task<NP, BF_NW>(tb, sd, tw, sdw, plan, task / plan.m_parts, task % plan.m_parts, lane_state + threadIdx.x,
-                         lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
+    warp_task<NP, BF_NW>(tb, sd, rt, tw, sdw, rtw, plan, task / plan.m_parts, task % plan.m_parts,
+                         lane_state + threadIdx.x, lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
   block_min_to(sink.best, key);
 }
 
@@ -121,6 +127,7 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
   extern __shared__ uint32_t lane_state[];
   __shared__ BatchRecord rec;
   __shared__ SmemTables sd, sdw;
+  __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
   const uint32_t sc = blockIdx.x / blocks_per_scenario;
   const uint32_t b = blockIdx.x - sc * blocks_per_scenario;
   {
@@ -131,12 +138,15 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
   __syncthreads();
   load_smem_tables(rec.full, sd);
   load_smem_tables(rec.window, sdw);
+  fill_ready_table<NP>(rec.full, rt);
+  fill_ready_table<BF_NW>(rec.window, rtw);
   __syncthreads();
   const uint32_t task = b * kWarps + (threadIdx.x >> 5);
   MinKeySink sink;
   if (task < rec.plan.groups * rec.plan.m_parts)
-    warp_task<NP, BF_NW>(rec.full, sd, rec.window, sdw, rec.plan, task / rec.plan.m_parts, task % rec.plan.m_parts,
-                         lane_state + threadIdx.x, lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
+    warp_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, task / rec.plan.m_parts,
+                         task % rec.plan.m_parts, lane_state + threadIdx.x,
+                         lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
   block_min_to(sink.best, keys + sc);
 }
 
@@ -147,7 +157,9 @@ __global__ void __launch_bounds__(kThreads) list_kernel(const __grid_constant__ 
                                                         const uint64_t* __restrict__ idx, uint64_t count,
                                                         uint32_t* __restrict__ ms_out, uint8_t* __restrict__ fe_out) {
   __shared__ SmemTables sd;
+  __shared__ uint32_t rt[ReadyTable<NP>::size];
   load_smem_tables(tb, sd);
+  fill_ready_table<NP>(tb, rt);
   __syncthreads();
   const uint64_t stride = (uint64_t)gridDim.x * blockDim.x;
   for (uint64_t j = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x; j < count; j += stride) {
@@ -159,7 +171,7 @@ __global__ void __launch_bounds__(kThreads) list_kernel(const __grid_constant__ 
       if ((d.que & tb.big_mask) == 0u) {
         State<NP> s;
         init_state(s, tb.all_mask);
-        if (run<NP>(s, tb, sd, d, 0u) == kRunFinished) ms = s.T;
+        if (run<NP>(s, tb, sd, rt, d, 0u) == kRunFinished) ms = s.T;
       }
       fe = ms != kInfeasible;
     }

@@ -181,12 +181,39 @@ __device__ __forceinline__ void init_state(State<NT>& s, uint32_t all_mask) {
 // makespan is s.T), the mapping proves infeasible (kRunInfeasible), or a tool
 // of `stop_mask` would become ready (kRunStopped, state left before that
 // admission).  A stalled run reports kRunFinished with s.T = kStalled.
+// Readiness tables: for states of at most kReadyTableSlots slots, entry e of
+// the table is the set of tools all of whose predecessors are in the set e,
+// so an admission finds its ready tools with one shared-memory load.
+constexpr int kReadyTableSlots = 10;
+
+template <int NT>
+struct ReadyTable {
+  static constexpr int size = (NT <= kReadyTableSlots) ? (1 << NT) : 1;
+};
+
+// Fill a readiness table for NT slots (block-cooperative; tools >= n never
+// matter because they are never pending).
 template <int NT, typename TB>
-__device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTables& sd, Digits dg,
-                                        uint32_t stop_mask) {
+__device__ __forceinline__ void fill_ready_table(const TB& tb, uint32_t* table) {
+  if constexpr (NT <= kReadyTableSlots) {
+    for (uint32_t e = threadIdx.x; e < (1u << NT); e += blockDim.x) {
+      uint32_t r = 0u;
+#pragma unroll
+      for (int v = 0; v < NT; ++v)
+        if ((tb.pred[v] & ~e) == 0u) r |= 1u << v;
+      table[e] = r;
+    }
+  }
+}
+
+template <int NT, typename TB>
+__device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTables& sd, const uint32_t* ready_table,
+                                        Digits dg, uint32_t stop_mask) {
   const uint32_t cpu_mask = tb.all_mask & ~(dg.now | dg.que);
-  // Narrow states test every pending slot for readiness at each admission;
-  // wide ones only test the successors of the tools that just retired (cand).
+  // Narrow states look their ready tools up (up to 10 slots) or test every
+  // pending slot (up to 12); wide ones only test the successors of the tools
+  // that just retired (cand).
+  constexpr bool kTableReady = NT <= kReadyTableSlots;
   constexpr bool kScanReady = NT <= 12;
 #pragma unroll 1
   for (uint32_t events = 0;; ++events) {
@@ -197,7 +224,9 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
     // ---- admission at T ---------------------------------------------------
     uint32_t ready = 0u;
     const uint32_t notdone = ~s.done;
-    if constexpr (kScanReady) {
+    if constexpr (kTableReady) {
+      ready = s.pend & ready_table[s.done & ((1u << NT) - 1u)];
+    } else if constexpr (kScanReady) {
 #pragma unroll
       for (int i = 0; i < NT; ++i)
         if ((s.pend & (1u << i)) && (tb.pred[i] & notdone) == 0u) ready |= 1u << i;
