@@ -35,11 +35,13 @@ def _sources():
 
 
 def _fingerprint(extra) -> str:
+    """Hash of the kernel sources and flags, independent of where the repository lives."""
     h = hashlib.sha256()
     for path in _sources():
         with open(path, "rb") as fh:
-            h.update(path.encode() + fh.read())
-    h.update(" ".join(ARCH + NVCC_FLAGS + list(extra)).encode())
+            h.update(os.path.basename(path).encode() + fh.read())
+    flags = [f for f in NVCC_FLAGS if not f.startswith("-I")]
+    h.update(" ".join(ARCH + flags + list(extra)).encode())
     return h.hexdigest()
 
 
