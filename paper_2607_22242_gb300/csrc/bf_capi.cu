@@ -50,7 +50,7 @@ using bfk::host::split_and_window;
 constexpr uint64_t kSearchTasks = 32768;
 
 thread_local std::string g_error;
-uint32_t g_wait_timeout_ms = 600000;
+std::atomic<uint32_t> g_wait_timeout_ms{600000};
 
 int fail(int code, const char* fmt, ...) {
   char buf[512];
@@ -71,12 +71,12 @@ int cuda_fail(cudaError_t e, const char* what) {
 // Allocation-failure injection for host-side fault tests: BF_FAIL_ALLOC=<n>
 // makes the n-th library allocation of the process (1-based) fail.
 bool inject_alloc_failure() {
-  static int countdown = [] {
+  static std::atomic<int> countdown{[] {
     const char* s = std::getenv("BF_FAIL_ALLOC");
     return s ? std::atoi(s) : 0;
-  }();
-  if (countdown <= 0) return false;
-  return --countdown == 0;
+  }()};
+  if (countdown.load(std::memory_order_relaxed) <= 0) return false;
+  return countdown.fetch_sub(1) == 1;
 }
 
 cudaError_t lib_malloc(void** p, size_t bytes) {
@@ -133,11 +133,11 @@ int wait_stream(cudaStream_t st, const char* who) {
     const cudaError_t e = cudaStreamQuery(st);
     if (e == cudaSuccess) return BF_OK;
     if (e != cudaErrorNotReady) return cuda_fail(e, who);
-    if (g_wait_timeout_ms) {
+    const uint32_t limit = g_wait_timeout_ms.load(std::memory_order_relaxed);
+    if (limit) {
       const auto ms = std::chrono::duration_cast<std::chrono::milliseconds>(
                           std::chrono::steady_clock::now() - t0).count();
-      if (ms > (long long)g_wait_timeout_ms)
-        return fail(BF_ETIMEOUT, "%s: GPU work not finished after %u ms", who, g_wait_timeout_ms);
+      if (ms > (long long)limit) return fail(BF_ETIMEOUT, "%s: GPU work not finished after %u ms", who, limit);
     }
     std::this_thread::sleep_for(std::chrono::microseconds(20));
   }
@@ -417,9 +417,14 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
     BF_DISPATCH(bfk::bucket_for(wmax), CALL)
 #undef CALL
   }
-  if (e == cudaSuccess) e = cudaMemcpyAsync(keys.data(), d_keys, kbytes, cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
+  // Bounded wait first: a copy into pageable memory would block without limit.
   if (rc == BF_OK) rc = wait_stream(st, "bf_search_batch");
+  if (rc == BF_OK) {
+    e = cudaMemcpyAsync(keys.data(), d_keys, kbytes, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);
+    if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
+  }
   if (rc != BF_ETIMEOUT) {  // on timeout the kernel may still use the scratch: leak it rather than free in-use memory
     if (d_recs) cudaFree(d_recs);
     if (d_keys) cudaFree(d_keys);
@@ -545,7 +550,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
   return BF_OK;
 }
 
-void bf_set_wait_timeout_ms(uint32_t ms) { g_wait_timeout_ms = ms; }
+void bf_set_wait_timeout_ms(uint32_t ms) { g_wait_timeout_ms.store(ms, std::memory_order_relaxed); }
 
 const char* bf_last_error(void) { return g_error.c_str(); }
 
