@@ -154,6 +154,19 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
 int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                     void* cuda_stream);
 
+/* Same result as bf_search_best (the feasible mapping of lowest makespan over
+ * all 3^n, ties to the lowest index), found by branch and bound instead of
+ * full enumeration.  An incumbent is taken from a few mappings (hint_index if
+ * < 3^n, all-cpu, all-gpu_now, all-gpu_queue, each tool on its isolated-faster
+ * device); a prefix (or a mid combination) is skipped when the time at which
+ * its remaining tools can first start, plus the longest path through them in
+ * minimum isolated durations min(c, g + x), exceeds the incumbent's makespan
+ * -- no mode, contention or queueing makes a tool faster than that.  Exact:
+ * the optimum and all its ties are never skipped.  Allocates a 4-byte-per-
+ * prefix buffer in the handle on first use.  Blocks until the result is on
+ * the host. */
+int bf_search_pruned(const bf_scenario* scn, uint64_t hint_index, bf_result* out, void* cuda_stream);
+
 /* Makespans and feasibility of an arbitrary list of mappings: d_makespan[j] and
  * d_feasible[j] for mapping d_indices[j] (all three caller-owned device arrays
  * of >= count elements).  An index >= 3^n yields makespan 0xFFFFFFFF and

@@ -6,7 +6,7 @@ streams (``torch.cuda.current_stream()`` by default).  The functions mirror
 the C entry points without their ``bf_`` prefix: ``validate_desc``,
 ``create_scenario``, ``destroy_scenario``, ``eval_mappings``, ``search_best``,
 ``search_range``, ``search_batch``, ``search_batch_noalloc``, ``eval_indices``,
-``whatif``, ``set_wait_timeout_ms``, ``last_error``,
+``whatif``, ``search_pruned``, ``set_wait_timeout_ms``, ``last_error``,
 ``version``.
 
 There is no CPU fallback: if ``libbf.so`` has not been built, or no CUDA
@@ -29,7 +29,8 @@ STATUS_NAMES = {0: "BF_OK", 1: "BF_EINVAL", 2: "BF_ERANGE", 3: "BF_ENOMEM", 4: "
 INFEASIBLE = 0xFFFFFFFF
 EXPORTED = ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
             "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc",
-            "bf_eval_indices", "bf_whatif", "bf_set_wait_timeout_ms", "bf_last_error", "bf_version")
+            "bf_eval_indices", "bf_whatif", "bf_search_pruned", "bf_set_wait_timeout_ms", "bf_last_error",
+            "bf_version")
 MAX_PROBES = 2 * MAX_TOOLS + MAX_TOOLS * MAX_TOOLS
 NOALLOC_MAX_SCENARIOS = 1024
 
@@ -107,9 +108,10 @@ def load(path: str = LIB_PATH):
     lib.bf_search_batch_noalloc.argtypes = [ctypes.POINTER(Desc), u32, ctypes.POINTER(CResult), vp]
     lib.bf_eval_indices.argtypes = [vp, vp, u64, vp, vp, vp]
     lib.bf_whatif.argtypes = [vp, u64, ctypes.POINTER(CProbe), u32, ctypes.POINTER(u32), vp]
+    lib.bf_search_pruned.argtypes = [vp, u64, ctypes.POINTER(CResult), vp]
     for name in ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
                  "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc",
-                 "bf_eval_indices", "bf_whatif"):
+                 "bf_eval_indices", "bf_whatif", "bf_search_pruned"):
         getattr(lib, name).restype = ctypes.c_int
     lib.bf_set_wait_timeout_ms.argtypes = [u32]
     lib.bf_set_wait_timeout_ms.restype = None
@@ -352,6 +354,19 @@ def whatif(h: Union[ScenarioHandle, Scenario], base_index: int, stream=None) -> 
                                 ctypes.c_void_p(_stream_handle(stream))))
         return [Probe("swap" if p.kind else "single", p.tool, p.mode, None if p.kind == 0 else p.other,
                       p.index, p.makespan_us, bool(p.feasible)) for p in out[:count.value]]
+    finally:
+        if owned:
+            handle.close()
+
+
+def search_pruned(h: Union[ScenarioHandle, Scenario], hint_index: Optional[int] = None, stream=None) -> Result:
+    """The optimum of :func:`search_best`, found by branch and bound (exact)."""
+    handle, owned = _handle(h)
+    try:
+        r = CResult()
+        hint = (1 << 64) - 1 if hint_index is None else hint_index
+        _check(load().bf_search_pruned(handle.ptr, hint, ctypes.byref(r), ctypes.c_void_p(_stream_handle(stream))))
+        return _result(r, handle.scenario.n)
     finally:
         if owned:
             handle.close()

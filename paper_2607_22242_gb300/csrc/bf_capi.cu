@@ -21,6 +21,8 @@
 // the packed search key and the what-if probe list with its results.
 struct bf_scratch {
   unsigned long long key;
+  uint32_t survivors;   // pruned search: number of surviving prefixes
+  uint32_t pad;
   uint64_t idx[BF_MAX_PROBES];
   uint32_t ms[BF_MAX_PROBES];
   uint8_t fe[BF_MAX_PROBES];
@@ -36,6 +38,7 @@ struct bf_scenario {
   bf_scratch* h_scratch;      // pinned host mirror
   unsigned long long* d_key;  // &d_scratch->key
   unsigned long long* h_key;  // &h_scratch->key
+  uint32_t* d_survivors;      // pruned search: 3^P prefix slots, allocated on first use
 };
 
 namespace {
@@ -228,6 +231,7 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
 
 int bf_destroy_scenario(bf_scenario* scn) {
   if (!scn) return BF_OK;
+  if (scn->d_survivors) cudaFree(scn->d_survivors);
   cudaError_t e1 = scn->d_scratch ? cudaFree(scn->d_scratch) : cudaSuccess;
   cudaError_t e2 = scn->h_scratch ? cudaFreeHost(scn->h_scratch) : cudaSuccess;
   delete scn;
@@ -375,6 +379,96 @@ int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32
   if (k > capacity) return fail(BF_EINVAL, "%s: %u probes do not fit in capacity %u", who, k, capacity);
   std::memcpy(out, probes, sizeof(bf_probe) * k);
   *count = k;
+  return BF_OK;
+}
+
+int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_result* out, void* cuda_stream) {
+  const char* who = "bf_search_pruned";
+  if (!scn_const || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
+  // The handle's lazily allocated survivor buffer is scratch, not state.
+  bf_scenario* scn = const_cast<bf_scenario*>(scn_const);
+  const uint32_t n = scn->desc.n;
+  const uint64_t total = pow3(n);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  cudaError_t e = cudaSuccess;
+
+  // 1. Incumbent: the best feasible of a few mappings (the hint, all-cpu,
+  //    all-gpu_now, all-gpu_queue, each tool on its isolated-faster device).
+  bf_scratch* h = scn->h_scratch;
+  bf_scratch* dv = scn->d_scratch;
+  uint32_t nc = 0;
+  if (hint_index < total) h->idx[nc++] = hint_index;
+  {
+    uint64_t now = 0, que = 0, fast = 0, p = 1;
+    for (uint32_t i = 0; i < n; ++i, p *= 3) {
+      now += p;
+      que += 2 * p;
+      if (scn->tables.wnow[i] / 1024u < scn->tables.cpu[i]) fast += p;
+    }
+    h->idx[nc++] = 0;
+    h->idx[nc++] = now;
+    h->idx[nc++] = que;
+    h->idx[nc++] = fast;
+  }
+  e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) {
+#define CALL(NW) launch_list_nw##NW(scn->tables, total, dv->idx, nc, dv->ms, dv->fe, 1, st)
+    BF_DISPATCH(bfk::bucket_for(n), CALL)
+#undef CALL
+  }
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h->ms, dv->ms, sizeof(uint32_t) * nc, cudaMemcpyDeviceToHost, st);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(h->fe, dv->fe, nc, cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  int rc = wait_stream(st, who);
+  if (rc != BF_OK) return rc;
+  uint32_t bound = 0xFFFFFFFFu;
+  for (uint32_t j = 0; j < nc; ++j)
+    if (h->fe[j] == 1 && h->ms[j] < bound) bound = h->ms[j];
+
+  // 2. Keep the prefixes whose checkpoint bound does not exceed the incumbent.
+  bfk::Plan plan = make_plan(scn->plan, 0, total, kSearchTasks);
+  plan.bound = bound;
+  if (!scn->d_survivors) {
+    e = lib_malloc(reinterpret_cast<void**>(&scn->d_survivors), sizeof(uint32_t) * plan.pow3P);
+    if (e != cudaSuccess) return cuda_fail(e, who);
+  }
+  e = cudaMemsetAsync(&dv->survivors, 0, sizeof(uint32_t), st);
+  if (e == cudaSuccess) {
+#define CALL(NW) launch_prefix_filter_nw##NW(scn->tables, plan, scn->d_survivors, &dv->survivors, st)
+    BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
+#undef CALL
+  }
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(&h->survivors, &dv->survivors, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  rc = wait_stream(st, who);
+  if (rc != BF_OK) return rc;
+  const uint32_t nsurv = h->survivors;
+
+  // 3. Full enumeration of the survivors' mappings, bound applied again at the
+  //    inner checkpoint; tasks of at least 16 mid combinations, about
+  //    kSearchTasks of them.
+  plan.groups = (nsurv + 31u) / 32u;
+  e = cudaMemsetAsync(scn->d_key, 0xFF, sizeof(unsigned long long), st);
+  if (e == cudaSuccess && nsurv) {
+    const uint64_t num_m = (uint64_t)plan.m_hi - plan.m_lo + 1;
+    uint64_t parts = (kSearchTasks + plan.groups - 1) / plan.groups;
+    const uint64_t min_chunk = num_m < 16 ? num_m : 16;
+    const uint64_t max_parts = (num_m + min_chunk - 1) / min_chunk;
+    if (parts > max_parts) parts = max_parts;
+    if (parts < 1) parts = 1;
+    plan.m_chunk = (uint32_t)((num_m + parts - 1) / parts);
+    plan.m_parts = (uint32_t)((num_m + plan.m_chunk - 1) / plan.m_chunk);
+#define CALL(NW) launch_pruned_search_nw##NW(scn->tables, scn->window, plan, scn->d_survivors, nsurv, scn->d_key, st)
+    BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
+#undef CALL
+  }
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(scn->h_key, scn->d_key, sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  rc = wait_stream(st, who);
+  if (rc != BF_OK) return rc;
+  fill_result(*scn->h_key, n, 0, out);
   return BF_OK;
 }
 

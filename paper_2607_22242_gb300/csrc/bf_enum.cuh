@@ -24,36 +24,40 @@ __device__ __forceinline__ bool inner_range(const Plan& plan, uint64_t base, uin
   return a <= b;
 }
 
-// Run one warp task: prefix group `g` (prefix p_lo + 32 g + lane) and mid chunk
-// `part`.  NP >= n is the prefix simulation's slot count, NW >= the window's.
-// slotA / slotB are this lane's shared-memory areas of LaneWords<NW> words
-// (stride `stride`) for the state at the prefix checkpoint and at the inner
-// checkpoint.
-// rt / rtw are the readiness tables of the full and window tables (used when
-// NP / NW <= kReadyTableSlots).
-template <int NP, int NW, typename TBF, typename TBW, typename Sink>
-__device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, const uint32_t* rt, const TBW& tw,
-                                          const SmemTables& sdw, const uint32_t* rtw, const Plan& plan, uint32_t g,
-                                          uint32_t part, uint32_t* slotA, uint32_t* slotB, uint32_t stride,
-                                          Sink& sink) {
-  const uint32_t lane = threadIdx.x & 31u;
-  const uint64_t p64 = (uint64_t)plan.p_lo + 32ull * g + lane;
-  const bool p_valid = p64 <= plan.p_hi;
-  const uint32_t p = (uint32_t)p64;
+// Simulate prefix p up to the first instant a tool >= P would become ready.
+// Returns false if every mapping with this prefix is infeasible; otherwise
+// *T_check is that instant and, when slotA is not null, the window state is
+// saved there.
+template <int NP, int NW, typename TBF>
+__device__ __forceinline__ bool prefix_checkpoint(const TBF& tb, const SmemTables& sd, const uint32_t* rt,
+                                                  const Plan& plan, uint32_t p, Digits* dgp, uint32_t* T_check,
+                                                  uint32_t* slotA, uint32_t stride) {
+  *dgp = decode(p, plan.P);
+  if (dgp->que & tb.big_mask) return false;
+  State<NP> s;
+  init_state(s, tb.all_mask);
+  const uint32_t later = tb.all_mask & ~((1u << plan.P) - 1u);
+  if (run<NP>(s, tb, sd, rt, *dgp, later) != kRunStopped) return false;
+  *T_check = s.T;
+  if (slotA) save_prefix_window<NP, NW>(s, plan.W0, tb.n - plan.W0, slotA, stride);
+  return true;
+}
 
+// A warp task whose lanes hold prefixes p (valid when p_valid).  Mappings that
+// the plan's bound proves worse than a known feasible mapping (pruned
+// searches only) are skipped without reaching the sink.
+template <int NP, int NW, typename TBF, typename TBW, typename Sink>
+__device__ __forceinline__ void prefix_task(const TBF& tb, const SmemTables& sd, const uint32_t* rt, const TBW& tw,
+                                            const SmemTables& sdw, const uint32_t* rtw, const Plan& plan,
+                                            uint32_t p, bool p_valid, uint32_t part, uint32_t* slotA,
+                                            uint32_t* slotB, uint32_t stride, Sink& sink) {
   // ---- this lane's prefix, up to the first instant a tool >= P is ready ----
   Digits dgp{0u, 0u};
   bool ok = false;
   if (p_valid) {
-    dgp = decode(p, plan.P);
-    ok = (dgp.que & tb.big_mask) == 0u;
-    if (ok) {
-      State<NP> s;
-      init_state(s, tb.all_mask);
-      const uint32_t later = tb.all_mask & ~((1u << plan.P) - 1u);
-      ok = run<NP>(s, tb, sd, rt, dgp, later) == kRunStopped;
-      if (ok) save_prefix_window<NP, NW>(s, plan.W0, tb.n - plan.W0, slotA, stride);
-    }
+    uint32_t T_check = 0u;
+    ok = prefix_checkpoint<NP, NW>(tb, sd, rt, plan, p, &dgp, &T_check, slotA, stride);
+    if (ok && (uint64_t)T_check + plan.tail_p > plan.bound) p_valid = false;  // pruned
   }
 
   // ---- the task's mid combinations, in lockstep across the warp -----------
@@ -89,6 +93,7 @@ __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, c
       for (uint32_t i = i_lo; i <= i_hi; ++i) sink((uint32_t)(base + stride_i * i), kInfeasible);
       continue;
     }
+    if ((uint64_t)w.T + plan.tail_q > plan.bound) continue;  // pruned at the inner checkpoint
     save_lane(w, slotB, stride);
     for (uint32_t i = i_lo; i <= i_hi; ++i) {
       const Digits di = decode(i, plan.I);
@@ -101,6 +106,22 @@ __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, c
       sink((uint32_t)(base + stride_i * i), ms);
     }
   }
+}
+
+// Run one warp task of a plan: prefix group `g` (prefix p_lo + 32 g + lane)
+// and mid chunk `part`.  NP >= n is the prefix simulation's slot count, NW >=
+// the window's.  slotA / slotB are this lane's shared-memory areas of
+// LaneWords<NW> words (stride `stride`) for the state at the prefix checkpoint
+// and at the inner checkpoint; rt / rtw are the readiness tables of the full
+// and window tables (used when NP / NW <= kReadyTableSlots).
+template <int NP, int NW, typename TBF, typename TBW, typename Sink>
+__device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, const uint32_t* rt, const TBW& tw,
+                                          const SmemTables& sdw, const uint32_t* rtw, const Plan& plan, uint32_t g,
+                                          uint32_t part, uint32_t* slotA, uint32_t* slotB, uint32_t stride,
+                                          Sink& sink) {
+  const uint64_t p64 = (uint64_t)plan.p_lo + 32ull * g + (threadIdx.x & 31u);
+  prefix_task<NP, NW>(tb, sd, rt, tw, sdw, rtw, plan, (uint32_t)p64, p64 <= plan.p_hi, part, slotA, slotB, stride,
+                      sink);
 }
 
 struct MinKeySink {

@@ -180,6 +180,52 @@ __global__ void __launch_bounds__(kThreads) list_kernel(const __grid_constant__ 
   }
 }
 
+// Pruned search, pass 1: one thread per prefix; keeps the prefixes whose
+// checkpoint time plus the tail bound does not exceed plan.bound.
+template <int NP>
+__global__ void __launch_bounds__(kThreads) prefix_filter_kernel(const __grid_constant__ Tables tb,
+                                                                 const __grid_constant__ Plan plan,
+                                                                 uint32_t* __restrict__ survivors,
+                                                                 uint32_t* __restrict__ count) {
+  __shared__ SmemTables sd;
+  __shared__ uint32_t rt[ReadyTable<NP>::size];
+  load_smem_tables(tb, sd);
+  fill_ready_table<NP>(tb, rt);
+  __syncthreads();
+  const uint64_t p = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= plan.pow3P) return;
+  Digits dgp;
+  uint32_t T = 0u;
+  if (prefix_checkpoint<NP, BF_NW>(tb, sd, rt, plan, (uint32_t)p, &dgp, &T, nullptr, 0u) &&
+      (uint64_t)T + plan.tail_p <= plan.bound)
+    survivors[atomicAdd(count, 1u)] = (uint32_t)p;
+}
+
+// Pruned search, pass 2: warp tasks over the surviving prefixes (32 per group).
+template <int NP>
+__global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) pruned_search_kernel(
+    const __grid_constant__ Tables tb, const __grid_constant__ Tables tw, const __grid_constant__ Plan plan,
+    const uint32_t* __restrict__ survivors, uint32_t nsurv, unsigned long long* key) {
+  extern __shared__ uint32_t lane_state[];
+  __shared__ SmemTables sd, sdw;
+  __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
+  load_smem_tables(tb, sd);
+  load_smem_tables(tw, sdw);
+  fill_ready_table<NP>(tb, rt);
+  fill_ready_table<BF_NW>(tw, rtw);
+  __syncthreads();
+  const uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5);
+  MinKeySink sink;
+  if (task < plan.groups * plan.m_parts) {
+    const uint32_t slot = (task / plan.m_parts) * 32u + (threadIdx.x & 31u);
+    const bool valid = slot < nsurv;
+    prefix_task<NP, BF_NW>(tb, sd, rt, tw, sdw, rtw, plan, valid ? survivors[slot] : 0u, valid,
+                           task % plan.m_parts, lane_state + threadIdx.x,
+                           lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
+  }
+  block_min_to(sink.best, key);
+}
+
 // Allow the kernel more than the default 48 KB of dynamic shared memory (once per kernel).
 template <typename K>
 static cudaError_t allow_dyn_smem(K kernel, bool* done) {
@@ -222,6 +268,23 @@ cudaError_t BF_PASTE(launch_eval_nw, BF_NW)(const Tables& tb, const Tables& tw, 
 cudaError_t BF_PASTE(launch_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                               unsigned long long* key, cudaStream_t st) {
   BF_LAUNCH(search_kernel, tb.n <= (uint32_t)BF_NW, plan.I, blocks_for(plan), tb, tw, plan, key);
+}
+
+cudaError_t BF_PASTE(launch_prefix_filter_nw, BF_NW)(const Tables& tb, const Plan& plan, uint32_t* survivors,
+                                                     uint32_t* count, cudaStream_t st) {
+  const unsigned grid = (unsigned)(((uint64_t)plan.pow3P + kThreads - 1) / kThreads);
+  if (tb.n <= (uint32_t)BF_NW)
+    prefix_filter_kernel<BF_NW><<<grid, kThreads, 0, st>>>(tb, plan, survivors, count);
+  else
+    prefix_filter_kernel<kMaxTools><<<grid, kThreads, 0, st>>>(tb, plan, survivors, count);
+  return cudaGetLastError();
+}
+
+cudaError_t BF_PASTE(launch_pruned_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
+                                                     const uint32_t* survivors, uint32_t nsurv,
+                                                     unsigned long long* key, cudaStream_t st) {
+  BF_LAUNCH(pruned_search_kernel, tb.n <= (uint32_t)BF_NW, plan.I, blocks_for(plan), tb, tw, plan, survivors, nsurv,
+            key);
 }
 
 // Index lists run the whole scenario in one simulation: this unit handles n <= BF_NW.

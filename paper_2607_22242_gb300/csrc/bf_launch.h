@@ -39,7 +39,12 @@ inline int bucket_for(uint32_t w) {
                                   uint32_t any_inner, uint32_t blocks_per_scenario,                  \
                                   unsigned long long* keys, cudaStream_t st);                        \
   cudaError_t launch_list_nw##NW(const Tables& tb, uint64_t total, const uint64_t* idx, uint64_t count, \
-                                 uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st);
+                                 uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st);             \
+  cudaError_t launch_prefix_filter_nw##NW(const Tables& tb, const Plan& plan, uint32_t* survivors,   \
+                                          uint32_t* count, cudaStream_t st);                         \
+  cudaError_t launch_pruned_search_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan,       \
+                                          const uint32_t* survivors, uint32_t nsurv,                 \
+                                          unsigned long long* key, cudaStream_t st);
 BF_FOR_EACH_BUCKET(BF_DECLARE_BUCKET)
 #undef BF_DECLARE_BUCKET
 

@@ -107,6 +107,25 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
   pl->M = M;
   pl->I = I;
   pl->W0 = w0;
+  // Lower-bound tails: no mode runs a tool faster than min(c, g + x) (GPU
+  // contention and the queue only slow it), and a tool starts after all its
+  // predecessors end, so a tool not started by time T finishes the whole
+  // mapping no earlier than T + tail[tool].
+  uint64_t tail[BF_MAX_TOOLS] = {0};
+  for (int v = (int)n - 1; v >= 0; --v) {
+    const uint64_t gpu = t.wnow[v] / 1024u;
+    const uint64_t dmin = t.cpu[v] < gpu ? t.cpu[v] : gpu;
+    uint64_t longest = 0;
+    for (uint32_t s = (uint32_t)v + 1; s < n; ++s)
+      if ((t.succ[v] >> s) & 1u) longest = tail[s] > longest ? tail[s] : longest;
+    tail[v] = dmin + longest;
+  }
+  uint64_t tp = 0, tq = 0;
+  for (uint32_t v = P; v < n; ++v) tp = tail[v] > tp ? tail[v] : tp;
+  for (uint32_t v = n - I; v < n; ++v) tq = tail[v] > tq ? tail[v] : tq;
+  pl->tail_p = (uint32_t)(tp < 0xFFFFFFFFull ? tp : 0xFFFFFFFFull);
+  pl->tail_q = (uint32_t)(tq < 0xFFFFFFFFull ? tq : 0xFFFFFFFFull);
+  pl->bound = 0xFFFFFFFFu;
   pl->pow3P = (uint32_t)pow3(P);
   pl->pow3M = (uint32_t)pow3(M);
   pl->pow3I = (uint32_t)pow3(I);

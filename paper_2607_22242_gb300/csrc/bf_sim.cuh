@@ -92,6 +92,12 @@ struct Plan {
   uint32_t m_chunk;         // mid combinations per warp task
   uint32_t m_parts;         // warp tasks per prefix group
   uint32_t full;            // 1 if [first, last] is all of [0, 3^n)
+  // Pruned searches only: a mapping whose state at the prefix (inner)
+  // checkpoint has T + tail_p (T + tail_q) > bound cannot be optimal.
+  // tail_p = the longest path, in minimum isolated durations min(c, g + x),
+  // from any tool >= P to the end; tail_q likewise from tools >= Q.
+  uint32_t tail_p, tail_q;
+  uint32_t bound;           // 0xFFFFFFFF: no pruning
 };
 
 // Tables read with a per-thread (dynamic) index, staged in shared memory:

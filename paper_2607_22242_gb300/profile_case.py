@@ -22,7 +22,7 @@ if ROOT not in sys.path:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=("search", "eval", "batch", "list", "whatif"), default="search")
+    ap.add_argument("--kernel", choices=("search", "pruned", "eval", "batch", "list", "whatif"), default="search")
     ap.add_argument("--config", type=int, default=3)
     ap.add_argument("--first", type=int, default=0)
     ap.add_argument("--count", type=int, default=1 << 26)
@@ -49,6 +49,9 @@ def main():
         h = bf.create_scenario(scn)
         if args.kernel == "search":
             call = lambda: bf.search_range(h, args.first, count, stream)
+        elif args.kernel == "pruned":  # branch and bound over the whole space (count ignored)
+            work = 3 ** scn.n
+            call = lambda: bf.search_pruned(h, None, stream)
         elif args.kernel == "list":  # uniformly random mapping indices of the whole space
             g = torch.Generator(device="cuda").manual_seed(1)
             idx = torch.randint(0, 3 ** scn.n, (count,), device="cuda", generator=g, dtype=torch.int64)
@@ -71,7 +74,7 @@ def main():
         b.synchronize()
         t = a.elapsed_time(b)
         print(f"{args.kernel} rep {rep}: {t:.3f} ms, {work / (t / 1e3):.4g} mappings/s"
-              + (f", best {out.index}/{out.makespan_us}" if args.kernel == "search" else ""), flush=True)
+              + (f", best {out.index}/{out.makespan_us}" if args.kernel in ("search", "pruned") else ""), flush=True)
 
 
 if __name__ == "__main__":

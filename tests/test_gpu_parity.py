@@ -360,3 +360,37 @@ def test_whatif_range_error():
         with pytest.raises(bf.BfError) as ei:
             bf.whatif(h, 3 ** 8)
         assert ei.value.code == bf.BF_ERANGE
+
+
+# --------------------------------------------------------------------------- branch and bound
+
+def test_pruned_search_equals_exhaustive_small():
+    rng = np.random.default_rng(2718)
+    for t in range(120):
+        n = int(rng.integers(1, 10))
+        scn = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.3, 0.7])), tight=bool(t % 3),
+                             max_time=int(rng.choice([6, 30, 2000])))
+        want = oracle.search(scn)
+        with bf.create_scenario(scn) as h:
+            for hint in (None, int(rng.integers(0, 3 ** n)), want[0]):
+                r = bf.search_pruned(h, hint)
+                assert (r.index, r.makespan_us, r.feasible) == (want[0], want[1], True), (scn, hint)
+
+
+@pytest.mark.parametrize("cfg", [0, 1, 2, 3])
+def test_pruned_search_standard_workloads(cfg, golden):
+    scn = S.config(cfg)
+    g = golden[str(cfg)]["summary"]
+    with bf.create_scenario(scn) as h:
+        for hint in (None, 0, g["best_index"]):
+            r = bf.search_pruned(h, hint)
+            assert (r.index, r.makespan_us, r.feasible) == (g["best_index"], g["best_makespan"], True)
+
+
+def test_pruned_search_batch_scenarios(golden):
+    batch = S.config4(64)
+    want_i, want_m = golden["4"]["best_index"], golden["4"]["best_makespan"]
+    for k, scn in enumerate(batch):
+        with bf.create_scenario(scn) as h:
+            r = bf.search_pruned(h)
+        assert (r.index, r.makespan_us) == (want_i[k], want_m[k]), k
