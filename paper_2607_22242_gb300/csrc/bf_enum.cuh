@@ -113,7 +113,7 @@ __device__ __forceinline__ void prefix_task(const TBF& tb, const SmemTables& sd,
 // the window's.  slotA / slotB are this lane's shared-memory areas of
 // LaneWords<NW> words (stride `stride`) for the state at the prefix checkpoint
 // and at the inner checkpoint; rt / rtw are the readiness tables of the full
-// and window tables (used when NP / NW <= kReadyTableSlots).
+// and window tables.
 template <int NP, int NW, typename TBF, typename TBW, typename Sink>
 __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, const uint32_t* rt, const TBW& tw,
                                           const SmemTables& sdw, const uint32_t* rtw, const Plan& plan, uint32_t g,

@@ -159,8 +159,6 @@ struct State {
   uint32_t pend;     // not yet ready
   uint32_t run_g;    // running GPU tools
   uint32_t qwait;    // queued tools waiting
-  uint32_t cand;     // tools that may have become ready at T (successors of the last
-                     // retirees); maintained by runs wider than 12 slots only
   uint32_t T, V, L;  // (k, the number of running GPU tools, is popc(run_g); the running
                      // queued tool, if any, is run_g & the gpu_queue digits)
   uint32_t tc;       // earliest CPU end (0xFFFFFFFF if none)
@@ -177,7 +175,6 @@ __device__ __forceinline__ void init_state(State<NT>& s, uint32_t all_mask) {
   s.done = ~all_mask;
   s.pend = all_mask;
   s.run_g = s.qwait = 0u;
-  s.cand = all_mask;  // at T = 0 every tool is a candidate
   s.T = s.V = s.L = 0u;
   s.tc = 0xFFFFFFFFu;
   s.gmin = 0u;
@@ -187,40 +184,48 @@ __device__ __forceinline__ void init_state(State<NT>& s, uint32_t all_mask) {
 // makespan is s.T), the mapping proves infeasible (kRunInfeasible), or a tool
 // of `stop_mask` would become ready (kRunStopped, state left before that
 // admission).  A stalled run reports kRunFinished with s.T = kStalled.
-// Readiness tables: for states of at most kReadyTableSlots slots, entry e of
-// the table is the set of tools all of whose predecessors are in the set e,
-// so an admission finds its ready tools with one shared-memory load.
-constexpr int kReadyTableSlots = 10;
-
+// Readiness tables.  A tool is ready when all its predecessors are done; the
+// done-set is cut into chunks (the whole state when it has at most 10 slots,
+// else 8 slots per chunk) and, for every value of a chunk, a table holds the
+// tools whose predecessors inside that chunk are all done.  The ready set is
+// the pending set ANDed with one table entry per chunk: one shared-memory load
+// per chunk instead of a per-tool test.
 template <int NT>
 struct ReadyTable {
-  static constexpr int size = (NT <= kReadyTableSlots) ? (1 << NT) : 1;
+  static constexpr int chunk_bits = (NT <= 10) ? NT : 8;
+  static constexpr int chunks = (NT + chunk_bits - 1) / chunk_bits;
+  static constexpr int size = chunks << chunk_bits;
 };
 
-// Fill a readiness table for NT slots (block-cooperative; tools >= n never
-// matter because they are never pending).
+// Fill a readiness table for NT slots (block-cooperative).
 template <int NT, typename TB>
 __device__ __forceinline__ void fill_ready_table(const TB& tb, uint32_t* table) {
-  if constexpr (NT <= kReadyTableSlots) {
-    for (uint32_t e = threadIdx.x; e < (1u << NT); e += blockDim.x) {
-      uint32_t r = 0u;
+  constexpr int kBits = ReadyTable<NT>::chunk_bits;
+  constexpr uint32_t kMask = (1u << kBits) - 1u;
+  for (uint32_t e = threadIdx.x; e < (uint32_t)ReadyTable<NT>::size; e += blockDim.x) {
+    const uint32_t c = e >> kBits, x = e & kMask;
+    uint32_t r = 0u;
 #pragma unroll
-      for (int v = 0; v < NT; ++v)
-        if ((tb.pred[v] & ~e) == 0u) r |= 1u << v;
-      table[e] = r;
-    }
+    for (int v = 0; v < NT; ++v)
+      if ((((tb.pred[v] >> (c * kBits)) & kMask) & ~x) == 0u) r |= 1u << v;
+    table[e] = r;
   }
+}
+
+template <int NT>
+__device__ __forceinline__ uint32_t ready_of(const uint32_t* table, uint32_t pend, uint32_t done) {
+  constexpr int kBits = ReadyTable<NT>::chunk_bits;
+  constexpr uint32_t kMask = (1u << kBits) - 1u;
+  uint32_t r = pend;
+#pragma unroll
+  for (int c = 0; c < ReadyTable<NT>::chunks; ++c) r &= table[(c << kBits) + ((done >> (c * kBits)) & kMask)];
+  return r;
 }
 
 template <int NT, typename TB>
 __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTables& sd, const uint32_t* ready_table,
                                         Digits dg, uint32_t stop_mask) {
   const uint32_t cpu_mask = tb.all_mask & ~(dg.now | dg.que);
-  // Narrow states look their ready tools up (up to 10 slots) or test every
-  // pending slot (up to 12); wide ones only test the successors of the tools
-  // that just retired (cand).
-  constexpr bool kTableReady = NT <= kReadyTableSlots;
-  constexpr bool kScanReady = NT <= 12;
 #pragma unroll 1
   for (uint32_t events = 0;; ++events) {
     if (events > (uint32_t)NT + 1u) {
@@ -228,22 +233,7 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
       return kRunFinished;
     }
     // ---- admission at T ---------------------------------------------------
-    uint32_t ready = 0u;
-    const uint32_t notdone = ~s.done;
-    if constexpr (kTableReady) {
-      ready = s.pend & ready_table[s.done & ((1u << NT) - 1u)];
-    } else if constexpr (kScanReady) {
-#pragma unroll
-      for (int i = 0; i < NT; ++i)
-        if ((s.pend & (1u << i)) && (tb.pred[i] & notdone) == 0u) ready |= 1u << i;
-    } else {
-      uint32_t c = s.cand & s.pend;
-      while (c) {
-        const int v = __ffs(c) - 1;
-        c &= c - 1u;
-        if ((sd.pred[v] & notdone) == 0u) ready |= 1u << v;
-      }
-    }
+    const uint32_t ready = ready_of<NT>(ready_table, s.pend, s.done);
     if (ready & stop_mask) return kRunStopped;
     if (ready) {
       s.pend &= ~ready;
@@ -325,7 +315,6 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
     }
 
     // ---- retire everything that ends at T ------------------------------------
-    s.cand = 0u;
     if (s.tc == s.T) {
       uint32_t ntc = 0xFFFFFFFFu;
 #pragma unroll
@@ -333,7 +322,6 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
         if (s.ec[i] == s.T) {
           s.ec[i] = 0xFFFFFFFFu;
           s.done |= 1u << i;
-          if constexpr (!kScanReady) s.cand |= tb.succ[i];
         }
         ntc = min(ntc, s.ec[i]);
       }
@@ -347,7 +335,6 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
           if (s.eg[i] == s.V) {
             rg |= 1u << i;
             s.L -= tb.vram[i];
-            if constexpr (!kScanReady) s.cand |= tb.succ[i];
           } else {
             nrem = min(nrem, s.eg[i] - s.V);
           }
@@ -365,7 +352,7 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
 // accesses to the same word hit 32 different banks.
 template <int NW>
 struct LaneWords {
-  static constexpr int value = 2 * NW + 10;
+  static constexpr int value = 2 * NW + 9;
 };
 
 template <int NW>
@@ -380,12 +367,11 @@ __device__ __forceinline__ void save_lane(const State<NW>& s, uint32_t* slot, ui
   t[1 * stride] = s.pend;
   t[2 * stride] = s.run_g;
   t[3 * stride] = s.qwait;
-  t[4 * stride] = s.cand;
-  t[5 * stride] = s.T;
-  t[6 * stride] = s.V;
-  t[7 * stride] = s.L;
-  t[8 * stride] = s.tc;
-  t[9 * stride] = s.gmin;
+  t[4 * stride] = s.T;
+  t[5 * stride] = s.V;
+  t[6 * stride] = s.L;
+  t[7 * stride] = s.tc;
+  t[8 * stride] = s.gmin;
 }
 
 template <int NW>
@@ -400,12 +386,11 @@ __device__ __forceinline__ void load_lane(const uint32_t* slot, uint32_t stride,
   s.pend = t[1 * stride];
   s.run_g = t[2 * stride];
   s.qwait = t[3 * stride];
-  s.cand = t[4 * stride];
-  s.T = t[5 * stride];
-  s.V = t[6 * stride];
-  s.L = t[7 * stride];
-  s.tc = t[8 * stride];
-  s.gmin = t[9 * stride];
+  s.T = t[4 * stride];
+  s.V = t[5 * stride];
+  s.L = t[6 * stride];
+  s.tc = t[7 * stride];
+  s.gmin = t[8 * stride];
 }
 
 // Save the window part [W0, n) of a prefix state (NP slots) as a window state
@@ -432,12 +417,11 @@ __device__ __forceinline__ void save_prefix_window(const State<NP>& s, uint32_t 
   t[1 * stride] = (s.pend >> W0) & wmask;
   t[2 * stride] = s.run_g >> W0;
   t[3 * stride] = s.qwait >> W0;
-  t[4 * stride] = (s.cand >> W0) & wmask;
-  t[5 * stride] = s.T;
-  t[6 * stride] = s.V;
-  t[7 * stride] = s.L;
-  t[8 * stride] = s.tc;
-  t[9 * stride] = s.gmin;
+  t[4 * stride] = s.T;
+  t[5 * stride] = s.V;
+  t[6 * stride] = s.L;
+  t[7 * stride] = s.tc;
+  t[8 * stride] = s.gmin;
 }
 
 }  // namespace bfk
