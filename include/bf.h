@@ -61,7 +61,10 @@
 extern "C" {
 #endif
 
-#define BF_MAX_TOOLS 20
+#define BF_MAX_TOOLS 32       /* largest scenario (32-bit tool masks) */
+#define BF_MAX_TOOLS_ENUM 20  /* largest scenario of the full-enumeration entry points
+                                 (bf_eval_mappings, bf_search_best, bf_search_range,
+                                 bf_search_pruned, bf_search_batch*): 3^20 < 2^32 */
 
 enum bf_status {
   BF_OK = 0,
@@ -78,7 +81,8 @@ enum bf_mode { BF_MODE_CPU = 0, BF_MODE_GPU_NOW = 1, BF_MODE_GPU_QUEUE = 2 };
  * One workflow (§2.1) with the per-tool profile of Table 1 / §3.1 plus a
  * transfer time.  Tools are numbered 0..n-1 in a topological order.
  * Validity (checked by every entry point that takes a desc):
- *   1 <= n <= 20; pred_mask[v] has bits only below v (u < v) and below n;
+ *   1 <= n <= 32 (the full-enumeration entry points take n <= 20 and return
+ *   BF_EINVAL above); pred_mask[v] has bits only below v (u < v);
  *   cpu_us >= 1, gpu_us >= 1; load_us + gpu_us + xfer_us < 2^22;
  *   vram_mib <= 2^27, vram_budget_mib <= 2^31;
  *   slowdown_q10[1] == 1024, slowdown_q10[k] non-decreasing and <= 65536 for
@@ -88,7 +92,7 @@ enum bf_mode { BF_MODE_CPU = 0, BF_MODE_GPU_NOW = 1, BF_MODE_GPU_QUEUE = 2 };
  * Entries at index >= n are ignored.
  */
 typedef struct bf_scenario_desc {
-  uint32_t n;                               /* number of tools, 1..20 */
+  uint32_t n;                               /* number of tools, 1..32 */
   uint32_t pred_mask[BF_MAX_TOOLS];         /* bit u of pred_mask[v] <=> edge u->v */
   uint32_t cpu_us[BF_MAX_TOOLS];            /* c_i: CPU latency, us */
   uint32_t gpu_us[BF_MAX_TOOLS];            /* g_i: isolated GPU latency, us */

@@ -30,7 +30,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(BUILD_DIR, "libbforacle.so")
 SOURCE = os.path.join(HERE, "bf_oracle.cpp")
 
-MAX_TOOLS = 20
+MAX_TOOLS = 32
 FLAT_WORDS = 2 + 6 * MAX_TOOLS + (MAX_TOOLS + 1)
 INFEASIBLE = 0xFFFFFFFF
 
@@ -51,7 +51,7 @@ def build(force: bool = False, source: str = SOURCE, out: str = LIB_PATH) -> str
 
 
 def flat(scn) -> np.ndarray:
-    """The oracle's own flat record: n, M, pred[20], c[20], g[20], x[20], l[20], m[20], f[21]."""
+    """The oracle's own flat record: n, M, pred[32], c[32], g[32], x[32], l[32], m[32], f[33]."""
     w = np.zeros(FLAT_WORDS, dtype=np.uint32)
     n = scn.n
     w[0] = n
@@ -59,7 +59,7 @@ def flat(scn) -> np.ndarray:
     cols = (scn.pred_mask, scn.cpu_us, scn.gpu_us, scn.xfer_us, scn.load_us, scn.vram_mib)
     for j, col in enumerate(cols):
         w[2 + j * MAX_TOOLS: 2 + j * MAX_TOOLS + n] = np.asarray(col[:n], dtype=np.uint64)
-    f = np.asarray(scn.slowdown_q10, dtype=np.uint64)
+    f = np.asarray(scn.slowdown_q10[:MAX_TOOLS + 1], dtype=np.uint64)
     w[2 + 6 * MAX_TOOLS: 2 + 6 * MAX_TOOLS + len(f)] = f
     return w
 
@@ -93,6 +93,9 @@ class OracleLib:
         lib.bf_oracle_search_batch.restype = None
         lib.bf_oracle_summary_range.argtypes = [u32p, ctypes.c_uint64, ctypes.c_uint64, u64p, ctypes.c_int]
         lib.bf_oracle_summary_range.restype = None
+        lib.bf_oracle_search_binary_range.argtypes = [u32p, ctypes.c_uint64, ctypes.c_uint64, u64p, u64p,
+                                                      ctypes.c_int]
+        lib.bf_oracle_search_binary_range.restype = ctypes.c_int
         assert lib.bf_oracle_flat_words() == FLAT_WORDS
         self.lib = lib
 
@@ -123,6 +126,23 @@ class OracleLib:
 
     def search(self, scn, threads: int = 1) -> Tuple[int, int]:
         return self.search_range(scn, 0, 3 ** scn.n, threads)
+
+    def search_binary_range(self, scn, first: int, count: int, threads: int = 1) -> Tuple[int, int]:
+        """Best feasible mapping among members [first, first+count) of the binary (cpu/gpu_now)
+        decision space, member b having a_i = bit i of b; (index, makespan), (-1, INFEASIBLE) if none."""
+        w = flat(scn)
+        idx = np.zeros(1, dtype=np.uint64)
+        ms = np.zeros(1, dtype=np.uint64)
+        found = self.lib.bf_oracle_search_binary_range(_ptr(w, ctypes.c_uint32), first, count,
+                                                       _ptr(idx, ctypes.c_uint64), _ptr(ms, ctypes.c_uint64),
+                                                       threads)
+        if not found:
+            return -1, INFEASIBLE
+        return int(idx[0]), int(ms[0])
+
+    def search_binary(self, scn, threads: int = 1) -> Tuple[int, int]:
+        """Optimum of the binary decision space (§4.1's S1-S10: each tool on the CPU or the GPU)."""
+        return self.search_binary_range(scn, 0, 2 ** scn.n, threads)
 
     def summary_range(self, scn, first: int, count: int, threads: int = 1) -> dict:
         """Feasible count, makespan sum, order-sensitive hash and argmin of a range."""
@@ -167,6 +187,14 @@ def search(scn, threads: int = 1):
 
 def search_batch(scns: Sequence, threads: int = 1):
     return default().search_batch(scns, threads)
+
+
+def search_binary(scn, threads: int = 1):
+    return default().search_binary(scn, threads)
+
+
+def search_binary_range(scn, first: int, count: int, threads: int = 1):
+    return default().search_binary_range(scn, first, count, threads)
 
 
 def summary_range(scn, first: int, count: int, threads: int = 1):

@@ -40,6 +40,12 @@
 // 2=gpu_queue}; tool 0 is the least-significant digit.  The argmin compares
 // (makespan, idx) lexicographically over feasible mappings, so ties go to the
 // lowest index.
+//
+// The binary decision space (§4.1: every scenario of S1-S10 chooses between
+// CPU and GPU only, 2^N mappings): mappings whose digits are all 0 or 1.  The
+// b-th of them (b = sum_i b_i 2^i) is the mapping with a_i = b_i; its index
+// is sum_i b_i 3^i.  The binary search below enumerates b and compares
+// (makespan, idx) as above.
 
 #include <cstdint>
 #include <cstring>
@@ -48,7 +54,7 @@
 
 namespace {
 
-const int kMaxTools = 20;
+const int kMaxTools = 32;
 const uint64_t kInfinity = UINT64_MAX;
 const uint64_t kInfeasibleMakespan = 0xFFFFFFFFull;
 const uint64_t kStalled = 0xFFFFFFFFFFFFFFFEull;  // never produced by a correct model
@@ -57,7 +63,7 @@ enum Mode { kCpu = 0, kGpuNow = 1, kGpuQueue = 2 };
 enum Status { kPending, kWaitingInQueue, kRunning, kDone };
 
 // The oracle's own scenario record, unpacked from a flat uint32 array:
-//   [0] n, [1] M, then 20 words each of pred, c, g, x, l, m, then 21 words f.
+//   [0] n, [1] M, then 32 words each of pred, c, g, x, l, m, then 33 words f.
 struct OracleScenario {
   int n;
   uint64_t budget;
@@ -225,6 +231,14 @@ uint64_t evaluate(const OracleScenario& s, uint64_t idx) {
   return sim.run();
 }
 
+// Index of the b-th mapping of the binary decision space.
+uint64_t binary_to_index(uint64_t b, int n) {
+  uint64_t idx = 0, p = 1;
+  for (int i = 0; i < n; ++i, p *= 3)
+    if ((b >> i) & 1) idx += p;
+  return idx;
+}
+
 uint64_t num_mappings(int n) {
   uint64_t p = 1;
   for (int i = 0; i < n; ++i) p *= 3;
@@ -345,6 +359,34 @@ void bf_oracle_summary_range(const uint32_t* flat, uint64_t first, uint64_t coun
   }
   out[3] = all.found ? all.index : kInfinity;
   out[4] = all.found ? all.makespan : kInfeasibleMakespan;
+}
+
+// Best feasible mapping of the binary decision space among its members
+// b in [first, first+count) (b as above, 0 <= b < 2^n): writes its
+// (ternary) index and makespan; returns 1 if one was found, 0 otherwise.
+int bf_oracle_search_binary_range(const uint32_t* flat, uint64_t first, uint64_t count,
+                                  uint64_t* out_index, uint64_t* out_makespan, int nthreads) {
+  const OracleScenario s = unpack(flat);
+  nthreads = clamp_threads(nthreads, count);
+  std::vector<Best> best(nthreads);
+  std::vector<std::thread> pool;
+  for (int t = 0; t < nthreads; ++t) {
+    uint64_t lo = count * t / nthreads, hi = count * (t + 1) / nthreads;
+    pool.emplace_back([&, t, lo, hi]() {
+      for (uint64_t j = lo; j < hi; ++j) {
+        const uint64_t idx = binary_to_index(first + j, s.n);
+        best[t].offer(evaluate(s, idx), idx);
+      }
+    });
+  }
+  for (auto& th : pool) th.join();
+  Best all;
+  for (auto& b : best)
+    if (b.found) all.offer(b.makespan, b.index);
+  if (!all.found) return 0;
+  *out_index = all.index;
+  *out_makespan = all.makespan;
+  return 1;
 }
 
 // Full search of each of `count` scenarios (flat records back to back).

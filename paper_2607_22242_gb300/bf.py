@@ -42,13 +42,13 @@ class BfError(RuntimeError):
         self.message = message
 
 
-U32x20 = ctypes.c_uint32 * MAX_TOOLS
+U32xT = ctypes.c_uint32 * MAX_TOOLS
 
 
 class Desc(ctypes.Structure):
     """``bf_scenario_desc``."""
-    _fields_ = [("n", ctypes.c_uint32), ("pred_mask", U32x20), ("cpu_us", U32x20), ("gpu_us", U32x20),
-                ("xfer_us", U32x20), ("load_us", U32x20), ("vram_mib", U32x20),
+    _fields_ = [("n", ctypes.c_uint32), ("pred_mask", U32xT), ("cpu_us", U32xT), ("gpu_us", U32xT),
+                ("xfer_us", U32xT), ("load_us", U32xT), ("vram_mib", U32xT),
                 ("vram_budget_mib", ctypes.c_uint32), ("slowdown_q10", ctypes.c_uint32 * (MAX_TOOLS + 1))]
 
 
@@ -171,14 +171,16 @@ def pack_descs(scns: Sequence[Scenario]):
         for j, name in enumerate(cols):
             arr[:, 1 + MAX_TOOLS * j: 1 + MAX_TOOLS * j + n] = flat((getattr(sc, name)[:n] for sc in scns), n)
         arr[:, 1 + 6 * MAX_TOOLS] = np.fromiter((sc.vram_budget_mib for sc in scns), dtype=np.uint32, count=count)
-        arr[:, 2 + 6 * MAX_TOOLS:] = flat((sc.slowdown_q10[:MAX_TOOLS + 1] for sc in scns), MAX_TOOLS + 1)
+        pad = [0] * (MAX_TOOLS + 1)
+        arr[:, 2 + 6 * MAX_TOOLS:] = flat(((sc.slowdown_q10 + pad)[:MAX_TOOLS + 1] for sc in scns), MAX_TOOLS + 1)
         return arr
     for r, sc in enumerate(scns):
         arr[r, 0] = sc.n
         for j, name in enumerate(cols):
             arr[r, 1 + MAX_TOOLS * j: 1 + MAX_TOOLS * j + sc.n] = getattr(sc, name)[:sc.n]
         arr[r, 1 + 6 * MAX_TOOLS] = sc.vram_budget_mib
-        arr[r, 2 + 6 * MAX_TOOLS:] = sc.slowdown_q10[:MAX_TOOLS + 1]
+        f = sc.slowdown_q10[:MAX_TOOLS + 1]
+        arr[r, 2 + 6 * MAX_TOOLS: 2 + 6 * MAX_TOOLS + len(f)] = f
     return arr
 
 

@@ -30,7 +30,7 @@ struct bf_scratch {
 
 struct bf_scenario {
   bf_scenario_desc desc;
-  bfk::Tables tables;   // all n tools
+  bfk::Tables tables;   // all n tools (n <= BF_MAX_TOOLS_ENUM; zero otherwise)
   bfk::Tables window;   // tools [W0, n), renumbered from 0
   bfk::Plan plan;       // enumeration split and window (see bfk::Plan), full range
   int device;
@@ -146,6 +146,13 @@ int wait_stream(cudaStream_t st, const char* who) {
   }
 }
 
+// The entry points that enumerate index ranges hold indices in 32 bits.
+int require_enum(const bf_scenario_desc& d, const char* who) {
+  if (d.n > BF_MAX_TOOLS_ENUM)
+    return fail(BF_EINVAL, "%s: n=%u; full enumeration takes n <= %d (3^n < 2^32)", who, d.n, BF_MAX_TOOLS_ENUM);
+  return BF_OK;
+}
+
 void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* out) {
   std::memset(out, 0, sizeof *out);
   const uint32_t ms = (uint32_t)(key >> 32);
@@ -212,8 +219,10 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   if (!s) return fail(BF_ENOMEM, "bf_create_scenario: host allocation failed");
   std::memset(s, 0, sizeof *s);
   s->desc = *desc;
-  build_tables(desc, &s->tables);
-  split_and_window(s->tables, &s->plan, &s->window);
+  if (desc->n <= BF_MAX_TOOLS_ENUM) {
+    build_tables(desc, &s->tables);
+    split_and_window(s->tables, &s->plan, &s->window);
+  }
   cudaError_t e = cudaGetDevice(&s->device);
   if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_scratch), sizeof(bf_scratch));
   if (e == cudaSuccess) e = lib_malloc_host(reinterpret_cast<void**>(&s->h_scratch), sizeof(bf_scratch));
@@ -243,6 +252,7 @@ int bf_destroy_scenario(bf_scenario* scn) {
 int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count, uint32_t* d_makespan,
                      uint8_t* d_feasible, void* cuda_stream) {
   if (!scn) return fail(BF_EINVAL, "bf_eval_mappings: scenario is NULL");
+  if (require_enum(scn->desc, "bf_eval_mappings") != BF_OK) return BF_EINVAL;
   const uint64_t total = pow3(scn->desc.n);
   if (first > total || count > total - first)
     return fail(BF_ERANGE, "bf_eval_mappings: [%llu, %llu+%llu) is outside [0, 3^%u)",
@@ -261,12 +271,14 @@ int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count, uin
 
 int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_stream) {
   if (!scn || !out) return fail(BF_EINVAL, "bf_search_best: NULL argument");
+  if (require_enum(scn->desc, "bf_search_best") != BF_OK) return BF_EINVAL;
   return run_search(scn, 0, pow3(scn->desc.n), out, static_cast<cudaStream_t>(cuda_stream), "bf_search_best");
 }
 
 int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result* out,
                     void* cuda_stream) {
   if (!scn || !out) return fail(BF_EINVAL, "bf_search_range: NULL argument");
+  if (require_enum(scn->desc, "bf_search_range") != BF_OK) return BF_EINVAL;
   const uint64_t total = pow3(scn->desc.n);
   if (first > total || count > total - first)
     return fail(BF_ERANGE, "bf_search_range: [%llu, %llu+%llu) is outside [0, 3^%u)",
@@ -277,6 +289,7 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count, bf_r
 int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t count, uint32_t* d_makespan,
                     uint8_t* d_feasible, void* cuda_stream) {
   if (!scn) return fail(BF_EINVAL, "bf_eval_indices: scenario is NULL");
+  if (require_enum(scn->desc, "bf_eval_indices") != BF_OK) return BF_EINVAL;
   if (count == 0) return BF_OK;
   if (!d_indices || !d_makespan || !d_feasible) return fail(BF_EINVAL, "bf_eval_indices: NULL buffer");
   int sms = 0;
@@ -297,6 +310,7 @@ int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32
               void* cuda_stream) {
   const char* who = "bf_whatif";
   if (!scn || !out || !count) return fail(BF_EINVAL, "%s: NULL argument", who);
+  if (require_enum(scn->desc, who) != BF_OK) return BF_EINVAL;
   const uint32_t n = scn->desc.n;
   const uint64_t total = pow3(n);
   if (base_index >= total)
@@ -385,6 +399,7 @@ int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32
 int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_result* out, void* cuda_stream) {
   const char* who = "bf_search_pruned";
   if (!scn_const || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
+  if (require_enum(scn_const->desc, who) != BF_OK) return BF_EINVAL;
   // The handle's lazily allocated survivor buffer is scratch, not state.
   bf_scenario* scn = const_cast<bf_scenario*>(scn_const);
   const uint32_t n = scn->desc.n;
@@ -477,7 +492,8 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
   if (!descs || !out) return fail(BF_EINVAL, "bf_search_batch: NULL argument");
   uint32_t nmax = 0;
   for (uint32_t i = 0; i < count; ++i) {
-    const int rc = validate(descs + i, "bf_search_batch");
+    int rc = validate(descs + i, "bf_search_batch");
+    if (rc == BF_OK) rc = require_enum(descs[i], "bf_search_batch");
     if (rc != BF_OK) return fail(rc, "bf_search_batch: descs[%u]: %s", i, g_error.c_str());
     if (descs[i].n > nmax) nmax = descs[i].n;
   }
@@ -588,7 +604,8 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
                 "batch or use bf_search_batch", who, count, BF_NOALLOC_MAX_SCENARIOS);
   uint32_t nmax = 0;
   for (uint32_t i = 0; i < count; ++i) {
-    const int rc = validate(descs + i, who);
+    int rc = validate(descs + i, who);
+    if (rc == BF_OK) rc = require_enum(descs[i], who);
     if (rc != BF_OK) return fail(rc, "%s: descs[%u]: %s", who, i, g_error.c_str());
     if (descs[i].n > nmax) nmax = descs[i].n;
   }

@@ -21,7 +21,10 @@ inline uint64_t pow3(uint32_t n) {
   return p;
 }
 
-inline void build_tables(const bf_scenario_desc* d, bfk::Tables* t) {
+// Tables of capacity CAP >= n (kMaxTools for the enumerating searches, 32 for
+// the tree search and wide index lists).
+template <int CAP>
+inline void build_tables(const bf_scenario_desc* d, bfk::TablesT<CAP>* t) {
   std::memset(t, 0, sizeof *t);
   const uint32_t n = d->n;
   t->n = n;
@@ -37,7 +40,7 @@ inline void build_tables(const bf_scenario_desc* d, bfk::Tables* t) {
     t->vram[v] = d->vram_mib[v];
     if (d->vram_mib[v] > d->vram_budget_mib) t->big_mask |= 1u << v;
   }
-  for (uint32_t k = 1; k <= BF_MAX_TOOLS; ++k) {
+  for (uint32_t k = 1; k <= (uint32_t)CAP; ++k) {
     // Entries above n are never used; fill them with f[n] so every k is defined.
     const uint32_t f = d->slowdown_q10[k <= n ? k : n];
     uint32_t l = 0;
@@ -143,7 +146,7 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
     w->wq[j] = t.wq[w0 + j];
     w->vram[j] = t.vram[w0 + j];
   }
-  for (uint32_t k = 0; k <= BF_MAX_TOOLS; ++k) {
+  for (uint32_t k = 0; k <= (uint32_t)bfk::kMaxTools; ++k) {
     w->f[k] = t.f[k];
     w->fshift[k] = t.fshift[k];
     w->fmagic[k] = t.fmagic[k];

@@ -50,21 +50,26 @@ enum RunResult : uint32_t { kRunFinished = 0, kRunInfeasible = 1, kRunStopped = 
 
 // Device-format scenario tables (per tool: index order), passed by value as a
 // __grid_constant__ kernel parameter (constant bank) or staged in shared memory.
-struct Tables {
+// CAP is the slot capacity: kMaxTools for the enumerating searches, 32 for the
+// tree search and index lists beyond 20 tools.
+template <int CAP>
+struct TablesT {
+  static constexpr int cap = CAP;
   uint32_t n;
   uint32_t budget;       // M
   uint32_t all_mask;     // (1 << n) - 1
   uint32_t big_mask;     // tools with m > M
-  uint32_t pred[kMaxTools];
-  uint32_t succ[kMaxTools];
-  uint32_t cpu[kMaxTools];   // c_i
-  uint32_t wnow[kMaxTools];  // (g_i + x_i) * 1024
-  uint32_t wq[kMaxTools];    // (l_i + g_i + x_i) * 1024
-  uint32_t vram[kMaxTools];  // m_i
-  uint32_t f[kMaxTools + 1];        // f[k]; f[0] unused
-  uint32_t fshift[kMaxTools + 1];   // l - 12
-  uint64_t fmagic[kMaxTools + 1];   // ceil(2^(52+l) / f[k])
+  uint32_t pred[CAP];
+  uint32_t succ[CAP];
+  uint32_t cpu[CAP];   // c_i
+  uint32_t wnow[CAP];  // (g_i + x_i) * 1024
+  uint32_t wq[CAP];    // (l_i + g_i + x_i) * 1024
+  uint32_t vram[CAP];  // m_i
+  uint32_t f[CAP + 1];        // f[k]; f[0] unused
+  uint32_t fshift[CAP + 1];   // l - 12
+  uint64_t fmagic[CAP + 1];   // ceil(2^(52+l) / f[k])
 };
+using Tables = TablesT<kMaxTools>;
 
 // How a search enumerates the mapping index idx = p + 3^P * (m + 3^M * i):
 //   prefix p -> the modes of tools [0, P);
@@ -102,20 +107,22 @@ struct Plan {
 
 // Tables read with a per-thread (dynamic) index, staged in shared memory:
 // the per-k slowdown constants and the predecessor masks.
-struct SmemTables {
-  uint64_t magic[kMaxTools + 1];
-  uint32_t f[kMaxTools + 1];
-  uint32_t shift[kMaxTools + 1];
-  uint32_t pred[kMaxTools];
+template <int CAP>
+struct SmemTablesT {
+  uint64_t magic[CAP + 1];
+  uint32_t f[CAP + 1];
+  uint32_t shift[CAP + 1];
+  uint32_t pred[CAP];
 };
+using SmemTables = SmemTablesT<kMaxTools>;
 
-template <typename TB>
-__device__ __forceinline__ void load_smem_tables(const TB& tb, SmemTables& s) {
-  for (int k = threadIdx.x; k <= kMaxTools; k += blockDim.x) {
+template <int CAP>
+__device__ __forceinline__ void load_smem_tables(const TablesT<CAP>& tb, SmemTablesT<CAP>& s) {
+  for (int k = threadIdx.x; k <= CAP; k += blockDim.x) {
     s.magic[k] = tb.fmagic[k];
     s.f[k] = tb.f[k];
     s.shift[k] = tb.fshift[k];
-    if (k < kMaxTools) s.pred[k] = tb.pred[k];
+    if (k < CAP) s.pred[k] = tb.pred[k];
   }
 }
 
@@ -222,9 +229,10 @@ __device__ __forceinline__ uint32_t ready_of(const uint32_t* table, uint32_t pen
   return r;
 }
 
-template <int NT, typename TB>
-__device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTables& sd, const uint32_t* ready_table,
+template <int NT, typename TB, typename SD>
+__device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SD& sd, const uint32_t* ready_table,
                                         Digits dg, uint32_t stop_mask) {
+  static_assert(NT <= TB::cap, "state wider than its tables");
   const uint32_t cpu_mask = tb.all_mask & ~(dg.now | dg.que);
 #pragma unroll 1
   for (uint32_t events = 0;; ++events) {
@@ -296,7 +304,7 @@ __device__ __forceinline__ uint32_t run(State<NT>& s, const TB& tb, const SmemTa
 
     // ---- next event ---------------------------------------------------------
     const uint32_t k = __popc(s.run_g);
-    const uint32_t kk = min(k, (uint32_t)kMaxTools);  // k <= n always; keeps indexing in bounds
+    const uint32_t kk = min(k, (uint32_t)NT);  // k <= NT always; keeps indexing in bounds
     bool gpu_event = false;
     if (k) {
       const uint32_t rem = s.gmin - s.V;

@@ -24,7 +24,8 @@ from typing import List, Sequence
 
 import numpy as np
 
-MAX_TOOLS = 20
+MAX_TOOLS = 32          # largest scenario the library takes (32-bit tool masks)
+ENUM_MAX_TOOLS = 20     # largest scenario of the full-enumeration searches (3^20 < 2^32 indices)
 CPU, GPU_NOW, GPU_QUEUE = 0, 1, 2
 MODE_NAMES = ("cpu", "gpu_now", "gpu_queue")
 
@@ -41,7 +42,7 @@ class Scenario:
     load_us: List[int]        # l_i: gpu_queue load-in cost
     vram_mib: List[int]       # m_i: VRAM footprint
     vram_budget_mib: int      # M
-    slowdown_q10: List[int]   # f[k], k=1..20 at [k]; [0] unused; 1024 = no slowdown
+    slowdown_q10: List[int]   # f[k], k=1..n (or more) at [k]; [0] unused; 1024 = no slowdown
 
     def __post_init__(self):
         for name in ("pred_mask", "cpu_us", "gpu_us", "xfer_us", "load_us", "vram_mib"):
@@ -95,15 +96,15 @@ def mapping_modes(index: int, n: int) -> List[int]:
 # slow each other; CPU tools are unaffected).
 # ---------------------------------------------------------------------------
 
-def slowdown_flat() -> List[int]:
-    """No contention: f[k] = 1024 for every k."""
-    return [0] + [1024] * MAX_TOOLS
+def slowdown_flat(kmax: int = ENUM_MAX_TOOLS) -> List[int]:
+    """No contention: f[k] = 1024 for k = 1..kmax."""
+    return [0] + [1024] * kmax
 
 
-def slowdown_linear(pct_per_extra_tool: int = 35) -> List[int]:
-    """f[k] = round-half-up(1024 * (1 + pct/100 * (k-1))) for k = 1..20."""
+def slowdown_linear(pct_per_extra_tool: int = 35, kmax: int = ENUM_MAX_TOOLS) -> List[int]:
+    """f[k] = round-half-up(1024 * (1 + pct/100 * (k-1))) for k = 1..kmax."""
     return [0] + [(1024 * (100 + pct_per_extra_tool * (k - 1)) + 50) // 100
-                  for k in range(1, MAX_TOOLS + 1)]
+                  for k in range(1, kmax + 1)]
 
 
 # ---------------------------------------------------------------------------
@@ -194,6 +195,35 @@ CONFIG3_F2 = tuple(range(12, 18))
 GPU_PREFERRED, AMBIGUOUS, CPU_PREFERRED, NEUTRAL = range(4)
 
 
+def _zoned_tool(rng: np.random.Generator, cat: int):
+    """Draw one tool of a scheduling zone (§2.2): g, then the zone's c, x, m."""
+    gi = min(max(_rint(rng.lognormal(np.log(G_MEDIAN_US), G_SIGMA)), 1), G_MAX_US)
+    if cat == GPU_PREFERRED:
+        ci = gi * rng.uniform(5.0, 70.0)
+        xi = _rint(rng.uniform(1000.0, 30000.0))
+        mi = int(rng.integers(512, 6144, endpoint=True))
+    elif cat == AMBIGUOUS:
+        ci = gi * rng.uniform(0.8, 1.5)
+        xi = _rint(rng.uniform(1000.0, 30000.0))
+        mi = int(rng.integers(512, 6144, endpoint=True))
+    elif cat == CPU_PREFERRED:
+        xi = _rint(gi * rng.uniform(1.5, 3.0))
+        ci = (gi + xi) * rng.uniform(0.3, 0.5)
+        mi = int(rng.integers(512, 6144, endpoint=True))
+    else:
+        ci = gi * rng.uniform(0.95, 1.05)
+        xi = _rint(rng.uniform(0.0, 1000.0))
+        mi = int(rng.integers(16, 128, endpoint=True))
+    return min(max(_rint(ci), 1), C_MAX_US), gi, xi, mi
+
+
+def _zoned_tools(rng: np.random.Generator, zone_counts: Sequence[int]):
+    """Zones assigned to tools by a seeded permutation, then each tool's draws in index order."""
+    cats = rng.permutation(sum(([z] * k for z, k in enumerate(zone_counts)), []))
+    cols = [_zoned_tool(rng, int(cat)) for cat in cats]
+    return [list(t) for t in zip(*cols)]
+
+
 def config3() -> Scenario:
     """N=19 mixed DAG with the four scheduling zones of §2.2; 32 GiB budget; seed 3.
 
@@ -202,31 +232,7 @@ def config3() -> Scenario:
     """
     rng = np.random.default_rng(3)
     n = 19
-    cats = rng.permutation([GPU_PREFERRED] * 11 + [AMBIGUOUS] * 4 + [CPU_PREFERRED] + [NEUTRAL] * 3)
-    c, g, x, m = [], [], [], []
-    for i in range(n):
-        gi = min(max(_rint(rng.lognormal(np.log(G_MEDIAN_US), G_SIGMA)), 1), G_MAX_US)
-        cat = int(cats[i])
-        if cat == GPU_PREFERRED:
-            ci = gi * rng.uniform(5.0, 70.0)
-            xi = _rint(rng.uniform(1000.0, 30000.0))
-            mi = int(rng.integers(512, 6144, endpoint=True))
-        elif cat == AMBIGUOUS:
-            ci = gi * rng.uniform(0.8, 1.5)
-            xi = _rint(rng.uniform(1000.0, 30000.0))
-            mi = int(rng.integers(512, 6144, endpoint=True))
-        elif cat == CPU_PREFERRED:
-            xi = _rint(gi * rng.uniform(1.5, 3.0))
-            ci = (gi + xi) * rng.uniform(0.3, 0.5)
-            mi = int(rng.integers(512, 6144, endpoint=True))
-        else:
-            ci = gi * rng.uniform(0.95, 1.05)
-            xi = _rint(rng.uniform(0.0, 1000.0))
-            mi = int(rng.integers(16, 128, endpoint=True))
-        c.append(min(max(_rint(ci), 1), C_MAX_US))
-        g.append(gi)
-        x.append(xi)
-        m.append(mi)
+    c, g, x, m = _zoned_tools(rng, (11, 4, 1, 3))
     pred = [0] * n
     s0, s1, s2, s3, s4, s5, s6 = CONFIG3_SPINE
     pred[s1] = 1 << s0
@@ -266,6 +272,71 @@ def config4(count: int = 4096) -> List[Scenario]:
     return out
 
 
+# ---------------------------------------------------------------------------
+# Workloads beyond 20 tools (the tree search, bf_search_tree).  The config-3
+# recipe grown by one more spine segment and wider fan-outs: spine
+# s0 -> s1 -> s2 -> s3 -> ... ; fan-out j (width w) hangs off spine tool
+# s(3j+1) and joins at s(3j+3), beside s(3j+2).  Zones in config 3's
+# proportions (11 : 4 : 1 : 3 of 19), seeded permutation; 32 GiB budget;
+# f = 1 + 0.35 (k-1) up to k = n.
+# ---------------------------------------------------------------------------
+
+def spine_fanout_layout(fanouts: int, width: int, tail: int):
+    """(n, pred) of the spine/fan-out DAG in topological numbering, ``tail`` spine tools after the last join."""
+    pred: List[int] = []
+    prev = None
+
+    def add(mask):
+        pred.append(mask)
+        return len(pred) - 1
+
+    prev = add(0)                      # s0
+    for _ in range(fanouts):
+        head = add(1 << prev)          # s(3j+1): the fan-out's source
+        side = add(1 << head)          # s(3j+2)
+        fan = [add(1 << head) for _ in range(width)]
+        prev = add((1 << side) | sum(1 << v for v in fan))  # s(3j+3): the join
+    for _ in range(tail):
+        prev = add(1 << prev)
+    return len(pred), pred
+
+
+def _wide(fanouts: int, width: int, tail: int, zones, seed: int) -> Scenario:
+    n, pred = spine_fanout_layout(fanouts, width, tail)
+    assert sum(zones) == n
+    rng = np.random.default_rng(seed)
+    c, g, x, m = _zoned_tools(rng, zones)
+    return Scenario(n, pred, c, g, x, [_load_from_vram(v) for v in m], m,
+                    32768, slowdown_linear(kmax=n))
+
+
+def wide28() -> Scenario:
+    """N=28: spine of 10, three fan-outs of 6; zones 16/6/2/4; seed 5 (the full 3^28 space)."""
+    return _wide(3, 6, 0, (16, 6, 2, 4), 5)
+
+
+def wide32() -> Scenario:
+    """N=32: spine of 11, three fan-outs of 7; zones 18/7/2/5; seed 6 (the binary 2^32 space)."""
+    return _wide(3, 7, 1, (18, 7, 2, 5), 6)
+
+
+def layered24() -> Scenario:
+    """N=24 random layered DAG (6 layers of 4, p=0.4), 2..16 GiB tools vs 40 GiB; seed 7.
+    No serialisation point: its binary space (2^24) is searched whole by the oracle."""
+    rng = np.random.default_rng(7)
+    c, g, x, m = _ordinary(rng, 24, 2048, 16384)
+    pred = _layered_edges(rng, [4] * 6, 0.4)
+    return Scenario(24, pred, c, g, x, [_load_from_vram(v) for v in m], m,
+                    40960, slowdown_linear(kmax=24))
+
+
+WIDE_NAMES = {
+    "wide28": "N=28 spine+3 fan-outs of 6, 4 zones, 32 GiB (3^28 mappings)",
+    "wide32": "N=32 spine+3 fan-outs of 7, 4 zones, 32 GiB (3^32 mappings; binary space 2^32)",
+    "layered24": "N=24 layered 6x4 p=0.4, 2-16 GiB vs 40 GiB (binary space, 2^24 mappings)",
+}
+
+
 def config(i: int):
     return (config0, config1, config2, config3, config4)[i]()
 
@@ -300,8 +371,29 @@ def random_small(rng: np.random.Generator, n: int, *, edge_p: float = 0.4,
     budget = int(rng.integers(5, 16)) if tight else 10 * n + 10
     if contention:
         f = [0, 1024]
-        for _ in range(2, MAX_TOOLS + 1):
+        for _ in range(2, max(ENUM_MAX_TOOLS, n) + 1):
             f.append(f[-1] + int(rng.integers(0, 700)))
     else:
-        f = slowdown_flat()
+        f = slowdown_flat(max(ENUM_MAX_TOOLS, n))
     return Scenario(n, pred, c, g, x, load, m, budget, f)
+
+
+def random_segmented(rng: np.random.Generator, n: int, *, seg_max: int = 6, edge_p: float = 0.4,
+                     **kw) -> Scenario:
+    """A ``random_small`` scenario whose DAG is a row of segments joined at
+    serialisation points: each segment's first tool has every tool of the
+    previous segment as a predecessor, and every other tool of a segment has at
+    least one predecessor inside it (random edges with probability ``edge_p``,
+    else the segment's first tool).  Segment lengths are uniform in 1..seg_max."""
+    base = random_small(rng, n, edge_p=0.0, **kw)
+    cuts = [0]
+    while cuts[-1] < n:
+        cuts.append(min(n, cuts[-1] + int(rng.integers(1, seg_max + 1))))
+    pred = [0] * n
+    for j in range(len(cuts) - 1):
+        lo, hi = cuts[j], cuts[j + 1]
+        pred[lo] = ((1 << lo) - 1) & ~((1 << cuts[j - 1]) - 1) if j else 0
+        for v in range(lo + 1, hi):
+            m = sum(1 << u for u in range(lo, v) if rng.uniform() < edge_p)
+            pred[v] = m or (1 << lo)
+    return Scenario(**{**base.to_dict(), "pred_mask": pred})

@@ -302,3 +302,89 @@ def check_fig7_whatif(lib):
 
 
 ALL_CHECKS.append(check_fig7_whatif)
+
+
+# ---------------------------------------------------------------------------
+# Scenarios of up to 32 tools, the binary decision space and the segment rule.
+# ---------------------------------------------------------------------------
+
+def check_wide_closed_forms(lib, seed=21):
+    """Closed forms at 21..32 tools (the last tool sits at bit 31 of every mask)."""
+    rng = np.random.default_rng(seed)
+    for n in (21, 27, 32):
+        c = [int(v) for v in rng.integers(1, 100000, n)]
+        g = [int(v) for v in rng.integers(1, 100000, n)]
+        x = [int(v) for v in rng.integers(0, 30000, n)]
+        l = [int(v) for v in rng.integers(0, 50000, n)]
+        m = [int(v) for v in rng.integers(1, 5000, n)]
+        scn = _chain(n, c, g, x, l, m, max(m), S.slowdown_linear(35, kmax=n))
+        ones = sum(3 ** i for i in range(n))
+        assert lib.evaluate(scn, 0) == sum(c)
+        assert lib.evaluate(scn, ones) == sum(g) + sum(x)
+        assert lib.evaluate(scn, 2 * ones) == sum(l) + sum(g) + sum(x)
+        for idx in rng.integers(0, 2 ** 62, 6):
+            idx = int(idx) % 3 ** n
+            modes = S.mapping_modes(idx, n)
+            dur = [(c[i], g[i] + x[i], l[i] + g[i] + x[i])[a] for i, a in enumerate(modes)]
+            assert lib.evaluate(scn, idx) == sum(dur), (n, idx)
+        # identical fan-out of n tools on gpu_now: each ends at ceil(w f[n] / 1024)
+        w = int(rng.integers(1, 200000))
+        f = S.slowdown_linear(int(rng.integers(0, 80)), kmax=n)
+        fan = Scenario(n, [0] * n, [10 ** 7] * n, [w] * n, [0] * n, [0] * n, [1] * n, n, f)
+        assert lib.evaluate(fan, ones) == -(-w * f[n] // 1024), (n, w)
+        # one tool over budget, at the top digit
+        big = Scenario(n, scn.pred_mask, c, g, x, l, m[:-1] + [max(m) + 1], max(m), scn.slowdown_q10)
+        assert lib.evaluate(big, 3 ** (n - 1)) == INF and lib.evaluate(big, 2 * 3 ** (n - 1)) == INF
+        # all-cpu mapping of a random DAG: its critical path
+        dag = S.random_small(rng, n, tight=True, max_time=500)
+        assert lib.evaluate(dag, 0) == _longest_path(dag, dag.cpu_us)
+
+
+def check_binary_space(lib, trials=40, seed=22):
+    """The binary (cpu/gpu_now) optimum: hand-worked values, and every binary mapping of small DAGs."""
+    for ex in _load("hand_examples.json")["examples"]:
+        scn = Scenario.from_dict(ex["scenario"])
+        members = [sum(3 ** i for i in range(scn.n) if (b >> i) & 1) for b in range(2 ** scn.n)]
+        if not all(str(i) in ex["expected"] for i in members):
+            continue
+        feas = [(ex["expected"][str(i)], i) for i in members if ex["expected"][str(i)] != INF]
+        want = min(feas)
+        assert lib.search_binary(scn) == (want[1], want[0]), ex["name"]
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 8))
+        scn = S.random_small(rng, n)
+        ms, fe = lib.eval_range(scn, 0, 3 ** n)
+        best = None
+        for b in range(2 ** n):
+            idx = sum(3 ** i for i in range(n) if (b >> i) & 1)
+            if fe[idx] and (best is None or (int(ms[idx]), idx) < best):
+                best = (int(ms[idx]), idx)
+        assert lib.search_binary(scn) == (best[1], best[0]), scn
+        lo = int(rng.integers(0, 2 ** n))
+        cnt = int(rng.integers(1, 2 ** n - lo + 1))
+        sub = [(int(ms[i]), i) for i in (sum(3 ** k for k in range(n) if (b >> k) & 1) for b in range(lo, lo + cnt))
+               if fe[i]]
+        got = lib.search_binary_range(scn, lo, cnt)
+        assert got == ((min(sub)[1], min(sub)[0]) if sub else (-1, INF)), (scn, lo, cnt)
+
+
+def check_segments(lib, trials=40, seed=23):
+    """Segment rule (oracle.segments): equal to full enumeration, and to the stored
+    brute-force optimum of the 19-tool workload."""
+    from oracle import segments
+    rng = np.random.default_rng(seed)
+    for t in range(trials):
+        n = int(rng.integers(2, 9))
+        scn = S.random_segmented(rng, n, seg_max=int(rng.choice([2, 3, 5])), tight=bool(t % 3),
+                                 max_time=int(rng.choice([8, 40, 500])))
+        assert segments.bounds(scn)[-1][1] == n
+        assert segments.search(scn, lib=lib) == lib.search(scn), scn
+        assert segments.search(scn, binary=True, lib=lib) == lib.search_binary(scn), scn
+        for idx in rng.integers(0, 3 ** n, 10):
+            assert segments.evaluate(scn, int(idx), lib=lib) == lib.evaluate(scn, int(idx)), (scn, idx)
+    golden = _load("config_results.json")["configs"]["3"]
+    assert segments.search(S.config3(), lib=lib) == (golden["summary"]["best_index"], golden["summary"]["best_makespan"])
+
+
+ALL_CHECKS += [check_wide_closed_forms, check_binary_space, check_segments]

@@ -52,7 +52,10 @@ def _with(**kw):
 
 INVALID = {
     "n=0": lambda: _with(n=0),
-    "n=21": lambda: S.Scenario(21, [0] * 21, [1] * 21, [1] * 21, [0] * 21, [0] * 21, [1] * 21, 10, S.slowdown_flat()),
+    "n=33": lambda: S.Scenario(33, [0] * 33, [1] * 33, [1] * 33, [0] * 33, [0] * 33, [1] * 33, 10,
+                               S.slowdown_flat(33)),
+    "f missing above k=20": lambda: S.Scenario(21, [0] * 21, [1] * 21, [1] * 21, [0] * 21, [0] * 21, [1] * 21, 10,
+                                               S.slowdown_flat()),
     "backward edge": lambda: _with(pred_mask=[0, 0, 1 << 5] + [0] * 5),
     "self loop": lambda: _with(pred_mask=[0, 1 << 1] + [0] * 6),
     "zero cpu": lambda: _with(cpu_us=[0] + _base().cpu_us[1:]),
@@ -112,3 +115,19 @@ def test_boundary_values_accepted(lib):
     s = S.Scenario(n, [0] + [1 << (i - 1) for i in range(1, n)], [1] * n, [(1 << 22) - 1] + [1] * 19,
                    [0] * n, [0] * n, [1 << 27] * n, 1 << 31, [0, 1024] + [65536] * 19)
     bf.validate_desc(s)
+
+
+def test_wide_desc_accepted(lib):
+    """32 tools validate; the enumerating batch search refuses more than 20 before touching the GPU."""
+    n = 32
+    s = S.Scenario(n, [0] + [1 << (i - 1) for i in range(1, n)], [1000] * n, [100] * n, [0] * n, [0] * n,
+                   [1] * n, 10, S.slowdown_linear(35, kmax=n))
+    bf.validate_desc(s)
+    bf.validate_desc(S.wide28())
+    bf.validate_desc(S.wide32())
+    bf.validate_desc(S.layered24())
+    descs = (bf.Desc * 1)(bf.to_desc(s))
+    out = (bf.CResult * 1)()
+    assert lib.bf_search_batch(descs, 1, out, None) == bf.BF_EINVAL
+    assert "n <= 20" in bf.last_error()
+    assert lib.bf_search_batch_noalloc(descs, 1, out, None) == bf.BF_EINVAL

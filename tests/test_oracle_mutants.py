@@ -29,6 +29,12 @@ MUTANTS = {
     "digits reversed": ("mode[i] = (int)(idx % 3);", "mode[n - 1 - i] = (int)(idx % 3);"),
     "argmin ties to higher index": ("(ms == makespan && idx < index)", "(ms == makespan && idx > index)"),
     "GPU tools not slowed by contention": ("(v_min - V) * s.slowdown[running_gpu]", "(v_min - V) * 1024"),
+    "binary member indexed in base 2": ("for (int i = 0; i < n; ++i, p *= 3)\n    if ((b >> i) & 1) idx += p;",
+                                        "for (int i = 0; i < n; ++i, p *= 2)\n    if ((b >> i) & 1) idx += p;"),
+    "binary member skips the top tool": ("for (int i = 0; i < n; ++i, p *= 3)\n    if ((b >> i) & 1) idx += p;",
+                                         "for (int i = 0; i + 1 < n; ++i, p *= 3)\n    if ((b >> i) & 1) idx += p;"),
+    "edges out of tool 30 ignored": ("if (((s.pred[v] >> u) & 1u) && status[u] != kDone) return false;",
+                                     "if (u != 30 && ((s.pred[v] >> u) & 1u) && status[u] != kDone) return false;"),
 }
 
 
