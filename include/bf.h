@@ -171,6 +171,49 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
  * the host. */
 int bf_search_pruned(const bf_scenario* scn, uint64_t hint_index, bf_result* out, void* cuda_stream);
 
+/* Decision spaces of bf_search_tree: the full space (each tool on cpu,
+ * gpu_now or gpu_queue; 3^n mappings) or the binary space the paper's S1-S10
+ * use (§4.1: each tool on the CPU or the GPU, i.e. cpu or gpu_now; 2^n
+ * mappings).  The value is the number of modes per tool. */
+#define BF_SPACE_BINARY 2u
+#define BF_SPACE_FULL 3u
+/* bf_search_tree flag: simulate every mapping of the space (no pruning). */
+#define BF_TREE_NO_PRUNE 1u
+
+/* What a tree search did (bf_search_tree, optional). */
+typedef struct bf_tree_stats {
+  uint64_t nodes;         /* prefix nodes created (tools assigned in index order), root included */
+  uint64_t leaf_nodes;    /* nodes whose last leaf_depth tools were enumerated */
+  uint64_t leaves;        /* mappings simulated to the end (at most leaf_nodes * modes^leaf_depth) */
+  uint32_t launches;      /* kernel launches */
+  uint32_t leaf_depth;    /* tools enumerated below each leaf node */
+  uint32_t incumbent_us;  /* the starting bound (0xFFFFFFFF with BF_TREE_NO_PRUNE) */
+  uint32_t pad;
+} bf_tree_stats;
+
+/* The optimum of a decision space -- the feasible mapping of lowest makespan,
+ * ties to the lowest canonical index, exactly as full enumeration would give
+ * it -- for scenarios of up to 32 tools (3^32 ~ 1.9e15 mappings), by depth-
+ * first branch and bound over the modes of tools 0, 1, 2, ... in index order.
+ * A node (the modes of tools [0, d)) carries the simulation state at the
+ * first instant a tool >= d could become ready, shared by all its mappings.
+ * A node is dropped when a lower bound on all of its mappings' makespans
+ * exceeds the best makespan known (strictly, so the optimum and its ties
+ * survive): running tools end no earlier than their remaining work at
+ * isolated speed allows, a tool not started ends no earlier than its duration
+ * in its mode (or min(c, g + x) if open) after the node's time, each tool's
+ * successors add the longest path through them in minimum durations, and
+ * queued tools run one at a time.  The first bound is the best of a few
+ * mappings of the space (hint_index if it lies in it, all-cpu, all-gpu_now,
+ * each tool on its isolated-faster device, all-gpu_queue); better ones are
+ * found as the search proceeds.  space: BF_SPACE_FULL or BF_SPACE_BINARY.
+ * flags: 0 or BF_TREE_NO_PRUNE (every mapping of the space is simulated:
+ * full enumeration).  `stats` may be NULL.  Allocates level buffers in the
+ * handle on first use (about 1.7 GB for 32 tools in the full space).  Blocks
+ * until the result is on the host; every level step is a bounded wait. */
+int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint64_t hint_index,
+                   bf_result* out, bf_tree_stats* stats, void* cuda_stream);
+
 /* Makespans and feasibility of an arbitrary list of mappings: d_makespan[j] and
  * d_feasible[j] for mapping d_indices[j] (all three caller-owned device arrays
  * of >= count elements).  An index >= 3^n yields makespan 0xFFFFFFFF and

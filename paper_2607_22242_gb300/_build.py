@@ -1,9 +1,10 @@
 """Build ``libbf.so`` in-tree with nvcc for sm_103a (GB300).
 
 Each window-width bucket of ``csrc/bf_kernels.cu`` is its own translation unit
-(``-DBF_NW=<slots>``); the units compile in parallel and link with ``bf_capi.cu``
-into ``paper_2607_22242_gb300/_build/libbf.so`` (CUDA runtime linked
-statically, so the library carries no path to a toolkit).
+(``-DBF_NW=<slots>``); the units compile in parallel and link with ``bf_tree.cu``
+(the tree search and 32-slot index lists) and ``bf_capi.cu`` into
+``paper_2607_22242_gb300/_build/libbf.so`` (CUDA runtime linked statically, so
+the library carries no path to a toolkit; no undefined symbol is allowed).
 """
 from __future__ import annotations
 
@@ -31,7 +32,8 @@ def nvcc() -> str:
 
 
 def _sources():
-    return [os.path.join(CSRC, f) for f in sorted(os.listdir(CSRC))] + [os.path.join(INCLUDE, "bf.h")]
+    return ([os.path.join(CSRC, f) for f in sorted(os.listdir(CSRC))] + [os.path.join(INCLUDE, "bf.h")]
+            + [os.path.abspath(__file__)])  # the build recipe itself
 
 
 def _fingerprint(extra) -> str:
@@ -60,8 +62,9 @@ def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
         obj = os.path.join(BUILD_DIR, f"bf_kernels_nw{nt}.o")
         jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, f"-DBF_NW={nt}", "-c",
                      os.path.join(CSRC, "bf_kernels.cu"), "-o", obj])
-    capi_obj = os.path.join(BUILD_DIR, "bf_capi.o")
-    jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, "bf_capi.cu"), "-o", capi_obj])
+    for unit in ("bf_tree", "bf_capi"):
+        jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, unit + ".cu"), "-o",
+                     os.path.join(BUILD_DIR, unit + ".o")])
 
     def run(cmd):
         res = subprocess.run(cmd, capture_output=True, text=True)
@@ -75,7 +78,7 @@ def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
     with cf.ThreadPoolExecutor(workers) as pool:
         objs = list(pool.map(run, jobs))
     tmp = LIB_PATH + f".tmp{os.getpid()}"
-    run([cc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs])
+    run([cc, *ARCH, "-shared", "-cudart", "static", "-Xlinker", "--no-undefined", "-o", tmp, *objs])
     os.replace(tmp, LIB_PATH)
     with open(stamp, "w") as fh:
         fh.write(fp)

@@ -29,8 +29,10 @@ STATUS_NAMES = {0: "BF_OK", 1: "BF_EINVAL", 2: "BF_ERANGE", 3: "BF_ENOMEM", 4: "
 INFEASIBLE = 0xFFFFFFFF
 EXPORTED = ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
             "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc",
-            "bf_eval_indices", "bf_whatif", "bf_search_pruned", "bf_set_wait_timeout_ms", "bf_last_error",
-            "bf_version")
+            "bf_eval_indices", "bf_whatif", "bf_search_pruned", "bf_search_tree", "bf_set_wait_timeout_ms",
+            "bf_last_error", "bf_version")
+SPACE_BINARY, SPACE_FULL = 2, 3
+TREE_NO_PRUNE = 1
 MAX_PROBES = 2 * MAX_TOOLS + MAX_TOOLS * MAX_TOOLS
 NOALLOC_MAX_SCENARIOS = 1024
 
@@ -78,6 +80,13 @@ class Probe:
     feasible: bool
 
 
+class CTreeStats(ctypes.Structure):
+    """``bf_tree_stats``."""
+    _fields_ = [("nodes", ctypes.c_uint64), ("leaf_nodes", ctypes.c_uint64), ("leaves", ctypes.c_uint64),
+                ("launches", ctypes.c_uint32), ("leaf_depth", ctypes.c_uint32), ("incumbent_us", ctypes.c_uint32),
+                ("pad", ctypes.c_uint32)]
+
+
 @dataclasses.dataclass
 class Result:
     index: int
@@ -109,9 +118,10 @@ def load(path: str = LIB_PATH):
     lib.bf_eval_indices.argtypes = [vp, vp, u64, vp, vp, vp]
     lib.bf_whatif.argtypes = [vp, u64, ctypes.POINTER(CProbe), u32, ctypes.POINTER(u32), vp]
     lib.bf_search_pruned.argtypes = [vp, u64, ctypes.POINTER(CResult), vp]
+    lib.bf_search_tree.argtypes = [vp, u32, u32, u64, ctypes.POINTER(CResult), ctypes.POINTER(CTreeStats), vp]
     for name in ("bf_validate_desc", "bf_create_scenario", "bf_destroy_scenario", "bf_eval_mappings",
                  "bf_search_best", "bf_search_range", "bf_search_batch", "bf_search_batch_noalloc",
-                 "bf_eval_indices", "bf_whatif", "bf_search_pruned"):
+                 "bf_eval_indices", "bf_whatif", "bf_search_pruned", "bf_search_tree"):
         getattr(lib, name).restype = ctypes.c_int
     lib.bf_set_wait_timeout_ms.argtypes = [u32]
     lib.bf_set_wait_timeout_ms.restype = None
@@ -369,6 +379,25 @@ def search_pruned(h: Union[ScenarioHandle, Scenario], hint_index: Optional[int] 
         hint = (1 << 64) - 1 if hint_index is None else hint_index
         _check(load().bf_search_pruned(handle.ptr, hint, ctypes.byref(r), ctypes.c_void_p(_stream_handle(stream))))
         return _result(r, handle.scenario.n)
+    finally:
+        if owned:
+            handle.close()
+
+
+def search_tree(h: Union[ScenarioHandle, Scenario], space: int = SPACE_FULL, prune: bool = True,
+                hint_index: Optional[int] = None, stream=None) -> Tuple[Result, dict]:
+    """Optimum of the full (space=3) or binary cpu/gpu_now (space=2) decision space of a scenario of up to
+    32 tools, by depth-first branch and bound (prune=False: every mapping simulated); (result, stats)."""
+    handle, owned = _handle(h)
+    try:
+        r = CResult()
+        st = CTreeStats()
+        hint = (1 << 64) - 1 if hint_index is None else hint_index
+        _check(load().bf_search_tree(handle.ptr, space, 0 if prune else TREE_NO_PRUNE, hint, ctypes.byref(r),
+                                     ctypes.byref(st), ctypes.c_void_p(_stream_handle(stream))))
+        stats = dict(nodes=st.nodes, leaf_nodes=st.leaf_nodes, leaves=st.leaves, launches=st.launches,
+                     leaf_depth=st.leaf_depth, incumbent_us=st.incumbent_us)
+        return _result(r, handle.scenario.n), stats
     finally:
         if owned:
             handle.close()

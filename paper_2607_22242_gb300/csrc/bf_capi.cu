@@ -6,6 +6,7 @@
 #include <atomic>
 #include <chrono>
 #include <cstdarg>
+#include <cstddef>
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
@@ -16,13 +17,19 @@
 #include "../../include/bf.h"
 #include "bf_launch.h"
 #include "bf_plan.h"
+#include "bf_tree.h"
 
 // Per-handle scratch, one block on the device and a pinned mirror on the host:
-// the packed search key and the what-if probe list with its results.
+// the packed search key, the tree search's best record, bound and counters,
+// and the what-if probe list with its results.
 struct bf_scratch {
   unsigned long long key;
   uint32_t survivors;   // pruned search: number of surviving prefixes
   uint32_t pad;
+  bfk::BestRecord best;      // tree search: best (makespan, index) so far
+  uint32_t bound;            // tree search: makespan bound for pruning
+  uint32_t level_count;      // tree search: nodes appended by the last expansion
+  bfk::TreeCounters ctr;     // tree search: counters and error bits
   uint64_t idx[BF_MAX_PROBES];
   uint32_t ms[BF_MAX_PROBES];
   uint8_t fe[BF_MAX_PROBES];
@@ -30,6 +37,7 @@ struct bf_scratch {
 
 struct bf_scenario {
   bf_scenario_desc desc;
+  bfk::TablesW wide;    // all n tools, 32 slots (index lists and the tree search)
   bfk::Tables tables;   // all n tools (n <= BF_MAX_TOOLS_ENUM; zero otherwise)
   bfk::Tables window;   // tools [W0, n), renumbered from 0
   bfk::Plan plan;       // enumeration split and window (see bfk::Plan), full range
@@ -39,6 +47,8 @@ struct bf_scenario {
   unsigned long long* d_key;  // &d_scratch->key
   unsigned long long* h_key;  // &h_scratch->key
   uint32_t* d_survivors;      // pruned search: 3^P prefix slots, allocated on first use
+  uint32_t* d_levels;         // tree search: node buffers of every level, allocated on first use
+  size_t levels_bytes;
 };
 
 namespace {
@@ -186,6 +196,19 @@ void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* 
     default: { e = bfk::CALL(20); } break;                \
   }
 
+// Index-list evaluation: the 20-slot kernels up to 20 tools, the 32-slot one above.
+cudaError_t launch_list(const bf_scenario* scn, const uint64_t* idx, uint64_t count, uint32_t* ms, uint8_t* fe,
+                        int grid, cudaStream_t st) {
+  const uint32_t n = scn->desc.n;
+  const uint64_t total = pow3(n);
+  if (n > BF_MAX_TOOLS_ENUM) return bfk::launch_wide_list(scn->wide, total, idx, count, ms, fe, grid, st);
+  cudaError_t e = cudaSuccess;
+#define CALL(NW) launch_list_nw##NW(scn->tables, total, idx, count, ms, fe, grid, st)
+  BF_DISPATCH(bfk::bucket_for(n), CALL)
+#undef CALL
+  return e;
+}
+
 int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result* out,
                cudaStream_t st, const char* who) {
   cudaError_t e = cudaMemsetAsync(scn->d_key, 0xFF, sizeof(unsigned long long), st);
@@ -219,6 +242,7 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   if (!s) return fail(BF_ENOMEM, "bf_create_scenario: host allocation failed");
   std::memset(s, 0, sizeof *s);
   s->desc = *desc;
+  build_tables(desc, &s->wide);
   if (desc->n <= BF_MAX_TOOLS_ENUM) {
     build_tables(desc, &s->tables);
     split_and_window(s->tables, &s->plan, &s->window);
@@ -241,6 +265,7 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
 int bf_destroy_scenario(bf_scenario* scn) {
   if (!scn) return BF_OK;
   if (scn->d_survivors) cudaFree(scn->d_survivors);
+  if (scn->d_levels) cudaFree(scn->d_levels);
   cudaError_t e1 = scn->d_scratch ? cudaFree(scn->d_scratch) : cudaSuccess;
   cudaError_t e2 = scn->h_scratch ? cudaFreeHost(scn->h_scratch) : cudaSuccess;
   delete scn;
@@ -289,7 +314,6 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count, bf_r
 int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t count, uint32_t* d_makespan,
                     uint8_t* d_feasible, void* cuda_stream) {
   if (!scn) return fail(BF_EINVAL, "bf_eval_indices: scenario is NULL");
-  if (require_enum(scn->desc, "bf_eval_indices") != BF_OK) return BF_EINVAL;
   if (count == 0) return BF_OK;
   if (!d_indices || !d_makespan || !d_feasible) return fail(BF_EINVAL, "bf_eval_indices: NULL buffer");
   int sms = 0;
@@ -297,11 +321,7 @@ int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t 
   if (e != cudaSuccess) return cuda_fail(e, "bf_eval_indices");
   const uint64_t need = (count + bfk::kThreads - 1) / bfk::kThreads, cap = (uint64_t)sms * 16;
   const int grid = (int)(need < cap ? need : cap);
-  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  const uint64_t total = pow3(scn->desc.n);
-#define CALL(NW) launch_list_nw##NW(scn->tables, total, d_indices, count, d_makespan, d_feasible, grid, st)
-  BF_DISPATCH(bfk::bucket_for(scn->desc.n), CALL)
-#undef CALL
+  e = launch_list(scn, d_indices, count, d_makespan, d_feasible, grid, static_cast<cudaStream_t>(cuda_stream));
   if (e != cudaSuccess) return cuda_fail(e, "bf_eval_indices");
   return BF_OK;
 }
@@ -310,7 +330,6 @@ int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32
               void* cuda_stream) {
   const char* who = "bf_whatif";
   if (!scn || !out || !count) return fail(BF_EINVAL, "%s: NULL argument", who);
-  if (require_enum(scn->desc, who) != BF_OK) return BF_EINVAL;
   const uint32_t n = scn->desc.n;
   const uint64_t total = pow3(n);
   if (base_index >= total)
@@ -343,11 +362,7 @@ int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   bf_scratch* dv = scn->d_scratch;
   cudaError_t e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) {
-#define CALL(NW) launch_list_nw##NW(scn->tables, total, dv->idx, nc, dv->ms, dv->fe, 1 + (int)(nc / bfk::kThreads), st)
-    BF_DISPATCH(bfk::bucket_for(n), CALL)
-#undef CALL
-  }
+  if (e == cudaSuccess) e = launch_list(scn, dv->idx, nc, dv->ms, dv->fe, 1 + (int)(nc / bfk::kThreads), st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(h->ms, dv->ms, sizeof(uint32_t) * nc, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(h->fe, dv->fe, nc, cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) return cuda_fail(e, who);
@@ -426,11 +441,7 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
     h->idx[nc++] = fast;
   }
   e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) {
-#define CALL(NW) launch_list_nw##NW(scn->tables, total, dv->idx, nc, dv->ms, dv->fe, 1, st)
-    BF_DISPATCH(bfk::bucket_for(n), CALL)
-#undef CALL
-  }
+  if (e == cudaSuccess) e = launch_list(scn, dv->idx, nc, dv->ms, dv->fe, 1, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(h->ms, dv->ms, sizeof(uint32_t) * nc, cudaMemcpyDeviceToHost, st);
   if (e == cudaSuccess) e = cudaMemcpyAsync(h->fe, dv->fe, nc, cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) return cuda_fail(e, who);
@@ -484,6 +495,174 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   rc = wait_stream(st, who);
   if (rc != BF_OK) return rc;
   fill_result(*scn->h_key, n, 0, out);
+  return BF_OK;
+}
+
+int bf_search_tree(const bf_scenario* scn_const, uint32_t space, uint32_t flags, uint64_t hint_index,
+                   bf_result* out, bf_tree_stats* stats, void* cuda_stream) {
+  const char* who = "bf_search_tree";
+  if (!scn_const || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
+  if (space != BF_SPACE_BINARY && space != BF_SPACE_FULL)
+    return fail(BF_EINVAL, "%s: space %u is neither BF_SPACE_BINARY (2) nor BF_SPACE_FULL (3)", who, space);
+  if (flags & ~(uint32_t)BF_TREE_NO_PRUNE) return fail(BF_EINVAL, "%s: unknown flags 0x%x", who, flags);
+  // The handle's lazily allocated level buffers are scratch, not state.
+  bf_scenario* scn = const_cast<bf_scenario*>(scn_const);
+  const bfk::TablesW& tb = scn->wide;
+  const uint32_t n = scn->desc.n, R = space;
+  const bool prune = !(flags & BF_TREE_NO_PRUNE);
+  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+
+  // Constants: the leaf depth, the bound's per-tool durations, digit powers.
+  bfk::TreeConsts tc;
+  std::memset(&tc, 0, sizeof tc);
+  tc.n = n;
+  tc.radix = R;
+  tc.D = n < (R == 3 ? 5u : 8u) ? n : (R == 3 ? 5u : 8u);
+  tc.leaf_level = n - tc.D;
+  tc.combos = 1;
+  for (uint32_t i = 0; i < tc.D; ++i) tc.combos *= R;
+  tc.prune = prune ? 1u : 0u;
+  {
+    uint64_t down[bfk::kTreeSlots] = {0};
+    for (int v = (int)n - 1; v >= 0; --v) {
+      const uint32_t gpu = tb.wnow[v] >> 10;
+      tc.dmin[v] = tb.cpu[v] < gpu ? tb.cpu[v] : gpu;
+      uint64_t longest = 0;
+      for (uint32_t w = (uint32_t)v + 1; w < n; ++w)
+        if ((tb.succ[v] >> w) & 1u) longest = down[w] > longest ? down[w] : longest;
+      tc.sdown[v] = (uint32_t)(longest < 0xFFFFFFFFull ? longest : 0xFFFFFFFFull);
+      down[v] = tc.dmin[v] + longest;
+    }
+    uint64_t p = 1;
+    for (uint32_t i = 0; i < (uint32_t)bfk::kTreeSlots; ++i, p *= 3) tc.pow3[i] = p;
+  }
+
+  // Level buffers: level d holds up to R * kPop nodes (one pop of its parent
+  // level); nodes are popped from the deepest non-empty level, so no level
+  // ever holds more.
+  constexpr uint32_t kPop = 65536;
+  const uint32_t cap = R * kPop;
+  const uint32_t levels = tc.leaf_level + 1;
+  const size_t level_words = bfk::tree_node_words() * cap;
+  const size_t need = sizeof(uint32_t) * level_words * levels;
+  cudaError_t e = cudaSuccess;
+  if (scn->levels_bytes < need) {
+    if (scn->d_levels) cudaFree(scn->d_levels);
+    scn->d_levels = nullptr;
+    scn->levels_bytes = 0;
+    e = lib_malloc(reinterpret_cast<void**>(&scn->d_levels), need);
+    if (e != cudaSuccess) return cuda_fail(e, who);
+    scn->levels_bytes = need;
+  }
+  auto level = [&](uint32_t d) { return scn->d_levels + level_words * d; };
+
+  bf_scratch* h = scn->h_scratch;
+  bf_scratch* dv = scn->d_scratch;
+  uint32_t launches = 0;
+
+  // 1. Incumbent: the best feasible of a few mappings of the space (the hint
+  //    if it lies in it, all-cpu, all-gpu_now, each tool on its isolated-faster
+  //    device, and all-gpu_queue in the full space).
+  uint32_t bound = 0xFFFFFFFFu;
+  if (prune) {
+    const uint64_t total = pow3(n);
+    uint32_t nc = 0;
+    bool hint_ok = hint_index < total;
+    if (hint_ok && R == 2)
+      for (uint64_t v = hint_index; v; v /= 3) hint_ok = hint_ok && (v % 3 != 2);
+    if (hint_ok) h->idx[nc++] = hint_index;
+    uint64_t now = 0, fast = 0, p = 1;
+    for (uint32_t i = 0; i < n; ++i, p *= 3) {
+      now += p;
+      if ((tb.wnow[i] >> 10) < tb.cpu[i]) fast += p;
+    }
+    h->idx[nc++] = 0;
+    h->idx[nc++] = now;
+    h->idx[nc++] = fast;
+    if (R == 3) h->idx[nc++] = 2 * now;
+    e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = launch_list(scn, dv->idx, nc, dv->ms, dv->fe, 1, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(h->ms, dv->ms, sizeof(uint32_t) * nc, cudaMemcpyDeviceToHost, st);
+    if (e == cudaSuccess) e = cudaMemcpyAsync(h->fe, dv->fe, nc, cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(e, who);
+    const int rc = wait_stream(st, who);
+    if (rc != BF_OK) return rc;
+    ++launches;
+    for (uint32_t j = 0; j < nc; ++j)
+      if (h->fe[j] == 1 && h->ms[j] < bound) bound = h->ms[j];
+  }
+
+  // 2. Reset the record, bound and counters; write the root node.
+  h->best.ms = ~0ull;
+  h->best.idx = ~0ull;
+  h->bound = bound;
+  h->level_count = 0;
+  std::memset(&h->ctr, 0, sizeof h->ctr);
+  e = cudaMemcpyAsync(&dv->best, &h->best,
+                      offsetof(bf_scratch, idx) - offsetof(bf_scratch, best), cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = bfk::launch_tree_root(tb, level(0), cap, st);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  ++launches;
+
+  // 3. Depth first over levels: pop up to kPop nodes (a whole leaf-level
+  //    buffer) from the deepest non-empty level, and expand them into the
+  //    next level or enumerate their leaves.
+  std::vector<uint32_t> size(levels, 0);
+  size[0] = 1;
+  uint64_t nodes = 1;
+  for (;;) {
+    int d = (int)levels - 1;
+    while (d >= 0 && size[d] == 0) --d;
+    if (d < 0) break;
+    const uint32_t L = (uint32_t)d;
+    const uint32_t take = L == tc.leaf_level ? size[L] : (size[L] < kPop ? size[L] : kPop);
+    const uint32_t lo = size[L] - take;
+    size[L] = lo;
+    if (L == tc.leaf_level) {
+      e = bfk::launch_tree_leaf(tb, tc, level(L), cap, lo, take, 16384, &dv->bound, &dv->best, &dv->ctr, st);
+      if (e != cudaSuccess) return cuda_fail(e, who);
+      ++launches;
+      continue;
+    }
+    e = cudaMemsetAsync(&dv->level_count, 0, sizeof(uint32_t), st);
+    if (e == cudaSuccess)
+      e = bfk::launch_tree_expand(tb, tc, level(L), cap, lo, take, L, level(L + 1), cap, &dv->level_count,
+                                  &dv->bound, &dv->ctr, st);
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(&h->level_count, &dv->level_count, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+    if (e != cudaSuccess) return cuda_fail(e, who);
+    const int rc = wait_stream(st, who);
+    if (rc != BF_OK) return rc;
+    ++launches;
+    size[L + 1] = h->level_count;
+    nodes += h->level_count;
+  }
+
+  // 4. The record.
+  e = cudaMemcpyAsync(&h->best, &dv->best,
+                      offsetof(bf_scratch, idx) - offsetof(bf_scratch, best), cudaMemcpyDeviceToHost, st);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  const int rc = wait_stream(st, who);
+  if (rc != BF_OK) return rc;
+  if (h->ctr.error) return fail(BF_ECUDA, "%s: internal error 0x%x in the tree kernels", who, h->ctr.error);
+  std::memset(out, 0, sizeof *out);
+  if (h->best.ms >= 0xFFFFFFFFull) {
+    out->makespan_us = 0xFFFFFFFFu;
+  } else {
+    out->index = h->best.idx;
+    out->makespan_us = (uint32_t)h->best.ms;
+    out->feasible = 1;
+    uint64_t idx = out->index;
+    for (uint32_t i = 0; i < n; ++i, idx /= 3) out->mode[i] = (uint8_t)(idx % 3);
+  }
+  if (stats) {
+    stats->nodes = nodes;
+    stats->leaf_nodes = h->ctr.leaf_nodes;
+    stats->leaves = h->ctr.leaves;
+    stats->launches = launches;
+    stats->leaf_depth = tc.D;
+    stats->incumbent_us = bound;
+  }
   return BF_OK;
 }
 

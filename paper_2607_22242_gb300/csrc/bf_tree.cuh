@@ -1,0 +1,212 @@
+// bf_tree.cuh -- the tree search: exact branch and bound over mode prefixes,
+// for scenarios of up to 32 tools, over the full decision space (3 modes per
+// tool) or the binary cpu/gpu_now space (§4.1: S1-S10 choose between CPU and
+// GPU only).
+//
+// A node at level d assigns modes to tools [0, d) and holds the simulation
+// state at its checkpoint: the first instant at which a tool >= d would
+// become ready (bf_sim.cuh, resumable runs).  Until then no tool >= d has
+// started, so that state is shared by every mapping extending the node.  A
+// child assigns tool d and resumes the parent's state up to its own
+// checkpoint.  Nodes at the leaf level L = n - D are not expanded further:
+// the leaf kernel resumes each one for all radix^D modes of the last D tools
+// and simulates them to the end.
+//
+// Pruning (Plan::bound's rule, with a per-node bound): the makespan of every
+// mapping extending a node is at least the node's lower bound (below); a node
+// whose bound exceeds the best makespan found so far (strictly) is dropped.
+// The optimum and all its ties have every prefix within the bound, so the
+// search returns the same (makespan, lowest index) as full enumeration.
+#pragma once
+
+#include "bf_sim.cuh"
+
+namespace bfk {
+
+constexpr int kTreeSlots = 32;
+using TablesW = TablesT<kTreeSlots>;
+using SmemTablesW = SmemTablesT<kTreeSlots>;
+
+// Per-scenario constants of a tree search.
+struct TreeConsts {
+  uint32_t n;
+  uint32_t radix;        // 2: {cpu, gpu_now}; 3: {cpu, gpu_now, gpu_queue}
+  uint32_t leaf_level;   // L: nodes at this level go to the leaf kernel
+  uint32_t D;            // n - L tools enumerated per leaf node
+  uint32_t combos;       // radix^D
+  uint32_t prune;        // 0: keep every node (full enumeration)
+  uint32_t dmin[kTreeSlots];   // min(c, g + x): no mode runs tool v faster
+  uint32_t sdown[kTreeSlots];  // longest path in dmin through v's successors (0 for a sink)
+  uint64_t pow3[kTreeSlots];
+};
+
+// A saved node: the state's words, then the digit masks; [word][node] layout
+// with stride `cap` (nodes of one level sit side by side, so a warp's accesses
+// to one word coalesce).
+template <int NT>
+struct NodeWords {
+  static constexpr int value = 2 * NT + 11;
+};
+
+template <int NT>
+__device__ __forceinline__ void store_node(const State<NT>& s, Digits dg, uint32_t* buf, uint32_t cap, uint32_t j) {
+  uint32_t* p = buf + j;
+#pragma unroll
+  for (int i = 0; i < NT; ++i) {
+    p[(size_t)(2 * i) * cap] = s.ec[i];
+    p[(size_t)(2 * i + 1) * cap] = s.eg[i];
+  }
+  p += (size_t)(2 * NT) * cap;
+  p[0 * (size_t)cap] = s.done;
+  p[1 * (size_t)cap] = s.pend;
+  p[2 * (size_t)cap] = s.run_g;
+  p[3 * (size_t)cap] = s.qwait;
+  p[4 * (size_t)cap] = s.T;
+  p[5 * (size_t)cap] = s.V;
+  p[6 * (size_t)cap] = s.L;
+  p[7 * (size_t)cap] = s.tc;
+  p[8 * (size_t)cap] = s.gmin;
+  p[9 * (size_t)cap] = dg.now;
+  p[10 * (size_t)cap] = dg.que;
+}
+
+template <int NT>
+__device__ __forceinline__ void load_node(const uint32_t* buf, uint32_t cap, uint32_t j, State<NT>& s, Digits& dg) {
+  const uint32_t* p = buf + j;
+#pragma unroll
+  for (int i = 0; i < NT; ++i) {
+    s.ec[i] = p[(size_t)(2 * i) * cap];
+    s.eg[i] = p[(size_t)(2 * i + 1) * cap];
+  }
+  p += (size_t)(2 * NT) * cap;
+  s.done = p[0 * (size_t)cap];
+  s.pend = p[1 * (size_t)cap];
+  s.run_g = p[2 * (size_t)cap];
+  s.qwait = p[3 * (size_t)cap];
+  s.T = p[4 * (size_t)cap];
+  s.V = p[5 * (size_t)cap];
+  s.L = p[6 * (size_t)cap];
+  s.tc = p[7 * (size_t)cap];
+  s.gmin = p[8 * (size_t)cap];
+  dg.now = p[9 * (size_t)cap];
+  dg.que = p[10 * (size_t)cap];
+}
+
+// Lower bound on the makespan of every mapping that extends a node whose
+// state `s` is at a checkpoint (before the admission at s.T), with the modes
+// of the tools in `known` given by `dg`:
+//   * a running CPU tool ends at ec (exact);
+//   * a running GPU tool with r work units left ends no earlier than
+//     T + ceil(r / 1024): f[k] >= f[1] = 1024, and the model rounds GPU
+//     progress down and completion times up;
+//   * a tool not started by T ends no earlier than T + its duration in its
+//     mode (c, g + x or l + g + x), or T + min(c, g + x) if its mode is open;
+//   * after a tool ends, its successors still need the longest path through
+//     them in minimum durations (sdown);
+//   * queued tools run one at a time, so all unfinished tools known to be
+//     queued end no earlier than T + the sum of their remaining durations.
+template <int NT, typename TB>
+__device__ __forceinline__ uint64_t lower_bound(const State<NT>& s, const TB& tb, const TreeConsts& tc, Digits dg,
+                                                uint32_t known) {
+  const uint64_t T = s.T;
+  uint64_t lb = T, qsum = 0u;
+#pragma unroll
+  for (int v = 0; v < NT; ++v) {
+    const uint32_t bit = 1u << v;
+    if (s.done & bit) continue;
+    uint64_t fin;
+    if (s.ec[v] != 0xFFFFFFFFu) {
+      fin = s.ec[v];
+    } else if (s.run_g & bit) {
+      const uint32_t left = ((s.eg[v] - s.V) >> 10) + (((s.eg[v] - s.V) & 1023u) != 0u);
+      fin = T + left;
+      if (dg.que & bit) qsum += left;
+    } else {
+      uint32_t d = tc.dmin[v];
+      if (known & bit) {
+        d = (dg.now & bit) ? (tb.wnow[v] >> 10) : (dg.que & bit) ? (tb.wq[v] >> 10) : tb.cpu[v];
+        if (dg.que & bit) qsum += d;
+      }
+      fin = T + d;
+    }
+    lb = max(lb, fin + tc.sdown[v]);
+  }
+  return max(lb, T + qsum);
+}
+
+// Child (tool d in mode a) of the node whose state and digits are in s / dg,
+// advanced in place to the child's checkpoint.  Returns false when every
+// mapping below the child is infeasible or, with pruning, provably worse
+// than `bound`.  Requires d + 1 < n.
+template <int NT, typename TB, typename SD>
+__device__ __forceinline__ bool expand_child(const TB& tb, const SD& sd, const uint32_t* rt, const TreeConsts& tc,
+                                             State<NT>& s, Digits& dg, uint32_t d, uint32_t a, uint32_t bound) {
+  const uint32_t bit = 1u << d;
+  if (a == 1u) dg.now |= bit;
+  if (a == 2u) {
+    if (tb.big_mask & bit) return false;  // a queued tool with m > M never starts
+    dg.que |= bit;
+  }
+  const uint32_t assigned = (bit << 1) - 1u;  // tools [0, d]; all ones for d = 31
+  if (run<NT>(s, tb, sd, rt, dg, tb.all_mask & ~assigned) != kRunStopped) return false;
+  return !tc.prune || lower_bound<NT>(s, tb, tc, dg, assigned) <= (uint64_t)bound;
+}
+
+// Digits of leaf combination c (tools [L, n)), as masks shifted to tool L.
+__device__ __forceinline__ Digits leaf_digits(uint32_t c, uint32_t radix, uint32_t D, uint32_t L) {
+  if (radix == 2u) return Digits{c << L, 0u};
+  const Digits d = decode(c, D);
+  return Digits{d.now << L, d.que << L};
+}
+
+// Canonical index of a mapping given as digit masks.
+__device__ __forceinline__ uint64_t index_of(Digits dg, const uint64_t* pow3) {
+  uint64_t idx = 0;
+  for (uint32_t m = dg.now; m; m &= m - 1u) idx += pow3[__ffs(m) - 1];
+  for (uint32_t m = dg.que; m; m &= m - 1u) idx += 2u * pow3[__ffs(m) - 1];
+  return idx;
+}
+
+// a < b in canonical index order: the highest tool whose digits differ decides.
+__device__ __forceinline__ bool index_less(Digits a, Digits b) {
+  const uint32_t diff = (a.now ^ b.now) | (a.que ^ b.que);
+  if (diff == 0u) return false;
+  const uint32_t top = 1u << (31 - __clz(diff));
+  const uint32_t da = ((a.now & top) ? 1u : 0u) + ((a.que & top) ? 2u : 0u);
+  const uint32_t db = ((b.now & top) ? 1u : 0u) + ((b.que & top) ? 2u : 0u);
+  return da < db;
+}
+
+// Best mapping seen: lowest makespan, ties to the lowest index.
+struct LaneBest {
+  uint32_t ms = kInfeasible;
+  Digits dg{0u, 0u};
+  __device__ __forceinline__ void offer(uint32_t m, Digits d) {
+    if (m < ms || (m == ms && m != kInfeasible && index_less(d, dg))) {
+      ms = m;
+      dg = d;
+    }
+  }
+};
+
+// Simulate combinations [c0, c1) of the leaf node saved in `slot` (a lane's
+// shared-memory state, stride `stride`) whose digits are `dg`; `valid` false
+// runs the loop without work (lanes of a warp stay in lockstep).
+template <int NT, typename TB, typename SD>
+__device__ __forceinline__ void leaf_combos(const TB& tb, const SD& sd, const uint32_t* rt, const TreeConsts& tc,
+                                            const uint32_t* slot, uint32_t stride, Digits dg, bool valid,
+                                            uint32_t c0, uint32_t c1, LaneBest& best) {
+  const uint32_t L = tc.leaf_level;
+  for (uint32_t c = c0; c < c1; ++c) {
+    if (!valid) continue;
+    const Digits dc = leaf_digits(c, tc.radix, tc.D, L);
+    const Digits full{dg.now | dc.now, dg.que | dc.que};
+    if (full.que & tb.big_mask) continue;
+    State<NT> w;
+    load_lane(slot, stride, w);
+    if (run<NT>(w, tb, sd, rt, full, 0u) != kRunFinished) continue;
+    best.offer(w.T, full);
+  }
+}
+
+}  // namespace bfk

@@ -5,6 +5,7 @@
   python -m paper_2607_22242_gb300.profile_case --kernel batch --batch 1024
   python -m paper_2607_22242_gb300.profile_case --kernel list --config 3 --count 16777216
   python -m paper_2607_22242_gb300.profile_case --kernel whatif --config 3 --reps 20
+  python -m paper_2607_22242_gb300.profile_case --kernel tree --workload wide32 --space 3
 
 Prints one line per repetition (CUDA-event time of the call and mappings/s).
 Sized so that a profiler capture of one launch stays short.
@@ -22,8 +23,12 @@ if ROOT not in sys.path:
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--kernel", choices=("search", "pruned", "eval", "batch", "list", "whatif"), default="search")
+    ap.add_argument("--kernel", choices=("search", "pruned", "eval", "batch", "list", "whatif", "tree"),
+                    default="search")
     ap.add_argument("--config", type=int, default=3)
+    ap.add_argument("--workload", default=None, help="wide28 | wide32 | layered24 (instead of --config)")
+    ap.add_argument("--space", type=int, default=3, help="tree search: 3 = full space, 2 = binary")
+    ap.add_argument("--no-prune", action="store_true", help="tree search: simulate every mapping")
     ap.add_argument("--first", type=int, default=0)
     ap.add_argument("--count", type=int, default=1 << 26)
     ap.add_argument("--batch", type=int, default=1024, help="scenarios for --kernel batch (config 4 prefix)")
@@ -43,11 +48,19 @@ def main():
         work = len(batch) * 3 ** 10
         call = lambda: bf.search_batch(batch, stream)
     else:
-        scn = S.config(args.config)
+        scn = getattr(S, args.workload)() if args.workload else S.config(args.config)
         count = min(args.count, 3 ** scn.n - args.first)
         work = count
         h = bf.create_scenario(scn)
-        if args.kernel == "search":
+        if args.kernel == "tree":  # branch and bound over the chosen space (count ignored)
+            work = args.space ** scn.n
+            stats = {}
+
+            def call():
+                res, st = bf.search_tree(h, args.space, not args.no_prune, None, stream)
+                stats.update(st)
+                return res
+        elif args.kernel == "search":
             call = lambda: bf.search_range(h, args.first, count, stream)
         elif args.kernel == "pruned":  # branch and bound over the whole space (count ignored)
             work = 3 ** scn.n
@@ -74,7 +87,8 @@ def main():
         b.synchronize()
         t = a.elapsed_time(b)
         print(f"{args.kernel} rep {rep}: {t:.3f} ms, {work / (t / 1e3):.4g} mappings/s"
-              + (f", best {out.index}/{out.makespan_us}" if args.kernel in ("search", "pruned") else ""), flush=True)
+              + (f", best {out.index}/{out.makespan_us}" if args.kernel in ("search", "pruned", "tree") else "")
+              + (f", {stats}" if args.kernel == "tree" else ""), flush=True)
 
 
 if __name__ == "__main__":
