@@ -185,6 +185,37 @@ def run_reference(args):
 
 # --------------------------------------------------------------------------- GPU arm
 
+def tree_search_times(torch, bf, S, stream, reps: int = 3):
+    """bf_search_tree on the 28- and 32-tool workloads: CUDA-event time of the call to the exact optimum
+    (median of `reps` after one warm-up), each result checked against the oracle's stored optimum."""
+    with open(os.path.join(ROOT, "tests", "golden", "wide_results.json")) as fh:
+        golden = json.load(fh)["workloads"]
+    cases = (("wide32", bf.SPACE_FULL, True), ("wide28", bf.SPACE_FULL, True), ("wide32", bf.SPACE_BINARY, True),
+             ("wide28", bf.SPACE_BINARY, False))
+    out = {}
+    for name, space, prune in cases:
+        scn = getattr(S, name)()
+        want = tuple(golden[name]["ternary" if space == bf.SPACE_FULL else "binary"])
+        times, stats = [], {}
+        with bf.create_scenario(scn) as h:
+            for rep in range(reps + 1):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                r, stats = bf.search_tree(h, space, prune, None, stream)
+                b.record(stream)
+                b.synchronize()
+                assert (r.index, r.makespan_us) == want, (name, space, prune, r, want)
+                if rep:
+                    times.append(a.elapsed_time(b))
+        ms = statistics.median(times)
+        key = f"{name}_{'full' if space == bf.SPACE_FULL else 'binary'}{'' if prune else '_unpruned'}"
+        out[key] = {"ms": ms, "mappings_in_space": space ** scn.n, "leaves_simulated": stats["leaves"],
+                    "nodes": stats["nodes"], "leaves_per_s": stats["leaves"] / (ms / 1e3)}
+    out["note"] = ("bf_search_tree: exact optimum (lowest makespan, lowest index) by branch and bound; "
+                   "'unpruned' simulates every mapping of the space")
+    return out
+
+
 def run_gpu(args):
     import torch
     rank, world, local = dist_env()
@@ -261,6 +292,9 @@ def run_gpu(args):
         assert (rp.index, rp.makespan_us) == (res.index, res.makespan_us)
     h.close()
 
+    # ---- beyond 20 tools: the tree search (exact optimum; reported beside `value`) ----
+    tree = tree_search_times(torch, bf, S, stream)
+
     if rank != 0:
         torch.distributed.destroy_process_group()
         return 0
@@ -286,6 +320,7 @@ def run_gpu(args):
                "median": statistics.median(pruned_ms), "min": min(pruned_ms),
                "note": "bf_search_pruned: exact branch and bound, same optimum; not a full enumeration"},
            "result": {"index": res.index, "makespan_us": res.makespan_us, "modes": res.modes},
+           "tree_search": tree,
            "roofline": roofline,
            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 572, "d2h_bytes_per_step": 8,
                    "path": "bf_create_scenario(host desc) + bf_search_best + bf_destroy_scenario"},
