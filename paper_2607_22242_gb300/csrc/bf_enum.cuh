@@ -94,6 +94,14 @@ __device__ __forceinline__ void prefix_task(const TBF& tb, const SmemTables& sd,
       continue;
     }
     if ((uint64_t)w.T + plan.tail_q > plan.bound) continue;  // pruned at the inner checkpoint
+    if ((w.done | inner_mask) == 0xFFFFFFFFu) {
+      // Everything but the last tool has ended: it runs alone from w.T.
+      for (uint32_t i = i_lo; i <= i_hi; ++i) {
+        const uint32_t d = plan.alone[i];
+        sink((uint32_t)(base + stride_i * i), d == kInfeasible ? kInfeasible : w.T + d);
+      }
+      continue;
+    }
     save_lane(w, slotB, stride);
     for (uint32_t i = i_lo; i <= i_hi; ++i) {
       const Digits di = decode(i, plan.I);

@@ -129,6 +129,13 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
   pl->tail_p = (uint32_t)(tp < 0xFFFFFFFFull ? tp : 0xFFFFFFFFull);
   pl->tail_q = (uint32_t)(tq < 0xFFFFFFFFull ? tq : 0xFFFFFFFFull);
   pl->bound = 0xFFFFFFFFu;
+  {
+    const uint32_t last = n - 1;
+    const bool fits = t.vram[last] <= t.budget;
+    pl->alone[0] = t.cpu[last];
+    pl->alone[1] = fits ? t.wnow[last] / 1024u : 0xFFFFFFFFu;
+    pl->alone[2] = fits ? t.wq[last] / 1024u : 0xFFFFFFFFu;
+  }
   pl->pow3P = (uint32_t)pow3(P);
   pl->pow3M = (uint32_t)pow3(M);
   pl->pow3I = (uint32_t)pow3(I);

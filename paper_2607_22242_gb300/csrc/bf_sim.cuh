@@ -103,6 +103,12 @@ struct Plan {
   // from any tool >= P to the end; tail_q likewise from tools >= Q.
   uint32_t tail_p, tail_q;
   uint32_t bound;           // 0xFFFFFFFF: no pruning
+  // I = 1 only: the last tool's duration in each mode when it runs alone
+  // (c; g + x; l + g + x), or 0xFFFFFFFF for a GPU mode whose footprint
+  // exceeds M.  A lone tool runs at f[1] = 1024 and finds no VRAM in use, so
+  // the model's one remaining event ends it exactly this long after it is
+  // ready.
+  uint32_t alone[3];
 };
 
 // Tables read with a per-thread (dynamic) index, staged in shared memory:
