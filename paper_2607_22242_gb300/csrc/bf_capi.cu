@@ -522,6 +522,7 @@ int bf_search_tree(const bf_scenario* scn_const, uint32_t space, uint32_t flags,
   tc.combos = 1;
   for (uint32_t i = 0; i < tc.D; ++i) tc.combos *= R;
   tc.prune = prune ? 1u : 0u;
+  tc.W0 = bfk::host::window_start(tb, tc.leaf_level);
   {
     uint64_t down[bfk::kTreeSlots] = {0};
     for (int v = (int)n - 1; v >= 0; --v) {

@@ -68,7 +68,8 @@ inline uint32_t mid_tools(uint32_t n) {
 // ready: the common ancestors of the "sources" of that range (tools >= from
 // whose predecessors are all < from); the first tool of the range to become
 // ready is one of them.
-inline uint32_t done_when_first_ready(const uint32_t* anc, const bfk::Tables& t, uint32_t from) {
+template <typename TB>
+inline uint32_t done_when_first_ready(const uint32_t* anc, const TB& t, uint32_t from) {
   const uint32_t below = (from >= 32) ? ~0u : ((1u << from) - 1u);
   uint32_t done = below;
   for (uint32_t v = from; v < t.n; ++v)
@@ -154,6 +155,51 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
     w->vram[j] = t.vram[w0 + j];
   }
   for (uint32_t k = 0; k <= (uint32_t)bfk::kMaxTools; ++k) {
+    w->f[k] = t.f[k];
+    w->fshift[k] = t.fshift[k];
+    w->fmagic[k] = t.fmagic[k];
+  }
+}
+
+// Ancestor masks of every tool (anc[v] = all tools with a path to v).
+template <typename TB>
+inline void ancestors(const TB& t, uint32_t* anc) {
+  for (uint32_t v = 0; v < t.n; ++v) {
+    anc[v] = t.pred[v];
+    for (uint32_t u = 0; u < v; ++u)
+      if (t.pred[v] & (1u << u)) anc[v] |= anc[u];
+  }
+}
+
+// Lowest tool not certainly done when the first tool of [from, n) becomes ready.
+template <typename TB>
+inline uint32_t window_start(const TB& t, uint32_t from) {
+  uint32_t anc[32];
+  ancestors(t, anc);
+  const uint32_t d = done_when_first_ready(anc, t, from);
+  uint32_t w0 = 0;
+  while (w0 < from && (d & (1u << w0))) ++w0;
+  return w0;
+}
+
+// Tables of tools [w0, n) renumbered from 0, in a table of capacity NW >= n - w0.
+template <int NW, int CAP>
+inline void build_window(const bfk::TablesT<CAP>& t, uint32_t w0, bfk::TablesT<NW>* w) {
+  std::memset(w, 0, sizeof *w);
+  const uint32_t nw = t.n - w0;
+  w->n = nw;
+  w->budget = t.budget;
+  w->all_mask = nw >= 32 ? ~0u : ((1u << nw) - 1u);
+  w->big_mask = t.big_mask >> w0;
+  for (uint32_t j = 0; j < nw; ++j) {
+    w->pred[j] = t.pred[w0 + j] >> w0;
+    w->succ[j] = t.succ[w0 + j] >> w0;
+    w->cpu[j] = t.cpu[w0 + j];
+    w->wnow[j] = t.wnow[w0 + j];
+    w->wq[j] = t.wq[w0 + j];
+    w->vram[j] = t.vram[w0 + j];
+  }
+  for (uint32_t k = 0; k <= (uint32_t)NW; ++k) {
     w->f[k] = t.f[k];
     w->fshift[k] = t.fshift[k];
     w->fmagic[k] = t.fmagic[k];

@@ -8,11 +8,15 @@
 //                        (one atomicAdd per warp).
 //   tree_leaf_kernel   : one warp per 32 leaf-level nodes (one per lane) and a
 //                        chunk of the radix^D combinations of the last D tools,
-//                        walked in lockstep; per-block best (makespan, index)
-//                        merged into one 16-byte record by compare-and-swap.
+//                        walked in lockstep over the leaf window (tools from the
+//                        lowest one that can still be running at a leaf
+//                        checkpoint; compiled for 8..32 slots); per-block best
+//                        (makespan, index) merged into one 16-byte record by
+//                        compare-and-swap.
 //   wide_list_kernel   : makespan of each listed mapping, simulated whole.
 #include <cuda_runtime.h>
 
+#include "bf_plan.h"
 #include "bf_tree.h"
 
 namespace bfk {
@@ -21,8 +25,6 @@ namespace {
 constexpr int kTreeThreads = 256;
 constexpr int kTreeWarps = kTreeThreads / 32;
 constexpr int kNW = NodeWords<kTreeSlots>::value;
-constexpr int kLW = LaneWords<kTreeSlots>::value;
-constexpr size_t kLeafSmemBytes = sizeof(uint32_t) * kLW * kTreeThreads;
 
 __device__ __forceinline__ uint32_t read_bound(const uint32_t* bound) {
   return *reinterpret_cast<const volatile uint32_t*>(bound);
@@ -93,16 +95,19 @@ __device__ __forceinline__ LaneBest shfl_best(const LaneBest& b, int o) {
   return r;
 }
 
-__global__ void __launch_bounds__(kTreeThreads, 2) tree_leaf_kernel(
-    const __grid_constant__ TablesW tb, const __grid_constant__ TreeConsts tc, const uint32_t* __restrict__ src,
-    uint32_t src_cap, uint32_t lo, uint32_t cnt, uint32_t parts, uint32_t chunk, uint32_t* bound, BestRecord* best,
-    TreeCounters* ctr) {
+// Leaf kernel over a window of NW slots (tools [W0, W0 + NW)); 4, 3 or 2
+// resident blocks per SM as the window widens (registers and shared memory).
+template <int NW>
+__global__ void __launch_bounds__(kTreeThreads, NW <= 12 ? 4 : NW <= 16 ? 3 : 2) tree_leaf_kernel(
+    const __grid_constant__ TablesW tb, const __grid_constant__ TablesT<NW> tw, const __grid_constant__ TreeConsts tc,
+    const uint32_t* __restrict__ src, uint32_t src_cap, uint32_t lo, uint32_t cnt, uint32_t parts, uint32_t chunk,
+    uint32_t* bound, BestRecord* best, TreeCounters* ctr) {
   extern __shared__ uint32_t lane_state[];
-  __shared__ SmemTablesW sd;
-  __shared__ uint32_t rt[ReadyTable<kTreeSlots>::size];
+  __shared__ SmemTablesT<NW> sdw;
+  __shared__ uint32_t rtw[ReadyTable<NW>::size];
   __shared__ uint32_t wb_ms[kTreeWarps], wb_now[kTreeWarps], wb_que[kTreeWarps];
-  load_smem_tables(tb, sd);
-  fill_ready_table<kTreeSlots>(tb, rt);
+  load_smem_tables(tw, sdw);
+  fill_ready_table<NW>(tw, rtw);
   __syncthreads();
   const uint32_t lane = threadIdx.x & 31u, warp = threadIdx.x >> 5;
   const uint32_t task = blockIdx.x * kTreeWarps + warp;
@@ -115,13 +120,14 @@ __global__ void __launch_bounds__(kTreeThreads, 2) tree_leaf_kernel(
     Digits dg{0u, 0u};
     uint32_t* slot = lane_state + threadIdx.x;
     if (valid) {
-      State<kTreeSlots> s;
-      load_node(src, src_cap, lo + j, s, dg);
+      const uint32_t* t = src + lo + j + (size_t)(2 * kTreeSlots) * src_cap;
+      dg = Digits{t[9 * (size_t)src_cap], t[10 * (size_t)src_cap]};
       // the incumbent may have improved since this node was bounded
-      if (tc.prune && lower_bound<kTreeSlots>(s, tb, tc, dg, tb.all_mask >> tc.D) > (uint64_t)read_bound(bound))
+      if (tc.prune &&
+          node_lower_bound(src, src_cap, lo + j, tb, tc, dg, tb.all_mask >> tc.D) > (uint64_t)read_bound(bound))
         valid = false;
       else
-        save_lane(s, slot, kTreeThreads);
+        node_to_window<NW>(src, src_cap, lo + j, tc.W0, tw.n, slot, kTreeThreads);
     }
     const uint32_t ran = __ballot_sync(0xFFFFFFFFu, valid);
     const uint32_t c0 = part * chunk;
@@ -130,7 +136,7 @@ __global__ void __launch_bounds__(kTreeThreads, 2) tree_leaf_kernel(
       if (part == 0) atomicAdd(&ctr->leaf_nodes, (unsigned long long)__popc(ran));
       atomicAdd(&ctr->leaves, (unsigned long long)__popc(ran) * (c1 - c0));
     }
-    if (ran) leaf_combos<kTreeSlots>(tb, sd, rt, tc, slot, kTreeThreads, dg, valid, c0, c1, lb);
+    if (ran) leaf_combos<NW>(tw, sdw, rtw, tc, slot, kTreeThreads, dg, valid, c0, c1, lb);
   }
   // warp, then block minimum; one record update per block
 #pragma unroll
@@ -214,16 +220,31 @@ cudaError_t launch_tree_expand(const TablesW& tb, const TreeConsts& tc, const ui
   return cudaGetLastError();
 }
 
-cudaError_t launch_tree_leaf(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
-                             uint32_t lo, uint32_t cnt, uint32_t target_tasks, uint32_t* bound, BestRecord* best,
-                             TreeCounters* ctr, cudaStream_t st) {
+// Window buckets of the leaf kernel.
+#define BF_TREE_BUCKETS(X) X(8) X(12) X(16) X(20) X(24) X(32)
+
+template <int NW>
+static cudaError_t leaf_launch(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
+                               uint32_t lo, uint32_t cnt, uint32_t parts, uint32_t chunk, unsigned grid,
+                               uint32_t* bound, BestRecord* best, TreeCounters* ctr, cudaStream_t st) {
   static bool ready = false;
+  const size_t smem = sizeof(uint32_t) * LaneWords<NW>::value * kTreeThreads;
   if (!ready) {
     const cudaError_t e =
-        cudaFuncSetAttribute(tree_leaf_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kLeafSmemBytes);
+        cudaFuncSetAttribute(tree_leaf_kernel<NW>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
     if (e != cudaSuccess) return e;
     ready = true;
   }
+  TablesT<NW> tw;
+  host::build_window(tb, tc.W0, &tw);
+  tree_leaf_kernel<NW><<<grid, kTreeThreads, smem, st>>>(tb, tw, tc, src, src_cap, lo, cnt, parts, chunk, bound, best,
+                                                         ctr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_tree_leaf(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
+                             uint32_t lo, uint32_t cnt, uint32_t target_tasks, uint32_t* bound, BestRecord* best,
+                             TreeCounters* ctr, cudaStream_t st) {
   // Split each group's combinations into parts so that about target_tasks
   // warp tasks exist, each covering at least 16 combinations.
   const uint32_t groups = (cnt + 31u) / 32u;
@@ -235,9 +256,13 @@ cudaError_t launch_tree_leaf(const TablesW& tb, const TreeConsts& tc, const uint
   parts = (tc.combos + chunk - 1u) / chunk;
   const uint64_t tasks = (uint64_t)groups * parts;
   const unsigned grid = (unsigned)((tasks + kTreeWarps - 1) / kTreeWarps);
-  tree_leaf_kernel<<<grid, kTreeThreads, kLeafSmemBytes, st>>>(tb, tc, src, src_cap, lo, cnt, parts, chunk, bound,
-                                                               best, ctr);
-  return cudaGetLastError();
+  const uint32_t nw = tb.n - tc.W0;
+#define BF_TRY(NW)                                                                                           \
+  if (nw <= (uint32_t)NW)                                                                                    \
+    return leaf_launch<NW>(tb, tc, src, src_cap, lo, cnt, parts, chunk, grid, bound, best, ctr, st);
+  BF_TREE_BUCKETS(BF_TRY)
+#undef BF_TRY
+  return cudaErrorInvalidValue;
 }
 
 cudaError_t launch_wide_list(const TablesW& tb, uint64_t total, const uint64_t* idx, uint64_t count, uint32_t* ms,

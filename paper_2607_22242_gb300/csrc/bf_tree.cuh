@@ -35,6 +35,7 @@ struct TreeConsts {
   uint32_t D;            // n - L tools enumerated per leaf node
   uint32_t combos;       // radix^D
   uint32_t prune;        // 0: keep every node (full enumeration)
+  uint32_t W0;           // leaf window start: tools below it have ended at every leaf checkpoint
   uint32_t dmin[kTreeSlots];   // min(c, g + x): no mode runs tool v faster
   uint32_t sdown[kTreeSlots];  // longest path in dmin through v's successors (0 for a sink)
   uint64_t pow3[kTreeSlots];
@@ -105,20 +106,23 @@ __device__ __forceinline__ void load_node(const uint32_t* buf, uint32_t cap, uin
 //     them in minimum durations (sdown);
 //   * queued tools run one at a time, so all unfinished tools known to be
 //     queued end no earlier than T + the sum of their remaining durations.
-template <int NT, typename TB>
-__device__ __forceinline__ uint64_t lower_bound(const State<NT>& s, const TB& tb, const TreeConsts& tc, Digits dg,
-                                                uint32_t known) {
-  const uint64_t T = s.T;
+template <int NT, typename TB, typename Slots>
+__device__ __forceinline__ uint64_t lower_bound_of(uint32_t done, uint32_t run_g, uint32_t T32, uint32_t V,
+                                                   const Slots& slot, const TB& tb, const TreeConsts& tc, Digits dg,
+                                                   uint32_t known) {
+  const uint64_t T = T32;
   uint64_t lb = T, qsum = 0u;
 #pragma unroll
   for (int v = 0; v < NT; ++v) {
     const uint32_t bit = 1u << v;
-    if (s.done & bit) continue;
+    if (done & bit) continue;
+    const uint32_t ec = slot.ec(v);
     uint64_t fin;
-    if (s.ec[v] != 0xFFFFFFFFu) {
-      fin = s.ec[v];
-    } else if (s.run_g & bit) {
-      const uint32_t left = ((s.eg[v] - s.V) >> 10) + (((s.eg[v] - s.V) & 1023u) != 0u);
+    if (ec != 0xFFFFFFFFu) {
+      fin = ec;
+    } else if (run_g & bit) {
+      const uint32_t r = slot.eg(v) - V;
+      const uint32_t left = (r >> 10) + ((r & 1023u) != 0u);
       fin = T + left;
       if (dg.que & bit) qsum += left;
     } else {
@@ -132,6 +136,66 @@ __device__ __forceinline__ uint64_t lower_bound(const State<NT>& s, const TB& tb
     lb = max(lb, fin + tc.sdown[v]);
   }
   return max(lb, T + qsum);
+}
+
+// Per-slot end times of a state held in registers, or of a node saved in HBM.
+template <int NT>
+struct StateSlots {
+  const State<NT>& s;
+  __device__ __forceinline__ uint32_t ec(int v) const { return s.ec[v]; }
+  __device__ __forceinline__ uint32_t eg(int v) const { return s.eg[v]; }
+};
+
+struct NodeSlots {
+  const uint32_t* p;  // word 0 of the node
+  uint32_t cap;
+  __device__ __forceinline__ uint32_t ec(int v) const { return p[(size_t)(2 * v) * cap]; }
+  __device__ __forceinline__ uint32_t eg(int v) const { return p[(size_t)(2 * v + 1) * cap]; }
+};
+
+template <int NT, typename TB>
+__device__ __forceinline__ uint64_t lower_bound(const State<NT>& s, const TB& tb, const TreeConsts& tc, Digits dg,
+                                                uint32_t known) {
+  return lower_bound_of<NT>(s.done, s.run_g, s.T, s.V, StateSlots<NT>{s}, tb, tc, dg, known);
+}
+
+// The bound of node j of a level buffer, read word by word from HBM.
+template <typename TB>
+__device__ __forceinline__ uint64_t node_lower_bound(const uint32_t* buf, uint32_t cap, uint32_t j, const TB& tb,
+                                                     const TreeConsts& tc, Digits dg, uint32_t known) {
+  const uint32_t* p = buf + j;
+  const uint32_t* t = p + (size_t)(2 * kTreeSlots) * cap;
+  return lower_bound_of<kTreeSlots>(t[0], t[2 * (size_t)cap], t[4 * (size_t)cap], t[5 * (size_t)cap],
+                                    NodeSlots{p, cap}, tb, tc, dg, known);
+}
+
+// Copy node j of a level buffer into a lane's shared-memory state over the
+// window [W0, W0 + NW) (slots past the last tool: no CPU end, stamp 0), with
+// masks shifted to window numbering.  Every tool below W0 has ended at every
+// leaf node's checkpoint, and no running tool lies outside the window.
+template <int NW>
+__device__ __forceinline__ void node_to_window(const uint32_t* buf, uint32_t cap, uint32_t j, uint32_t W0,
+                                               uint32_t nw, uint32_t* slot, uint32_t stride) {
+  const uint32_t* p = buf + j;
+#pragma unroll
+  for (int i = 0; i < NW; ++i) {
+    const uint32_t v = W0 + (uint32_t)i;
+    const bool in = v < (uint32_t)kTreeSlots;
+    slot[(2 * i) * stride] = in ? p[(size_t)(2 * v) * cap] : 0xFFFFFFFFu;
+    slot[(2 * i + 1) * stride] = in ? p[(size_t)(2 * v + 1) * cap] : 0u;
+  }
+  const uint32_t* t = p + (size_t)(2 * kTreeSlots) * cap;
+  const uint32_t wmask = nw >= 32u ? 0xFFFFFFFFu : ((1u << nw) - 1u);
+  uint32_t* q = slot + (2 * NW) * stride;
+  q[0 * stride] = (t[0 * (size_t)cap] >> W0) | ~wmask;  // done
+  q[1 * stride] = (t[1 * (size_t)cap] >> W0) & wmask;   // pend
+  q[2 * stride] = t[2 * (size_t)cap] >> W0;             // run_g
+  q[3 * stride] = t[3 * (size_t)cap] >> W0;             // qwait
+  q[4 * stride] = t[4 * (size_t)cap];                   // T
+  q[5 * stride] = t[5 * (size_t)cap];                   // V
+  q[6 * stride] = t[6 * (size_t)cap];                   // L
+  q[7 * stride] = t[7 * (size_t)cap];                   // tc
+  q[8 * stride] = t[8 * (size_t)cap];                   // gmin
 }
 
 // Child (tool d in mode a) of the node whose state and digits are in s / dg,
@@ -190,22 +254,24 @@ struct LaneBest {
 };
 
 // Simulate combinations [c0, c1) of the leaf node saved in `slot` (a lane's
-// shared-memory state, stride `stride`) whose digits are `dg`; `valid` false
-// runs the loop without work (lanes of a warp stay in lockstep).
-template <int NT, typename TB, typename SD>
-__device__ __forceinline__ void leaf_combos(const TB& tb, const SD& sd, const uint32_t* rt, const TreeConsts& tc,
+// shared-memory window state, stride `stride`) whose digits are `dg` (all
+// tools); tw/sdw/rtw are the window's tables.  `valid` false runs the loop
+// without work (lanes of a warp stay in lockstep).
+template <int NW, typename TBW, typename SD>
+__device__ __forceinline__ void leaf_combos(const TBW& tw, const SD& sdw, const uint32_t* rtw, const TreeConsts& tc,
                                             const uint32_t* slot, uint32_t stride, Digits dg, bool valid,
                                             uint32_t c0, uint32_t c1, LaneBest& best) {
-  const uint32_t L = tc.leaf_level;
+  const uint32_t L = tc.leaf_level, W0 = tc.W0;
+  const Digits dgw{dg.now >> W0, dg.que >> W0};
   for (uint32_t c = c0; c < c1; ++c) {
     if (!valid) continue;
-    const Digits dc = leaf_digits(c, tc.radix, tc.D, L);
-    const Digits full{dg.now | dc.now, dg.que | dc.que};
-    if (full.que & tb.big_mask) continue;
-    State<NT> w;
+    const Digits dc = leaf_digits(c, tc.radix, tc.D, L - W0);
+    const Digits sim{dgw.now | dc.now, dgw.que | dc.que};
+    if (sim.que & tw.big_mask) continue;
+    State<NW> w;
     load_lane(slot, stride, w);
-    if (run<NT>(w, tb, sd, rt, full, 0u) != kRunFinished) continue;
-    best.offer(w.T, full);
+    if (run<NW>(w, tw, sdw, rtw, sim, 0u) != kRunFinished) continue;
+    best.offer(w.T, Digits{dg.now | (dc.now << W0), dg.que | (dc.que << W0)});
   }
 }
 
