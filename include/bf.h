@@ -47,7 +47,9 @@
  *     current device.  `cuda_stream` is a cudaStream_t (NULL = legacy default
  *     stream); work is ordered on it.
  *   - A handle's scratch (search key, what-if list) is shared by the calls that
- *     use it: calls on one handle must not overlap in time.
+ *     use it: calls on one handle must not overlap in time.  A handle belongs
+ *     to the device that was current when it was created; calls on it with
+ *     another device current return BF_EINVAL.
  *   - Blocking calls wait with a time limit (bf_set_wait_timeout_ms) and
  *     return BF_ETIMEOUT if it passes; the GPU work is then still in flight,
  *     and the scenario must not be destroyed until the stream has finished.

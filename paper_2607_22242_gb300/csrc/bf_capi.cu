@@ -156,6 +156,18 @@ int wait_stream(cudaStream_t st, const char* who) {
   }
 }
 
+// A handle's scratch lives on the device that was current at creation; its
+// calls must run there.
+int check_device(const bf_scenario* scn, const char* who) {
+  int dev = -1;
+  const cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  if (dev != scn->device)
+    return fail(BF_EINVAL, "%s: the scenario was created on device %d but device %d is current", who, scn->device,
+                dev);
+  return BF_OK;
+}
+
 // The entry points that enumerate index ranges hold indices in 32 bits.
 int require_enum(const bf_scenario_desc& d, const char* who) {
   if (d.n > BF_MAX_TOOLS_ENUM)
@@ -278,6 +290,7 @@ int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count, uin
                      uint8_t* d_feasible, void* cuda_stream) {
   if (!scn) return fail(BF_EINVAL, "bf_eval_mappings: scenario is NULL");
   if (require_enum(scn->desc, "bf_eval_mappings") != BF_OK) return BF_EINVAL;
+  if (const int rc = check_device(scn, "bf_eval_mappings")) return rc;
   const uint64_t total = pow3(scn->desc.n);
   if (first > total || count > total - first)
     return fail(BF_ERANGE, "bf_eval_mappings: [%llu, %llu+%llu) is outside [0, 3^%u)",
@@ -297,6 +310,7 @@ int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count, uin
 int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_stream) {
   if (!scn || !out) return fail(BF_EINVAL, "bf_search_best: NULL argument");
   if (require_enum(scn->desc, "bf_search_best") != BF_OK) return BF_EINVAL;
+  if (const int rc = check_device(scn, "bf_search_best")) return rc;
   return run_search(scn, 0, pow3(scn->desc.n), out, static_cast<cudaStream_t>(cuda_stream), "bf_search_best");
 }
 
@@ -304,6 +318,7 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count, bf_r
                     void* cuda_stream) {
   if (!scn || !out) return fail(BF_EINVAL, "bf_search_range: NULL argument");
   if (require_enum(scn->desc, "bf_search_range") != BF_OK) return BF_EINVAL;
+  if (const int rc = check_device(scn, "bf_search_range")) return rc;
   const uint64_t total = pow3(scn->desc.n);
   if (first > total || count > total - first)
     return fail(BF_ERANGE, "bf_search_range: [%llu, %llu+%llu) is outside [0, 3^%u)",
@@ -316,6 +331,7 @@ int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t 
   if (!scn) return fail(BF_EINVAL, "bf_eval_indices: scenario is NULL");
   if (count == 0) return BF_OK;
   if (!d_indices || !d_makespan || !d_feasible) return fail(BF_EINVAL, "bf_eval_indices: NULL buffer");
+  if (const int rc = check_device(scn, "bf_eval_indices")) return rc;
   int sms = 0;
   cudaError_t e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, scn->device);
   if (e != cudaSuccess) return cuda_fail(e, "bf_eval_indices");
@@ -330,6 +346,7 @@ int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32
               void* cuda_stream) {
   const char* who = "bf_whatif";
   if (!scn || !out || !count) return fail(BF_EINVAL, "%s: NULL argument", who);
+  if (const int rc = check_device(scn, who)) return rc;
   const uint32_t n = scn->desc.n;
   const uint64_t total = pow3(n);
   if (base_index >= total)
@@ -415,6 +432,7 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   const char* who = "bf_search_pruned";
   if (!scn_const || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
   if (require_enum(scn_const->desc, who) != BF_OK) return BF_EINVAL;
+  if (const int rc = check_device(scn_const, who)) return rc;
   // The handle's lazily allocated survivor buffer is scratch, not state.
   bf_scenario* scn = const_cast<bf_scenario*>(scn_const);
   const uint32_t n = scn->desc.n;
@@ -505,6 +523,7 @@ int bf_search_tree(const bf_scenario* scn_const, uint32_t space, uint32_t flags,
   if (space != BF_SPACE_BINARY && space != BF_SPACE_FULL)
     return fail(BF_EINVAL, "%s: space %u is neither BF_SPACE_BINARY (2) nor BF_SPACE_FULL (3)", who, space);
   if (flags & ~(uint32_t)BF_TREE_NO_PRUNE) return fail(BF_EINVAL, "%s: unknown flags 0x%x", who, flags);
+  if (const int rc = check_device(scn_const, who)) return rc;
   // The handle's lazily allocated level buffers are scratch, not state.
   bf_scenario* scn = const_cast<bf_scenario*>(scn_const);
   const bfk::TablesW& tb = scn->wide;

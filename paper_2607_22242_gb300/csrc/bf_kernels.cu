@@ -226,15 +226,6 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) pruned_search_kernel(
   block_min_to(sink.best, key);
 }
 
-// Allow the kernel more than the default 48 KB of dynamic shared memory (once per kernel).
-template <typename K>
-static cudaError_t allow_dyn_smem(K kernel, bool* done) {
-  if (*done) return cudaSuccess;
-  const cudaError_t e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kDynSmemBytes);
-  if (e == cudaSuccess) *done = true;
-  return e;
-}
-
 }  // namespace
 
 #define BF_PASTE2(a, b) a##b
@@ -248,9 +239,9 @@ static unsigned blocks_for(const Plan& plan) {
 // Each launcher picks the prefix width (BF_NW when the scenario fits, else 20).
 #define BF_LAUNCH(KERNEL, FITS, INNER, GRID, ...)                                            \
   do {                                                                                       \
-    static bool ready_narrow = false, ready_wide = false;                                    \
-    cudaError_t e_ = (FITS) ? allow_dyn_smem(KERNEL<BF_NW>, &ready_narrow)                  \
-                            : allow_dyn_smem(KERNEL<kMaxTools>, &ready_wide);                \
+    static std::atomic<uint64_t> ready_narrow{0}, ready_wide{0};                           \
+    cudaError_t e_ = (FITS) ? allow_dyn_smem(KERNEL<BF_NW>, kDynSmemBytes, &ready_narrow)   \
+                            : allow_dyn_smem(KERNEL<kMaxTools>, kDynSmemBytes, &ready_wide); \
     if (e_ != cudaSuccess) return e_;                                                        \
     const size_t smem_ = dyn_smem_bytes(INNER);                                              \
     if (FITS)                                                                                \

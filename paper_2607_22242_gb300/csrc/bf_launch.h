@@ -5,11 +5,28 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <atomic>
+
 #include "bf_sim.cuh"
 
 namespace bfk {
 
 constexpr int kThreads = 256;  // threads per block of every kernel (8 warps, one prefix each)
+
+// Raise a kernel's dynamic shared memory limit to `bytes` on the current
+// device, once per device: the attribute belongs to the kernel's instance on
+// each device.  `done` is that kernel's set of devices already prepared.
+template <typename K>
+inline cudaError_t allow_dyn_smem(K kernel, size_t bytes, std::atomic<uint64_t>* done) {
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  const uint64_t bit = (dev >= 0 && dev < 64) ? (1ull << dev) : 0ull;
+  if (bit && (done->load(std::memory_order_acquire) & bit)) return cudaSuccess;
+  e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (e == cudaSuccess && bit) done->fetch_or(bit, std::memory_order_acq_rel);
+  return e;
+}
 
 // One scenario of a batched search: its tables, its window tables and plan.
 struct BatchRecord {

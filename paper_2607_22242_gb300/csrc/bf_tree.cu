@@ -16,6 +16,7 @@
 //   wide_list_kernel   : makespan of each listed mapping, simulated whole.
 #include <cuda_runtime.h>
 
+#include "bf_launch.h"
 #include "bf_plan.h"
 #include "bf_tree.h"
 
@@ -227,14 +228,10 @@ template <int NW>
 static cudaError_t leaf_launch(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
                                uint32_t lo, uint32_t cnt, uint32_t parts, uint32_t chunk, unsigned grid,
                                uint32_t* bound, BestRecord* best, TreeCounters* ctr, cudaStream_t st) {
-  static bool ready = false;
+  static std::atomic<uint64_t> ready{0};
   const size_t smem = sizeof(uint32_t) * LaneWords<NW>::value * kTreeThreads;
-  if (!ready) {
-    const cudaError_t e =
-        cudaFuncSetAttribute(tree_leaf_kernel<NW>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
-    if (e != cudaSuccess) return e;
-    ready = true;
-  }
+  const cudaError_t e = allow_dyn_smem(tree_leaf_kernel<NW>, smem, &ready);
+  if (e != cudaSuccess) return e;
   TablesT<NW> tw;
   host::build_window(tb, tc.W0, &tw);
   tree_leaf_kernel<NW><<<grid, kTreeThreads, smem, st>>>(tb, tw, tc, src, src_cap, lo, cnt, parts, chunk, bound, best,
