@@ -49,8 +49,8 @@ PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "search_kernel_config3_n19.md")
 
 def profiled_fields():
     """Fields of the committed ncu summary of the search kernel (DRAM bytes per launch, executed
-    thread instructions per mapping, issue-slot utilisation), or {} when the kernel sources changed
-    since that capture."""
+    thread instructions per mapping, issue-slot utilisation), or {} when the search kernel's
+    translation unit changed since that capture."""
     from paper_2607_22242_gb300 import _build
     try:
         text = open(PROFILE_SUMMARY).read()
@@ -58,7 +58,7 @@ def profiled_fields():
         return {}
     keys = ("source_fingerprint", "dram_bytes_per_launch", "thread_instructions_per_mapping", "issue_active")
     fields = dict(line.split(": ", 1) for line in text.splitlines() if line.startswith(tuple(k + ": " for k in keys)))
-    if fields.get("source_fingerprint", "").strip() != _build._fingerprint(()):
+    if fields.get("source_fingerprint", "").strip() != _build.kernel_fingerprint():
         return {}
     return fields
 
@@ -224,6 +224,71 @@ def tree_search_times(torch, bf, S, stream, reps: int = 3):
     return out
 
 
+def per_config_times(torch, bf, S, stream, reps: int = 5):
+    """Exhaustive search of each standard workload (the 4096-scenario batch as one call): median CUDA-event
+    time of the call and mappings/s, each optimum checked against the oracle's stored results."""
+    with open(os.path.join(ROOT, "tests", "golden", "config_results.json")) as fh:
+        golden = json.load(fh)["configs"]
+    out = {}
+    for cfg in range(4):
+        scn = S.config(cfg)
+        summ = golden[str(cfg)]["summary"]
+        times = []
+        with bf.create_scenario(scn) as h:
+            for rep in range(reps + 1):
+                a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+                a.record(stream)
+                r = bf.search_best(h, stream)
+                b.record(stream)
+                b.synchronize()
+                assert (r.index, r.makespan_us) == (summ["best_index"], summ["best_makespan"]), (cfg, r)
+                if rep:
+                    times.append(a.elapsed_time(b))
+        ms = statistics.median(times)
+        out[f"config{cfg}"] = {"ms": ms, "mappings": 3 ** scn.n, "mappings_per_s": 3 ** scn.n / (ms / 1e3)}
+    import ctypes
+    batch = S.config4()
+    packed = bf.pack_descs(batch)  # the C caller's array of bf_scenario_desc
+    descs = packed.ctypes.data_as(ctypes.POINTER(bf.Desc))
+    results = (bf.CResult * len(batch))()
+    want = list(zip(golden["4"]["best_index"], golden["4"]["best_makespan"]))
+    times = []
+    for rep in range(4):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        rc = bf.load().bf_search_batch(descs, len(batch), results, ctypes.c_void_p(stream.cuda_stream))
+        b.record(stream)
+        b.synchronize()
+        assert rc == bf.BF_OK, bf.last_error()
+        assert [(r.index, r.makespan_us) for r in results] == want
+        if rep:
+            times.append(a.elapsed_time(b))
+    ms = statistics.median(times)
+    total = len(batch) * 3 ** 10
+    out["config4_batch"] = {"ms": ms, "mappings": total, "mappings_per_s": total / (ms / 1e3),
+                            "note": "one bf_search_batch C call on an array of 4096 descs: per-scenario "
+                                    "tables and plans on the host, allocation, copies and the kernel"}
+    return out
+
+
+def oracle_single_core(S, seconds_per_config: float = 1.5):
+    """The oracle on one host thread: mappings/s per standard workload on a timed slice of its index space."""
+    import oracle
+    out = {}
+    for cfg in range(4):
+        scn = S.config(cfg)
+        total = 3 ** scn.n
+        count = min(total, 1 << 14)
+        n_done, t0 = 0, time.perf_counter()
+        while time.perf_counter() - t0 < seconds_per_config and n_done < total:
+            first = (n_done * 7919) % max(1, total - count)
+            oracle.search_range(scn, first, count, 1)
+            n_done += count
+        dt = time.perf_counter() - t0
+        out[f"config{cfg}"] = n_done / dt
+    return out
+
+
 def run_gpu(args):
     import torch
     rank, world, local = dist_env()
@@ -300,7 +365,17 @@ def run_gpu(args):
         assert (rp.index, rp.makespan_us) == (res.index, res.makespan_us)
     h.close()
 
-    # ---- beyond 20 tools: the tree search (exact optimum; reported beside `value`) ----
+    # ---- host wall time of the blocking call, scenario already created ----------
+    h = bf.create_scenario(scn)
+    host_ms = []
+    for _ in range(10):
+        t0 = time.perf_counter()
+        bf.search_best(h, stream)
+        host_ms.append((time.perf_counter() - t0) * 1e3)
+    h.close()
+
+    # ---- every standard workload, and beyond 20 tools the tree search ---------------
+    per_config = per_config_times(torch, bf, S, stream)
     tree = tree_search_times(torch, bf, S, stream)
 
     if rank != 0:
@@ -331,7 +406,11 @@ def run_gpu(args):
            "config": {"workload": WORKLOAD, "mappings_per_step": total, "parallelism": f"replicas x{world}",
                       "l2": "flushed between steps (256 MiB write, outside the timed events)"},
            "wall_time_to_optimum_ms": {"median": statistics.median(step_ms), "min": min(step_ms),
-                                       "max": max(step_ms)},
+                                       "max": max(step_ms),
+                                       "host_median": statistics.median(host_ms),
+                                       "host_note": "bf_search_best call as seen by the host (blocks until the "
+                                                    "result is in pinned host memory), median of 10"},
+           "per_config": per_config,
            "pruned_wall_time_to_optimum_ms": {
                "median": statistics.median(pruned_ms), "min": min(pruned_ms),
                "note": "bf_search_pruned: exact branch and bound, same optimum; not a full enumeration"},
@@ -349,7 +428,8 @@ def run_gpu(args):
         n, dt = oracle_sample_time(scn, args.cpu_sample, threads)
         out["cpu_baseline"] = {"value": n / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
                                "sample": f"{n} mappings of the same workload in 16 contiguous chunks spread "
-                                         f"evenly over [0, 3^19), oracle search, {dt:.1f} s"}
+                                         f"evenly over [0, 3^19), oracle search, {dt:.1f} s",
+                               "single_core_per_config": oracle_single_core(S)}
     emit(out)
     if world > 1:
         torch.distributed.destroy_process_group()

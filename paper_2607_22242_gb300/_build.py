@@ -47,6 +47,22 @@ def _fingerprint(extra) -> str:
     return h.hexdigest()
 
 
+# Sources of the enumerating kernels' translation unit (bf_kernels.cu and what it includes).
+KERNEL_UNIT = ("bf_kernels.cu", "bf_enum.cuh", "bf_sim.cuh", "bf_launch.h")
+
+
+def kernel_fingerprint() -> str:
+    """Hash of the enumerating kernels' sources and flags: a profile taken of those kernels stays
+    valid while this is unchanged (changes elsewhere in the library do not touch them)."""
+    h = hashlib.sha256()
+    for name in KERNEL_UNIT:
+        with open(os.path.join(CSRC, name), "rb") as fh:
+            h.update(name.encode() + fh.read())
+    flags = [f for f in NVCC_FLAGS if not f.startswith("-I")]
+    h.update(" ".join(ARCH + flags).encode())
+    return h.hexdigest()
+
+
 def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
     """Compile and link libbf.so unless an up-to-date copy exists; return its path."""
     os.makedirs(BUILD_DIR, exist_ok=True)

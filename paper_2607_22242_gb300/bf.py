@@ -308,18 +308,20 @@ def search_range(h: Union[ScenarioHandle, Scenario], first: int, count: int, str
             handle.close()
 
 
-def _batch_call(fn, scns: Sequence[Scenario], stream) -> List[Result]:
+def _batch_call(fn, scns: Sequence[Scenario], stream, packed=None) -> List[Result]:
     count = len(scns)
-    packed = pack_descs(scns) if count else None
+    if packed is None and count:
+        packed = pack_descs(scns)
     descs = packed.ctypes.data_as(ctypes.POINTER(Desc)) if count else None
     results = (CResult * max(count, 1))()
     _check(fn(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
     return [_result(results[i], scns[i].n) for i in range(count)]
 
 
-def search_batch(scns: Sequence[Scenario], stream=None) -> List[Result]:
-    """Full search of each scenario, one launch for the whole batch."""
-    return _batch_call(load().bf_search_batch, scns, stream)
+def search_batch(scns: Sequence[Scenario], stream=None, packed=None) -> List[Result]:
+    """Full search of each scenario, one launch for the whole batch.  ``packed`` (from
+    :func:`pack_descs` of the same scenarios) skips the packing when a batch is searched repeatedly."""
+    return _batch_call(load().bf_search_batch, scns, stream, packed)
 
 
 def search_batch_noalloc(scns: Sequence[Scenario], stream=None) -> List[Result]:
