@@ -208,6 +208,16 @@ void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* 
     default: { e = bfk::CALL(20); } break;                \
   }
 
+// Plan of one scenario of a batch (one block of kThreads / 32 warps each): a
+// scenario with fewer prefix groups than warps splits its mid combinations
+// so that as many warps as possible share it.
+bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n) {
+  constexpr uint32_t kWarps = bfk::kThreads / 32;
+  const uint32_t groups = (base.pow3P + 31u) / 32u;
+  const uint32_t fill = groups < kWarps ? kWarps / groups : 1u;
+  return make_plan(base, 0, pow3(n), (uint64_t)fill * groups);
+}
+
 // Index-list evaluation: the 20-slot kernels up to 20 tools, the 32-slot one above.
 cudaError_t launch_list(const bf_scenario* scn, const uint64_t* idx, uint64_t count, uint32_t* ms, uint8_t* fe,
                         int grid, cudaStream_t st) {
@@ -704,7 +714,7 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
     build_tables(descs + i, &r.full);
     bfk::Plan base;
     split_and_window(r.full, &base, &r.window);
-    r.plan = make_plan(base, 0, pow3(descs[i].n), 1);
+    r.plan = batch_plan(base, descs[i].n);
     if (r.window.n > wmax) wmax = r.window.n;
     const uint32_t tasks = r.plan.groups * r.plan.m_parts;
     if (tasks > pmax) pmax = tasks;
@@ -829,7 +839,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
       build_tables(descs + i0 + j, &r.full);
       bfk::Plan plan;
       split_and_window(r.full, &plan, &r.window);
-      r.plan = make_plan(plan, 0, pow3(descs[i0 + j].n), 1);
+      r.plan = batch_plan(plan, descs[i0 + j].n);
       if (r.window.n > wmax) wmax = r.window.n;
       const uint32_t tasks = r.plan.groups * r.plan.m_parts;
       if (tasks > pmax) pmax = tasks;
