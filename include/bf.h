@@ -202,13 +202,15 @@ typedef struct bf_tree_stats {
  * A node is dropped when a lower bound on all of its mappings' makespans
  * exceeds the best makespan known (strictly, so the optimum and its ties
  * survive): running tools end no earlier than their remaining work at
- * isolated speed allows, a tool not started ends no earlier than its duration
- * in its mode (or min(c, g + x) if open) after the node's time, each tool's
- * successors add the longest path through them in minimum durations, and
- * queued tools run one at a time.  The first bound is the best of a few
- * mappings of the space (hint_index if it lies in it, all-cpu, all-gpu_now,
- * each tool on its isolated-faster device, all-gpu_queue); better ones are
- * found as the search proceeds.  space: BF_SPACE_FULL or BF_SPACE_BINARY.
+ * isolated speed allows, every other tool ends no earlier than the latest of
+ * the node's time and its predecessors' earliest ends plus its duration in
+ * its mode (or min(c, g + x) if open), and queued tools run one at a time.
+ * The first bound is the best of a few mappings of the space (hint_index if
+ * it lies in it, all-cpu, all-gpu_now, each tool on its isolated-faster
+ * device, all-gpu_queue); when the tree is large, a narrow dive to the leaves
+ * (8192 nodes per level) tightens it before the search restarts from the root;
+ * better bounds are found as the search proceeds.  space: BF_SPACE_FULL or
+ * BF_SPACE_BINARY.
  * flags: 0 or BF_TREE_NO_PRUNE (every mapping of the space is simulated:
  * full enumeration).  `stats` may be NULL.  Allocates level buffers in the
  * handle on first use (about 1.7 GB for 32 tools in the full space).  Blocks

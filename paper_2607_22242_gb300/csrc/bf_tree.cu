@@ -43,6 +43,7 @@ __global__ void __launch_bounds__(kTreeThreads, 2) tree_expand_kernel(
     uint32_t* dst_count, const uint32_t* bound, TreeCounters* ctr) {
   __shared__ SmemTablesW sd;
   __shared__ uint32_t rt[ReadyTable<kTreeSlots>::size];
+  __shared__ uint32_t ef[kTreeSlots * kTreeThreads];  // forward_bound scratch, [tool][thread]
   load_smem_tables(tb, sd);
   fill_ready_table<kTreeSlots>(tb, rt);
   __syncthreads();
@@ -55,7 +56,7 @@ __global__ void __launch_bounds__(kTreeThreads, 2) tree_expand_kernel(
   Digits dg{0u, 0u};
   if (a < tc.radix) {
     load_node(src, src_cap, lo + j, s, dg);
-    keep = expand_child<kTreeSlots>(tb, sd, rt, tc, s, dg, d, a, read_bound(bound));
+    keep = expand_child<kTreeSlots>(tb, sd, rt, tc, s, dg, d, a, read_bound(bound), ef + threadIdx.x, kTreeThreads);
   }
   const uint32_t ballot = __ballot_sync(0xFFFFFFFFu, keep);
   if (ballot == 0u) return;

@@ -198,13 +198,58 @@ __device__ __forceinline__ void node_to_window(const uint32_t* buf, uint32_t cap
   q[8 * stride] = t[8 * (size_t)cap];                   // gmin
 }
 
+// The stronger bound of the expansions: the earliest finish EF of every
+// unfinished tool, in index (topological) order -- a running CPU tool its end
+// time, a running GPU tool T + ceil(r / 1024), any other tool the latest of T
+// and its unfinished predecessors' EF, plus its duration in its mode (the
+// least over the modes if open) -- and the makespan is at least the largest
+// EF and the serial-queue sum of lower_bound().  Every start is no earlier
+// than T and than the ends of its predecessors, and no tool runs faster than
+// its isolated duration, so EF never exceeds the true end.  `ef` is a
+// per-thread column of NT words in shared memory (stride `stride`).  Times fit
+// in 32 bits: T plus the durations of a chain of remaining tools stays below
+// the validated makespan bound.
+template <int NT, typename TB>
+__device__ __forceinline__ uint32_t forward_bound(const State<NT>& s, const TB& tb, const TreeConsts& tc, Digits dg,
+                                                  uint32_t known, uint32_t* ef, uint32_t stride) {
+  const uint32_t T = s.T;
+  uint32_t lb = T, qsum = 0u;
+#pragma unroll
+  for (int v = 0; v < NT; ++v) {
+    const uint32_t bit = 1u << v;
+    if (s.done & bit) continue;
+    uint32_t fin;
+    if (s.ec[v] != 0xFFFFFFFFu) {
+      fin = s.ec[v];
+    } else if (s.run_g & bit) {
+      const uint32_t r = s.eg[v] - s.V;
+      const uint32_t left = (r >> 10) + ((r & 1023u) != 0u);
+      fin = T + left;
+      if (dg.que & bit) qsum += left;
+    } else {
+      uint32_t d = tc.dmin[v];
+      if (known & bit) {
+        d = (dg.now & bit) ? (tb.wnow[v] >> 10) : (dg.que & bit) ? (tb.wq[v] >> 10) : tb.cpu[v];
+        if (dg.que & bit) qsum += d;
+      }
+      uint32_t start = T;
+      for (uint32_t m = tb.pred[v] & ~s.done; m; m &= m - 1u) start = max(start, ef[(__ffs(m) - 1) * stride]);
+      fin = start + d;
+    }
+    ef[v * stride] = fin;
+    lb = max(lb, fin);
+  }
+  return max(lb, T + qsum);
+}
+
 // Child (tool d in mode a) of the node whose state and digits are in s / dg,
 // advanced in place to the child's checkpoint.  Returns false when every
 // mapping below the child is infeasible or, with pruning, provably worse
-// than `bound`.  Requires d + 1 < n.
+// than `bound` (forward_bound, scratch column `ef`).  Requires d + 1 < n.
 template <int NT, typename TB, typename SD>
 __device__ __forceinline__ bool expand_child(const TB& tb, const SD& sd, const uint32_t* rt, const TreeConsts& tc,
-                                             State<NT>& s, Digits& dg, uint32_t d, uint32_t a, uint32_t bound) {
+                                             State<NT>& s, Digits& dg, uint32_t d, uint32_t a, uint32_t bound,
+                                             uint32_t* ef, uint32_t stride) {
   const uint32_t bit = 1u << d;
   if (a == 1u) dg.now |= bit;
   if (a == 2u) {
@@ -213,7 +258,7 @@ __device__ __forceinline__ bool expand_child(const TB& tb, const SD& sd, const u
   }
   const uint32_t assigned = (bit << 1) - 1u;  // tools [0, d]; all ones for d = 31
   if (run<NT>(s, tb, sd, rt, dg, tb.all_mask & ~assigned) != kRunStopped) return false;
-  return !tc.prune || lower_bound<NT>(s, tb, tc, dg, assigned) <= (uint64_t)bound;
+  return !tc.prune || forward_bound<NT>(s, tb, tc, dg, assigned, ef, stride) <= bound;
 }
 
 // Digits of leaf combination c (tools [L, n)), as masks shifted to tool L.
