@@ -22,6 +22,7 @@ step time is the max over ranks.
 from __future__ import annotations
 
 import argparse
+import ctypes
 import json
 import os
 import statistics
@@ -417,8 +418,11 @@ def run_gpu(args):
            "result": {"index": res.index, "makespan_us": res.makespan_us, "modes": res.modes},
            "tree_search": tree,
            "roofline": roofline,
-           "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": 572, "d2h_bytes_per_step": 8,
-                   "path": "bf_create_scenario(host desc) + bf_search_best + bf_destroy_scenario"},
+           "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": ctypes.sizeof(bf.Desc),
+                   "d2h_bytes_per_step": 8,
+                   "path": "bf_create_scenario(host desc) + bf_search_best + bf_destroy_scenario",
+                   "bytes_note": "in: the step's input, one bf_scenario_desc (its derived tables reach the GPU "
+                                 "as kernel parameters); out: the 8-byte result key"},
            "gpu_launches": args.steps,  # one search kernel per timed step
            "clocks": clocks, "timed_wall_s": wall, "sm_count": sm_count}
     if world == 1 and not args.no_cpu_baseline:
