@@ -1,14 +1,18 @@
-"""Splitting one search over several ranks (one GPU each).
+"""Splitting one search, or one batch of searches, over several ranks (one GPU each).
 
 The mapping index space [0, 3^n) splits into contiguous ranges; each rank
 searches its own with ``bf_search_range`` and the ranks exchange one packed
 key each (makespan << 32 | index).  The smallest key is the answer of the
 whole search: ranges compose because the argmin is a minimum over (makespan,
 index) pairs.  The exchange is the only collective, 8 bytes per rank.
+
+A batch of independent scenarios splits into contiguous blocks of scenarios,
+one per rank (``bf_search_batch`` on each); one all-gather of the per-rank
+result lists returns every scenario's optimum to every rank.
 """
 from __future__ import annotations
 
-from typing import Callable, Optional, Tuple
+from typing import Callable, List, Optional, Sequence, Tuple
 
 INFEASIBLE = 0xFFFFFFFF
 NO_KEY = (1 << 64) - 1
@@ -78,4 +82,30 @@ def gpu_search_range(handle, stream=None) -> Callable[[int, int], Tuple[int, int
     def run(first: int, count: int) -> Tuple[int, int, bool]:
         r = bf.search_range(handle, first, count, stream)
         return r.index, r.makespan_us, r.feasible
+    return run
+
+
+def sharded_batch(search_batch: Callable[[Sequence], List[Tuple[int, int, bool]]], scenarios: Sequence,
+                  group=None) -> List[Tuple[int, int, bool]]:
+    """Search every scenario of `scenarios`, split over the ranks of `group`.
+
+    ``search_batch(block) -> [(index, makespan, feasible), ...]`` searches one
+    contiguous block of scenarios on this rank (``bf.search_batch`` on a GPU).
+    Returns the results of all scenarios, in order, on every rank.
+    """
+    import torch.distributed as dist
+    rank, world = dist.get_rank(group), dist.get_world_size(group)
+    first, count = shard_range(len(scenarios), rank, world)
+    mine = list(search_batch(scenarios[first:first + count])) if count else []
+    parts = [None] * world
+    dist.all_gather_object(parts, mine, group=group)
+    return [r for part in parts for r in part]
+
+
+def gpu_search_batch(stream=None) -> Callable[[Sequence], List[Tuple[int, int, bool]]]:
+    """A ``search_batch`` callable on this rank's GPU."""
+    from . import bf
+
+    def run(block: Sequence) -> List[Tuple[int, int, bool]]:
+        return [(r.index, r.makespan_us, r.feasible) for r in bf.search_batch(block, stream)]
     return run

@@ -299,6 +299,21 @@ def test_shards_combine_to_full_search(golden):
             assert shard.unpack_key(min(keys)) == (g["best_index"], g["best_makespan"], True)
 
 
+def test_batch_shards_combine_to_full_batch(golden):
+    """The per-rank blocks of a sharded batch (shard.gpu_search_batch on each rank's block of the
+    4096 scenarios), concatenated in rank order, give every scenario's optimum."""
+    from paper_2607_22242_gb300 import shard
+    batch = S.config4()
+    want = [(i, m, True) for i, m in zip(golden["4"]["best_index"], golden["4"]["best_makespan"])]
+    search = shard.gpu_search_batch()
+    for world in (2, 3, 8):
+        got = []
+        for r in range(world):
+            first, count = shard.shard_range(len(batch), r, world)
+            got += search(batch[first:first + count])
+        assert got == want, world
+
+
 # --------------------------------------------------------------------------- what-if and index lists
 
 def _same_probes(got, want):

@@ -79,3 +79,43 @@ def test_key_order_is_makespan_then_index():
     assert min(a, b, c) == b
     assert shard.unpack_key(min(a, b, c)) == (3, 100, True)
     assert shard.unpack_key(shard.pack_key(5, 0, False)) == (-1, shard.INFEASIBLE, False)
+
+
+def _batch_worker(rank, world, port, count, out):
+    import torch.distributed as dist
+    import oracle
+    from paper_2607_22242_gb300 import scenarios as S
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        scns = S.config4(count)
+
+        def search_batch(block):
+            idx, ms = oracle.search_batch(block)
+            return [(int(i), int(m), int(m) != shard.INFEASIBLE) for i, m in zip(idx, ms)]
+        out.put((rank, shard.sharded_batch(search_batch, scns)))
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("count,world", [(9, 2), (7, 3), (2, 3)])
+def test_sharded_batch_equals_single_process(count, world):
+    """Scenarios split into contiguous blocks per rank (one with none when count < world):
+    every rank gets every scenario's optimum, in order."""
+    import oracle
+    from paper_2607_22242_gb300 import scenarios as S
+    oracle.build()
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_batch_worker, args=(r, world, port, count, out)) for r in range(world)]
+    for p in procs:
+        p.start()
+    results = [out.get(timeout=120) for _ in range(world)]
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    idx, ms = oracle.search_batch(S.config4(count))
+    want = [(int(i), int(m), True) for i, m in zip(idx, ms)]
+    for rank, got in results:
+        assert got == want, rank
