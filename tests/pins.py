@@ -387,4 +387,22 @@ def check_segments(lib, trials=40, seed=23):
     assert segments.search(S.config3(), lib=lib) == (golden["summary"]["best_index"], golden["summary"]["best_makespan"])
 
 
-ALL_CHECKS += [check_wide_closed_forms, check_binary_space, check_segments]
+def check_degenerate_budgets(lib, trials=30, seed=24):
+    """M = 0: every GPU mode is infeasible (gpu_now overflows at start, a queued tool can never fit), so the
+    all-cpu mapping is the only feasible one and the optimum is the critical path of CPU times; and a
+    budget that fits everything at once with f[k] = 65536 for k >= 2: every mapping stays feasible."""
+    rng = np.random.default_rng(seed)
+    for _ in range(trials):
+        n = int(rng.integers(1, 7))
+        base = S.random_small(rng, n, max_time=300)
+        zero = Scenario(**{**base.to_dict(), "vram_budget_mib": 0})
+        ms, fe = lib.eval_range(zero, 0, 3 ** n)
+        assert fe[0] == 1 and not fe[1:].any(), zero
+        assert lib.search(zero) == (0, _longest_path(zero, zero.cpu_us))
+        steep = Scenario(**{**base.to_dict(), "vram_budget_mib": sum(base.vram_mib),
+                            "slowdown_q10": [0, 1024] + [65536] * (len(base.slowdown_q10) - 2)})
+        ms, fe = lib.eval_range(steep, 0, 3 ** n)
+        assert fe.all(), steep
+
+
+ALL_CHECKS += [check_wide_closed_forms, check_binary_space, check_segments, check_degenerate_budgets]

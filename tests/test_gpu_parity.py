@@ -106,6 +106,28 @@ def test_every_bucket_edge(n):
         assert (r.index, r.makespan_us) == oracle.search(scn, THREADS)
 
 
+def test_degenerate_budgets_all_paths():
+    """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
+    the batch, the branch and bound and the tree search, against the oracle."""
+    rng = np.random.default_rng(2222)
+    scns = []
+    for _ in range(12):
+        n = int(rng.integers(2, 9))
+        base = S.random_small(rng, n, max_time=300)
+        scns.append(S.Scenario(**{**base.to_dict(), "vram_budget_mib": 0}))
+        scns.append(S.Scenario(**{**base.to_dict(), "vram_budget_mib": sum(base.vram_mib),
+                                  "slowdown_q10": [0, 1024] + [65536] * (len(base.slowdown_q10) - 2)}))
+    batch = bf.search_batch(scns)
+    for scn, rb in zip(scns, batch):
+        want = oracle.search(scn)
+        with bf.create_scenario(scn) as h:
+            assert_same(h, scn, 0, 3 ** scn.n)
+            for r in (bf.search_best(h), bf.search_pruned(h), rb, bf.search_tree(h)[0]):
+                assert (r.index, r.makespan_us) == want, (scn, r, want)
+        if scn.vram_budget_mib == 0:
+            assert want[0] == 0
+
+
 # --------------------------------------------------------------------------- standard workloads
 
 @pytest.mark.parametrize("cfg", [0, 1, 2])
