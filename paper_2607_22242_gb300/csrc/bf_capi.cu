@@ -218,6 +218,49 @@ bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n) {
   return make_plan(base, 0, pow3(n), (uint64_t)fill * groups);
 }
 
+// Records (tables, window tables, plan) of descs[0, count), built on up to 16
+// host threads (about half a microsecond per scenario); the largest window,
+// task count and whether any plan has an inner level are returned too.
+void build_records(const bf_scenario_desc* descs, uint32_t count, bfk::BatchRecord* recs, uint32_t* wmax,
+                   uint32_t* pmax, uint32_t* any_inner) {
+  struct Part {
+    uint32_t wmax = 0, pmax = 0, inner = 0;
+  };
+  auto work = [&](uint32_t lo, uint32_t hi, Part* part) {
+    for (uint32_t i = lo; i < hi; ++i) {
+      bfk::BatchRecord& r = recs[i];
+      std::memset(&r, 0, sizeof r);
+      build_tables(descs + i, &r.full);
+      bfk::Plan base;
+      split_and_window(r.full, &base, &r.window);
+      r.plan = batch_plan(base, descs[i].n);
+      if (r.window.n > part->wmax) part->wmax = r.window.n;
+      const uint32_t tasks = r.plan.groups * r.plan.m_parts;
+      if (tasks > part->pmax) part->pmax = tasks;
+      part->inner |= r.plan.I;
+    }
+  };
+  const unsigned hw = std::thread::hardware_concurrency();
+  uint32_t nthreads = count / 256u;  // a thread is worth starting for a few hundred scenarios
+  if (nthreads > 16u) nthreads = 16u;
+  if (hw && nthreads > hw) nthreads = hw;
+  std::vector<Part> parts(nthreads > 1 ? nthreads : 1);
+  if (nthreads <= 1) {
+    work(0, count, &parts[0]);
+  } else {
+    std::vector<std::thread> pool;
+    for (uint32_t t = 0; t < nthreads; ++t)
+      pool.emplace_back(work, (uint32_t)((uint64_t)count * t / nthreads), (uint32_t)((uint64_t)count * (t + 1) / nthreads),
+                        &parts[t]);
+    for (auto& th : pool) th.join();
+  }
+  for (const Part& p : parts) {
+    *wmax = p.wmax > *wmax ? p.wmax : *wmax;
+    *pmax = p.pmax > *pmax ? p.pmax : *pmax;
+    *any_inner |= p.inner;
+  }
+}
+
 // Index-list evaluation: the 20-slot kernels up to 20 tools, the 32-slot one above.
 cudaError_t launch_list(const bf_scenario* scn, const uint64_t* idx, uint64_t count, uint32_t* ms, uint8_t* fe,
                         int grid, cudaStream_t st) {
@@ -729,18 +772,7 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
   }
   std::vector<bfk::BatchRecord> recs(count);
   uint32_t wmax = 0, pmax = 0, any_inner = 0;
-  for (uint32_t i = 0; i < count; ++i) {
-    bfk::BatchRecord& r = recs[i];
-    std::memset(&r, 0, sizeof r);
-    build_tables(descs + i, &r.full);
-    bfk::Plan base;
-    split_and_window(r.full, &base, &r.window);
-    r.plan = batch_plan(base, descs[i].n);
-    if (r.window.n > wmax) wmax = r.window.n;
-    const uint32_t tasks = r.plan.groups * r.plan.m_parts;
-    if (tasks > pmax) pmax = tasks;
-    any_inner |= r.plan.I;
-  }
+  build_records(descs, count, recs.data(), &wmax, &pmax, &any_inner);
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   bfk::BatchRecord* d_recs = nullptr;
   unsigned long long* d_keys = nullptr;
