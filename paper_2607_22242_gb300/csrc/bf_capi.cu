@@ -234,6 +234,7 @@ void build_records(const bf_scenario_desc* descs, uint32_t count, bfk::BatchReco
       bfk::Plan base;
       split_and_window(r.full, &base, &r.window);
       r.plan = batch_plan(base, descs[i].n);
+      r.mid_lanes = base.W0 == 0u ? 1u : 0u;
       if (r.window.n > part->wmax) part->wmax = r.window.n;
       const uint32_t tasks = r.plan.groups * r.plan.m_parts;
       if (tasks > part->pmax) part->pmax = tasks;
@@ -893,6 +894,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
       bfk::Plan plan;
       split_and_window(r.full, &plan, &r.window);
       r.plan = batch_plan(plan, descs[i0 + j].n);
+      r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
       if (r.window.n > wmax) wmax = r.window.n;
       const uint32_t tasks = r.plan.groups * r.plan.m_parts;
       if (tasks > pmax) pmax = tasks;

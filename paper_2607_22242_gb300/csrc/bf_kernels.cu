@@ -141,12 +141,17 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
   fill_ready_table<NP>(rec.full, rt);
   fill_ready_table<BF_NW>(rec.window, rtw);
   __syncthreads();
-  const uint32_t task = b * kWarps + (threadIdx.x >> 5);
+  const uint32_t warp = b * kWarps + (threadIdx.x >> 5);
   MinKeySink sink;
-  if (task < rec.plan.groups * rec.plan.m_parts)
-    warp_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, task / rec.plan.m_parts,
-                         task % rec.plan.m_parts, lane_state + threadIdx.x,
+  if (rec.mid_lanes) {  // block-uniform
+    for (uint32_t p = warp; p < rec.plan.pow3P; p += blocks_per_scenario * kWarps)
+      mid_lane_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, p, lane_state + threadIdx.x,
+                               lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
+  } else if (warp < rec.plan.groups * rec.plan.m_parts) {
+    warp_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, warp / rec.plan.m_parts,
+                         warp % rec.plan.m_parts, lane_state + threadIdx.x,
                          lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
+  }
   block_min_to(sink.best, keys + sc);
 }
 

@@ -28,12 +28,14 @@ inline cudaError_t allow_dyn_smem(K kernel, size_t bytes, std::atomic<uint64_t>*
   return e;
 }
 
-// One scenario of a batched search: its tables, its window tables and plan.
+// One scenario of a batched search: its tables, its window tables and plan,
+// and how its warps assign lanes (0: a prefix per lane, warp_task; 1: a mid
+// combination per lane, mid_lane_task).
 struct BatchRecord {
   Tables full;
   Tables window;
   Plan plan;
-  uint32_t pad;
+  uint32_t mid_lanes;
 };
 
 // Window-width buckets: kernels are compiled for NW in this list; a plan whose
