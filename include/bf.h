@@ -167,10 +167,13 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
  * device); a prefix (or a mid combination) is skipped when the time at which
  * its remaining tools can first start, plus the longest path through them in
  * minimum isolated durations min(c, g + x), exceeds the incumbent's makespan
- * -- no mode, contention or queueing makes a tool faster than that.  Exact:
- * the optimum and all its ties are never skipped.  Allocates a 4-byte-per-
- * prefix buffer in the handle on first use.  Blocks until the result is on
- * the host. */
+ * -- no mode, contention or queueing makes a tool faster than that.  When
+ * that first pass keeps more than 1/64 of the prefixes (a DAG without cut
+ * points), the call continues as bf_search_tree over the full space, whose
+ * bound is stronger.  Exact either way: the optimum and all its ties are
+ * never skipped.  Allocates a 4-byte-per-prefix buffer (and, when it hands
+ * over, the tree search's level buffers) in the handle on first use.  Blocks
+ * until the result is on the host. */
 int bf_search_pruned(const bf_scenario* scn, uint64_t hint_index, bf_result* out, void* cuda_stream);
 
 /* Decision spaces of bf_search_tree: the full space (each tool on cpu,

@@ -542,6 +542,10 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   rc = wait_stream(st, who);
   if (rc != BF_OK) return rc;
   const uint32_t nsurv = h->survivors;
+  // A weak prefix bound (no cut points in the DAG) keeps most prefixes; the
+  // tree search, whose expansions bound every node with the forward
+  // earliest-finish pass, then finds the same optimum faster.
+  if ((uint64_t)nsurv * 64u > plan.pow3P) return bf_search_tree(scn, BF_SPACE_FULL, 0u, hint_index, out, nullptr, cuda_stream);
 
   // 3. Full enumeration of the survivors' mappings, bound applied again at the
   //    inner checkpoint; tasks of at least 16 mid combinations, about
