@@ -258,6 +258,13 @@ def _handle(h: Union[ScenarioHandle, Scenario]) -> Tuple[ScenarioHandle, bool]:
     return ScenarioHandle(h), True
 
 
+def _check_out(out_makespan, out_feasible, count: int) -> None:
+    """Output buffers: contiguous CUDA tensors of >= count 4-byte / 1-byte elements."""
+    for t, size, name in ((out_makespan, 4, "out_makespan"), (out_feasible, 1, "out_feasible")):
+        if not (t.is_cuda and t.is_contiguous() and t.element_size() == size and t.numel() >= count):
+            raise ValueError(f"{name} must be a contiguous CUDA tensor of >= {count} {size}-byte elements")
+
+
 def eval_mappings(h: Union[ScenarioHandle, Scenario], first: int, count: int, out_makespan=None,
                   out_feasible=None, stream=None):
     """Makespans (torch.int32 CUDA tensor holding u32 bit patterns) and feasibility
@@ -271,9 +278,7 @@ def eval_mappings(h: Union[ScenarioHandle, Scenario], first: int, count: int, ou
             out_makespan = torch.empty(count, dtype=torch.int32, device="cuda")
         if out_feasible is None:
             out_feasible = torch.empty(count, dtype=torch.uint8, device="cuda")
-        assert out_makespan.is_cuda and out_feasible.is_cuda
-        assert out_makespan.numel() >= count and out_feasible.numel() >= count
-        assert out_makespan.element_size() == 4 and out_feasible.element_size() == 1
+        _check_out(out_makespan, out_feasible, count)
         _check(load().bf_eval_mappings(handle.ptr, first, count, ctypes.c_void_p(out_makespan.data_ptr()),
                                        ctypes.c_void_p(out_feasible.data_ptr()),
                                        ctypes.c_void_p(_stream_handle(stream))))
@@ -340,14 +345,16 @@ def eval_indices(h: Union[ScenarioHandle, Scenario], indices, out_makespan=None,
     """Makespans (torch.int32, u32 bit patterns) and flags (torch.uint8; 0xFF for an
     index outside [0, 3^n)) of the mappings in `indices` (a CUDA int64 tensor)."""
     import torch
+    if not (indices.is_cuda and indices.dtype == torch.int64 and indices.is_contiguous()):
+        raise ValueError("indices must be a contiguous CUDA int64 tensor")
     handle, owned = _handle(h)
     try:
-        assert indices.is_cuda and indices.dtype == torch.int64 and indices.is_contiguous()
         count = indices.numel()
         if out_makespan is None:
             out_makespan = torch.empty(count, dtype=torch.int32, device=indices.device)
         if out_feasible is None:
             out_feasible = torch.empty(count, dtype=torch.uint8, device=indices.device)
+        _check_out(out_makespan, out_feasible, count)
         _check(load().bf_eval_indices(handle.ptr, ctypes.c_void_p(indices.data_ptr()), count,
                                       ctypes.c_void_p(out_makespan.data_ptr()),
                                       ctypes.c_void_p(out_feasible.data_ptr()),

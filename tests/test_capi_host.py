@@ -131,3 +131,12 @@ def test_wide_desc_accepted(lib):
     assert lib.bf_search_batch(descs, 1, out, None) == bf.BF_EINVAL
     assert "n <= 20" in bf.last_error()
     assert lib.bf_search_batch_noalloc(descs, 1, out, None) == bf.BF_EINVAL
+
+
+def test_binding_rejects_bad_output_buffers(lib):
+    """Buffer checks are exceptions (not asserts that `python -O` would drop)."""
+    import torch
+    with pytest.raises(ValueError):
+        bf.eval_indices(S.config0(), torch.zeros(4, dtype=torch.int64))   # a CPU tensor
+    with pytest.raises(ValueError):
+        bf._check_out(torch.zeros(4, dtype=torch.int32), torch.zeros(4, dtype=torch.uint8), 4)
