@@ -63,6 +63,14 @@
 extern "C" {
 #endif
 
+/* Entry points are the library's only exported symbols (it is built with
+ * hidden visibility). */
+#if defined(__GNUC__)
+#define BF_API __attribute__((visibility("default")))
+#else
+#define BF_API
+#endif
+
 #define BF_MAX_TOOLS 32       /* largest scenario (32-bit tool masks) */
 #define BF_MAX_TOOLS_ENUM 20  /* largest scenario of the full-enumeration entry points
                                  (bf_eval_mappings, bf_search_best, bf_search_range,
@@ -118,30 +126,30 @@ typedef struct bf_result {
 typedef struct bf_scenario bf_scenario;
 
 /* Validate a desc without touching the GPU.  BF_OK or BF_EINVAL. */
-int bf_validate_desc(const bf_scenario_desc* desc);
+BF_API int bf_validate_desc(const bf_scenario_desc* desc);
 
 /* Validate `desc`, copy it, allocate the handle's scratch (8-byte device key,
  * 8-byte pinned host key) on the current device and return it in *out.
  * The caller releases it with bf_destroy_scenario.  BF_EINVAL, BF_ENOMEM,
  * BF_ECUDA. */
-int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out);
+BF_API int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out);
 
 /* Release a handle (NULL is accepted).  Synchronises with nothing: the caller
  * must make sure no work using it is still in flight. */
-int bf_destroy_scenario(bf_scenario* scn);
+BF_API int bf_destroy_scenario(bf_scenario* scn);
 
 /* Evaluate mappings [first, first+count) (§2.1's T_e2e under the model):
  * d_makespan[j] = makespan of mapping first+j (0xFFFFFFFF if infeasible),
  * d_feasible[j] = 1/0.  Both are caller-owned device arrays of >= count
  * elements.  Asynchronous on `cuda_stream`.  count == 0 is a no-op.
  * BF_ERANGE if first+count > 3^n; BF_EINVAL on NULL pointers. */
-int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count,
+BF_API int bf_eval_mappings(const bf_scenario* scn, uint64_t first, uint64_t count,
                      uint32_t* d_makespan, uint8_t* d_feasible, void* cuda_stream);
 
 /* Brute-force oracle of §2.3/§4.1 under the model: the feasible mapping of
  * lowest makespan over all 3^n, ties to the lowest index.  Blocks until the
  * result is on the host (bounded wait).  Writes *out on BF_OK. */
-int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_stream);
+BF_API int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_stream);
 
 /* As bf_search_best over mappings [first, first+count) only; out->feasible is
  * 0 (and index = first) when no mapping in the range is feasible.  Range
@@ -149,7 +157,7 @@ int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_stream);
  * lowest index) is the result of their union -- used to split one search
  * across devices or to resume it piecewise.  BF_ERANGE if outside [0, 3^n);
  * count == 0 gives feasible = 0. */
-int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
+BF_API int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
                     bf_result* out, void* cuda_stream);
 
 /* Full search of `count` independent scenarios in one launch (the batched
@@ -157,7 +165,7 @@ int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
  * the first invalid one fails the call with BF_EINVAL naming its position.
  * Allocates and frees its device scratch (packed tables + one key per
  * scenario) per call.  Blocks until the results are on the host. */
-int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
+BF_API int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                     void* cuda_stream);
 
 /* Same result as bf_search_best (the feasible mapping of lowest makespan over
@@ -174,7 +182,7 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
  * never skipped.  Allocates a 4-byte-per-prefix buffer (and, when it hands
  * over, the tree search's level buffers) in the handle on first use.  Blocks
  * until the result is on the host. */
-int bf_search_pruned(const bf_scenario* scn, uint64_t hint_index, bf_result* out, void* cuda_stream);
+BF_API int bf_search_pruned(const bf_scenario* scn, uint64_t hint_index, bf_result* out, void* cuda_stream);
 
 /* Decision spaces of bf_search_tree: the full space (each tool on cpu,
  * gpu_now or gpu_queue; 3^n mappings) or the binary space the paper's S1-S10
@@ -218,7 +226,7 @@ typedef struct bf_tree_stats {
  * full enumeration).  `stats` may be NULL.  Allocates level buffers in the
  * handle on first use (about 1.7 GB for 32 tools in the full space).  Blocks
  * until the result is on the host; every level step is a bounded wait. */
-int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint64_t hint_index,
+BF_API int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint64_t hint_index,
                    bf_result* out, bf_tree_stats* stats, void* cuda_stream);
 
 /* Makespans and feasibility of an arbitrary list of mappings: d_makespan[j] and
@@ -227,7 +235,7 @@ int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint6
  * d_feasible = 0xFF.  Asynchronous on `cuda_stream`; count == 0 is a no-op.
  * Used to score neighbourhoods of a mapping (bf_whatif) or any caller-chosen
  * candidate set. */
-int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t count,
+BF_API int bf_eval_indices(const bf_scenario* scn, const uint64_t* d_indices, uint64_t count,
                     uint32_t* d_makespan, uint8_t* d_feasible, void* cuda_stream);
 
 /* One probe of the runtime monitor's bounded what-if exploration. */
@@ -252,7 +260,7 @@ typedef struct bf_probe {
  * Writes the probes in that order to out[0 .. *count) (at most
  * BF_MAX_PROBES); BF_EINVAL if capacity is smaller than the number of probes,
  * BF_ERANGE if base_index >= 3^n.  Blocks until the results are on the host. */
-int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32_t capacity,
+BF_API int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32_t capacity,
               uint32_t* count, void* cuda_stream);
 
 /* Largest batch bf_search_batch_noalloc accepts. */
@@ -272,18 +280,18 @@ int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out, uint32
  * before any stream capture.  All calls share the one array, so calls whose
  * GPU work overlaps (other threads, other streams) race and must be
  * serialised by the caller.  Blocks until the results are on the host. */
-int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
+BF_API int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                             void* cuda_stream);
 
 /* Time limit of blocking waits, in milliseconds (default 600000; 0 = none).
  * Process-wide. */
-void bf_set_wait_timeout_ms(uint32_t ms);
+BF_API void bf_set_wait_timeout_ms(uint32_t ms);
 
 /* Description of the last failure on this thread ("" if none). */
-const char* bf_last_error(void);
+BF_API const char* bf_last_error(void);
 
 /* Library version string, e.g. "bf 1.0 (model v1)". */
-const char* bf_version(void);
+BF_API const char* bf_version(void);
 
 #ifdef __cplusplus
 }

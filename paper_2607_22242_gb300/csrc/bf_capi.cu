@@ -250,10 +250,19 @@ void build_records(const bf_scenario_desc* descs, uint32_t count, bfk::BatchReco
     work(0, count, &parts[0]);
   } else {
     std::vector<std::thread> pool;
-    for (uint32_t t = 0; t < nthreads; ++t)
-      pool.emplace_back(work, (uint32_t)((uint64_t)count * t / nthreads), (uint32_t)((uint64_t)count * (t + 1) / nthreads),
-                        &parts[t]);
+    bool threads_ok = true;
+    try {
+      for (uint32_t t = 0; t < nthreads; ++t)
+        pool.emplace_back(work, (uint32_t)((uint64_t)count * t / nthreads),
+                          (uint32_t)((uint64_t)count * (t + 1) / nthreads), &parts[t]);
+    } catch (const std::exception&) {
+      threads_ok = false;  // no more threads: finish on this one
+    }
     for (auto& th : pool) th.join();
+    if (!threads_ok) {
+      parts.assign(1, Part{});
+      work(0, count, &parts[0]);
+    }
   }
   for (const Part& p : parts) {
     *wmax = p.wmax > *wmax ? p.wmax : *wmax;
@@ -574,8 +583,8 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   return BF_OK;
 }
 
-int bf_search_tree(const bf_scenario* scn_const, uint32_t space, uint32_t flags, uint64_t hint_index,
-                   bf_result* out, bf_tree_stats* stats, void* cuda_stream) {
+static int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flags, uint64_t hint_index,
+                            bf_result* out, bf_tree_stats* stats, void* cuda_stream) {
   const char* who = "bf_search_tree";
   if (!scn_const || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
   if (space != BF_SPACE_BINARY && space != BF_SPACE_FULL)
@@ -765,7 +774,7 @@ int bf_search_tree(const bf_scenario* scn_const, uint32_t space, uint32_t flags,
   return BF_OK;
 }
 
-int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
+static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
   if (count == 0) return BF_OK;
   if (!descs || !out) return fail(BF_EINVAL, "bf_search_batch: NULL argument");
   uint32_t nmax = 0;
@@ -927,6 +936,28 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
     for (uint32_t j = 0; j < nk; ++j) fill_result(keys[j], descs[i0 + j].n, 0, out + i0 + j);
   }
   return BF_OK;
+}
+
+// Entry points that allocate host memory keep C++ exceptions inside the library.
+int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
+  try {
+    return search_batch_impl(descs, count, out, cuda_stream);
+  } catch (const std::bad_alloc&) {
+    return fail(BF_ENOMEM, "bf_search_batch: host allocation failed");
+  } catch (const std::exception& ex) {
+    return fail(BF_EINVAL, "bf_search_batch: %s", ex.what());
+  }
+}
+
+int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint64_t hint_index, bf_result* out,
+                   bf_tree_stats* stats, void* cuda_stream) {
+  try {
+    return search_tree_impl(scn, space, flags, hint_index, out, stats, cuda_stream);
+  } catch (const std::bad_alloc&) {
+    return fail(BF_ENOMEM, "bf_search_tree: host allocation failed");
+  } catch (const std::exception& ex) {
+    return fail(BF_EINVAL, "bf_search_tree: %s", ex.what());
+  }
 }
 
 void bf_set_wait_timeout_ms(uint32_t ms) { g_wait_timeout_ms.store(ms, std::memory_order_relaxed); }

@@ -20,7 +20,7 @@ def lib():
 
 def declared_functions():
     text = open(HEADER).read()
-    return sorted(set(re.findall(r"^\s*(?:int|void|const char\s*\*)\s*(bf_\w+)\s*\(", text, re.M)))
+    return sorted(set(re.findall(r"^\s*BF_API\s+(?:int|void|const char\s*\*)\s*(bf_\w+)\s*\(", text, re.M)))
 
 
 def test_header_declares_the_abi():
@@ -31,6 +31,17 @@ def test_every_declared_symbol_is_exported(lib):
     for name in declared_functions():
         assert hasattr(lib, name), name
     assert bf.version().startswith("bf ")
+
+
+def test_only_declared_symbols_are_exported(lib):
+    """The library exports its C entry points and nothing of its internals."""
+    import subprocess
+    out = subprocess.run(["nm", "-D", "--defined-only", bf.LIB_PATH], capture_output=True, text=True)
+    if out.returncode != 0:
+        pytest.skip("nm unavailable")
+    names = {line.split()[-1] for line in out.stdout.splitlines() if line.split()[1:2] == ["T"]}
+    assert {n for n in names if n.startswith("bf_")} == set(declared_functions())
+    assert not [n for n in names if n.startswith("_ZN3bfk")], "internal C++ symbols are exported"
 
 
 def test_generated_configs_validate(lib):
