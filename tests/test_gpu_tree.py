@@ -139,6 +139,25 @@ def test_tree_layered24_binary():
             assert _pair(res) == tuple(g["binary"]), (prune, res, st)
 
 
+def test_tree_21_tools_without_cut_points():
+    """A 21-tool layered DAG with no serialisation point: the pruned full-space search equals the
+    unpruned one (every one of the 3^21 mappings simulated), and the binary space equals the
+    oracle's full enumeration of its 2^21 mappings."""
+    rng = np.random.default_rng(21)
+    c, g, x, m = S._ordinary(rng, 21, 2048, 16384)
+    pred = S._layered_edges(rng, [4, 4, 4, 4, 5], 0.4)
+    scn = S.Scenario(21, pred, c, g, x, [40 * v for v in m], m, 40960, S.slowdown_linear(kmax=21))
+    assert segments.bounds(scn) == [(0, 21)]
+    with bf.create_scenario(scn) as h:
+        pruned, _ = bf.search_tree(h, bf.SPACE_FULL, True)
+        full, st = bf.search_tree(h, bf.SPACE_FULL, False)
+        assert _pair(pruned) == _pair(full), (pruned, full)
+        assert st["leaves"] <= 3 ** 21
+        assert oracle.evaluate(scn, pruned.index) == pruned.makespan_us
+        binary, _ = bf.search_tree(h, bf.SPACE_BINARY, True)
+        assert _pair(binary) == oracle.search_binary(scn, THREADS)
+
+
 def test_wide_eval_indices_and_whatif_match_oracle():
     """The 32-slot index-list kernel: random mappings of the 28- and 32-tool workloads, and the what-if probes."""
     import torch
