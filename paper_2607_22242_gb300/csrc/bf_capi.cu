@@ -29,7 +29,8 @@ struct bf_scratch {
   uint32_t pad;
   bfk::BestRecord best;      // tree search: best (makespan, index) so far
   uint32_t bound;            // tree search: makespan bound for pruning
-  uint32_t level_count;      // tree search: nodes appended by the last expansion
+  uint32_t pad2;
+  unsigned long long appended;  // tree search: nodes appended by all expansions so far
   bfk::TreeCounters ctr;     // tree search: counters and error bits
   uint64_t idx[BF_MAX_PROBES];
   uint32_t ms[BF_MAX_PROBES];
@@ -683,7 +684,7 @@ static int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32
   h->best.ms = ~0ull;
   h->best.idx = ~0ull;
   h->bound = bound;
-  h->level_count = 0;
+  h->appended = 0;
   std::memset(&h->ctr, 0, sizeof h->ctr);
   e = cudaMemcpyAsync(&dv->best, &h->best,
                       offsetof(bf_scratch, idx) - offsetof(bf_scratch, best), cudaMemcpyHostToDevice, st);
@@ -732,18 +733,18 @@ static int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32
       ++launches;
       continue;
     }
-    e = cudaMemsetAsync(&dv->level_count, 0, sizeof(uint32_t), st);
+    const unsigned long long before = h->appended;
+    e = bfk::launch_tree_expand(tb, tc, level(L), cap, lo, take, L, level(L + 1), cap, &dv->appended, before,
+                                &dv->bound, &dv->ctr, st);
     if (e == cudaSuccess)
-      e = bfk::launch_tree_expand(tb, tc, level(L), cap, lo, take, L, level(L + 1), cap, &dv->level_count,
-                                  &dv->bound, &dv->ctr, st);
-    if (e == cudaSuccess)
-      e = cudaMemcpyAsync(&h->level_count, &dv->level_count, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+      e = cudaMemcpyAsync(&h->appended, &dv->appended, sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
     if (e != cudaSuccess) return cuda_fail(e, who);
     const int rc = wait_stream(st, who);
     if (rc != BF_OK) return rc;
     ++launches;
-    size[L + 1] = h->level_count;
-    nodes += h->level_count;
+    const uint32_t added = (uint32_t)(h->appended - before);
+    size[L + 1] = added;
+    nodes += added;
   }
 
   // 4. The record.

@@ -5,7 +5,7 @@
 //   tree_expand_kernel : one thread per (parent, mode of the next tool); the
 //                        child is resumed to its checkpoint, bounded, and the
 //                        survivors are appended to the next level's buffer
-//                        (one atomicAdd per warp).
+//                        (one atomicAdd per warp on a running total).
 //   tree_leaf_kernel   : one warp per 32 leaf-level nodes (one per lane) and a
 //                        chunk of the radix^D combinations of the last D tools,
 //                        walked in lockstep over the leaf window (tools from the
@@ -40,7 +40,7 @@ __global__ void tree_root_kernel(const __grid_constant__ TablesW tb, uint32_t* b
 __global__ void __launch_bounds__(kTreeThreads, 2) tree_expand_kernel(
     const __grid_constant__ TablesW tb, const __grid_constant__ TreeConsts tc, const uint32_t* __restrict__ src,
     uint32_t src_cap, uint32_t lo, uint32_t cnt, uint32_t d, uint32_t* __restrict__ dst, uint32_t dst_cap,
-    uint32_t* dst_count, const uint32_t* bound, TreeCounters* ctr) {
+    unsigned long long* appended, unsigned long long base_total, const uint32_t* bound, TreeCounters* ctr) {
   __shared__ SmemTablesW sd;
   __shared__ uint32_t rt[ReadyTable<kTreeSlots>::size];
   __shared__ uint32_t ef[kTreeSlots * kTreeThreads];  // forward_bound scratch, [tool][thread]
@@ -62,16 +62,18 @@ __global__ void __launch_bounds__(kTreeThreads, 2) tree_expand_kernel(
   if (ballot == 0u) return;
   const uint32_t lane = threadIdx.x & 31u;
   const uint32_t leader = __ffs(ballot) - 1;
-  uint32_t base = 0u;
-  if (lane == leader) base = atomicAdd(dst_count, (uint32_t)__popc(ballot));
+  // `appended` counts every node appended by every expansion of this search;
+  // this launch's children get slots from base_total (its value at launch) on.
+  unsigned long long base = 0ull;
+  if (lane == leader) base = atomicAdd(appended, (unsigned long long)__popc(ballot));
   base = __shfl_sync(0xFFFFFFFFu, base, leader);
   if (!keep) return;
-  const uint32_t slot = base + __popc(ballot & ((1u << lane) - 1u));
+  const uint64_t slot = (base - base_total) + (uint64_t)__popc(ballot & ((1u << lane) - 1u));
   if (slot >= dst_cap) {  // cannot happen (cnt * radix <= dst_cap); recorded, never written
     atomicOr(&ctr->error, 1u);
     return;
   }
-  store_node(s, dg, dst, dst_cap, slot);
+  store_node(s, dg, dst, dst_cap, (uint32_t)slot);
 }
 
 // Lexicographic (makespan, index) minimum of the 16-byte record at *p.  Every
@@ -224,10 +226,11 @@ cudaError_t launch_tree_root(const TablesW& tb, uint32_t* buf, uint32_t cap, cud
 
 cudaError_t launch_tree_expand(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
                                uint32_t lo, uint32_t cnt, uint32_t d, uint32_t* dst, uint32_t dst_cap,
-                               uint32_t* dst_count, const uint32_t* bound, TreeCounters* ctr, cudaStream_t st) {
+                               unsigned long long* appended, unsigned long long base_total, const uint32_t* bound,
+                               TreeCounters* ctr, cudaStream_t st) {
   const uint64_t threads = (uint64_t)cnt * tc.radix;
   const unsigned grid = (unsigned)((threads + kTreeThreads - 1) / kTreeThreads);
-  tree_expand_kernel<<<grid, kTreeThreads, 0, st>>>(tb, tc, src, src_cap, lo, cnt, d, dst, dst_cap, dst_count, bound,
+  tree_expand_kernel<<<grid, kTreeThreads, 0, st>>>(tb, tc, src, src_cap, lo, cnt, d, dst, dst_cap, appended, base_total, bound,
                                                     ctr);
   return cudaGetLastError();
 }

@@ -29,7 +29,8 @@ size_t tree_node_words();
 cudaError_t launch_tree_root(const TablesW& tb, uint32_t* buf, uint32_t cap, cudaStream_t st);
 cudaError_t launch_tree_expand(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
                                uint32_t lo, uint32_t cnt, uint32_t d, uint32_t* dst, uint32_t dst_cap,
-                               uint32_t* dst_count, const uint32_t* bound, TreeCounters* ctr, cudaStream_t st);
+                               unsigned long long* appended, unsigned long long base_total, const uint32_t* bound,
+                               TreeCounters* ctr, cudaStream_t st);
 cudaError_t launch_tree_leaf(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
                              uint32_t lo, uint32_t cnt, uint32_t target_tasks, uint32_t* bound, BestRecord* best,
                              TreeCounters* ctr, cudaStream_t st);
