@@ -611,6 +611,16 @@ static int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32
   tc.prune = prune ? 1u : 0u;
   tc.W0 = bfk::host::window_start(tb, tc.leaf_level);
   {
+    uint32_t anc[bfk::kTreeSlots];
+    bfk::host::ancestors(tb, anc);
+    const uint32_t last = n - 1, others = (last >= 32u) ? ~0u : ((1u << last) - 1u);
+    tc.alone_last = (tc.D >= 1u && (anc[last] & others) == others) ? 1u : 0u;
+    const bool fits = tb.vram[last] <= tb.budget;
+    tc.alone[0] = tb.cpu[last];
+    tc.alone[1] = fits ? tb.wnow[last] >> 10 : 0xFFFFFFFFu;
+    tc.alone[2] = fits ? tb.wq[last] >> 10 : 0xFFFFFFFFu;
+  }
+  {
     uint64_t down[bfk::kTreeSlots] = {0};
     for (int v = (int)n - 1; v >= 0; --v) {
       const uint32_t gpu = tb.wnow[v] >> 10;

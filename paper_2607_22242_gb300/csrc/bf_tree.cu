@@ -144,11 +144,14 @@ __global__ void __launch_bounds__(LeafShape<NW>::threads, LeafShape<NW>::min_blo
         node_to_window<NW>(src, src_cap, lo + j, tc.W0, tw.n, slot, LeafShape<NW>::threads);
     }
     const uint32_t ran = __ballot_sync(0xFFFFFFFFu, valid);
+    // With a lone last tool, combinations cover the leaf tools but the last
+    // one, each standing for radix mappings.
+    const uint32_t ncomb = tc.alone_last ? tc.combos / tc.radix : tc.combos;
     const uint32_t c0 = part * chunk;
-    const uint32_t c1 = min(c0 + chunk, tc.combos);
+    const uint32_t c1 = min(c0 + chunk, ncomb);
     if (lane == 0 && ran) {
       if (part == 0) atomicAdd(&ctr->leaf_nodes, (unsigned long long)__popc(ran));
-      atomicAdd(&ctr->leaves, (unsigned long long)__popc(ran) * (c1 - c0));
+      atomicAdd(&ctr->leaves, (unsigned long long)__popc(ran) * (c1 - c0) * (tc.alone_last ? tc.radix : 1u));
     }
     if (ran) leaf_combos<NW>(tw, sdw, rtw, tc, slot, LeafShape<NW>::threads, dg, valid, c0, c1, lb);
   }
@@ -260,12 +263,13 @@ cudaError_t launch_tree_leaf(const TablesW& tb, const TreeConsts& tc, const uint
   // Split each group's combinations into parts so that about target_tasks
   // warp tasks exist, each covering at least 16 combinations.
   const uint32_t groups = (cnt + 31u) / 32u;
+  const uint32_t ncomb = tc.alone_last ? tc.combos / tc.radix : tc.combos;
   uint32_t parts = (target_tasks + groups - 1u) / groups;
-  const uint32_t max_parts = (tc.combos + 15u) / 16u;
+  const uint32_t max_parts = (ncomb + 15u) / 16u;
   if (parts > max_parts) parts = max_parts;
   if (parts < 1u) parts = 1u;
-  const uint32_t chunk = (tc.combos + parts - 1u) / parts;
-  parts = (tc.combos + chunk - 1u) / chunk;
+  const uint32_t chunk = (ncomb + parts - 1u) / parts;
+  parts = (ncomb + chunk - 1u) / chunk;
   const uint64_t tasks = (uint64_t)groups * parts;
   const unsigned grid = (unsigned)((tasks + kTreeWarps - 1) / kTreeWarps);
   const uint32_t nw = tb.n - tc.W0;

@@ -36,6 +36,11 @@ struct TreeConsts {
   uint32_t combos;       // radix^D
   uint32_t prune;        // 0: keep every node (full enumeration)
   uint32_t W0;           // leaf window start: tools below it have ended at every leaf checkpoint
+  // 1 when every other tool precedes the last one: when it becomes ready it
+  // runs alone, and ends alone[a] after that instant in mode a (0xFFFFFFFF: a
+  // GPU mode over budget) -- the model's one remaining event at k = 1.
+  uint32_t alone_last;
+  uint32_t alone[3];
   uint32_t dmin[kTreeSlots];   // min(c, g + x): no mode runs tool v faster
   uint32_t sdown[kTreeSlots];  // longest path in dmin through v's successors (0 for a sink)
   uint64_t pow3[kTreeSlots];
@@ -302,12 +307,34 @@ struct LaneBest {
 // shared-memory window state, stride `stride`) whose digits are `dg` (all
 // tools); tw/sdw/rtw are the window's tables.  `valid` false runs the loop
 // without work (lanes of a warp stay in lockstep).
+// With tc.alone_last, [c0, c1) are combinations of the leaf tools but the
+// last one: each is simulated until the last tool becomes ready (everything
+// else has ended then) and yields one makespan per mode of the last tool.
 template <int NW, typename TBW, typename SD>
 __device__ __forceinline__ void leaf_combos(const TBW& tw, const SD& sdw, const uint32_t* rtw, const TreeConsts& tc,
                                             const uint32_t* slot, uint32_t stride, Digits dg, bool valid,
                                             uint32_t c0, uint32_t c1, LaneBest& best) {
   const uint32_t L = tc.leaf_level, W0 = tc.W0;
   const Digits dgw{dg.now >> W0, dg.que >> W0};
+  if (tc.alone_last) {
+    const uint32_t last = tc.n - 1u, lastw = last - W0;
+    for (uint32_t c = c0; c < c1; ++c) {
+      if (!valid) continue;
+      const Digits dc = leaf_digits(c, tc.radix, tc.D - 1u, L - W0);
+      const Digits sim{dgw.now | dc.now, dgw.que | dc.que};
+      if (sim.que & tw.big_mask) continue;
+      State<NW> w;
+      load_lane(slot, stride, w);
+      if (run<NW>(w, tw, sdw, rtw, sim, 1u << lastw) != kRunStopped) continue;  // infeasible before it
+      const Digits full{dg.now | (dc.now << W0), dg.que | (dc.que << W0)};
+      for (uint32_t a = 0; a < tc.radix; ++a) {
+        if (tc.alone[a] == kInfeasible) continue;
+        best.offer(w.T + tc.alone[a], Digits{full.now | (a == 1u ? 1u << last : 0u),
+                                               full.que | (a == 2u ? 1u << last : 0u)});
+      }
+    }
+    return;
+  }
   for (uint32_t c = c0; c < c1; ++c) {
     if (!valid) continue;
     const Digits dc = leaf_digits(c, tc.radix, tc.D, L - W0);
