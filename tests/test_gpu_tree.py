@@ -182,6 +182,23 @@ def test_wide_eval_indices_and_whatif_match_oracle():
                 assert got == W.whatif(scn, base), (name, base)
 
 
+def test_empty_and_single_inputs():
+    """Empty index lists and batches, and one-tool scenarios, on every path that takes them."""
+    import torch
+    one = S.Scenario(1, [0], [50], [5], [3], [4], [10], 20, S.slowdown_flat())
+    with bf.create_scenario(one) as h:
+        ms, fe = bf.eval_indices(h, torch.empty(0, dtype=torch.int64, device="cuda"))
+        assert ms.numel() == 0 and fe.numel() == 0
+        want = oracle.search(one)
+        assert _pair(bf.search_best(h)) == want == (1, 8)
+        assert _pair(bf.search_pruned(h)) == want
+        for space in (bf.SPACE_FULL, bf.SPACE_BINARY):
+            for prune in (True, False):
+                assert _pair(bf.search_tree(h, space, prune)[0]) == want
+        assert [p.index for p in bf.whatif(h, 0)] == [1, 2]
+    assert bf.search_batch([]) == [] and bf.search_batch_noalloc([]) == []
+
+
 def test_tree_argument_errors():
     scn = S.config0()
     with bf.create_scenario(scn) as h:
