@@ -272,6 +272,26 @@ def per_config_times(torch, bf, S, stream, reps: int = 5):
     return out
 
 
+def cpu_model() -> str:
+    """Host CPU model name (lscpu, else /proc/cpuinfo, else the machine type)."""
+    import platform
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except (OSError, subprocess.SubprocessError):
+        pass
+    try:
+        with open("/proc/cpuinfo") as fh:
+            for line in fh:
+                if line.startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except OSError:
+        pass
+    return platform.machine()
+
+
 def oracle_single_core(S, seconds_per_config: float = 1.5):
     """The oracle on one host thread: mappings/s per standard workload on a timed slice of its index space."""
     import oracle
@@ -433,7 +453,8 @@ def run_gpu(args):
         out["cpu_baseline"] = {"value": n / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
                                "sample": f"{n} mappings of the same workload in 16 contiguous chunks spread "
                                          f"evenly over [0, 3^19), oracle search, {dt:.1f} s",
-                               "single_core_per_config": oracle_single_core(S)}
+                               "single_core_per_config": oracle_single_core(S),
+                               "cpu_model": cpu_model()}
     emit(out)
     if world > 1:
         torch.distributed.destroy_process_group()
