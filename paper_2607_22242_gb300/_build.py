@@ -2,7 +2,7 @@
 
 Each window-width bucket of ``csrc/bf_kernels.cu`` is its own translation unit
 (``-DBF_NW=<slots>``); the units compile in parallel and link with ``bf_tree.cu``
-(the tree search and 32-slot index lists) and ``bf_capi.cu`` into
+(the tree search and 32-slot index lists), ``bf_capi.cu`` and ``bf_capi_tree.cu`` into
 ``paper_2607_22242_gb300/_build/libbf.so`` (CUDA runtime linked statically, so
 the library carries no path to a toolkit; no undefined symbol is allowed).
 """
@@ -79,7 +79,7 @@ def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
         obj = os.path.join(BUILD_DIR, f"bf_kernels_nw{nt}.o")
         jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, f"-DBF_NW={nt}", "-c",
                      os.path.join(CSRC, "bf_kernels.cu"), "-o", obj])
-    for unit in ("bf_tree", "bf_capi"):
+    for unit in ("bf_tree", "bf_capi", "bf_capi_tree"):
         jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, unit + ".cu"), "-o",
                      os.path.join(BUILD_DIR, unit + ".o")])
 

@@ -1,6 +1,7 @@
 // bf_capi.cu -- the C ABI declared in include/bf.h: scenario validation, the
-// device-format tables, launches and bounded waits.  All search arithmetic
-// runs in the kernels (bf_kernels.cu, bf_sim.cuh); this file only marshals.
+// device-format tables, launches and bounded waits (the tree search's host
+// side is in bf_capi_tree.cu).  All search arithmetic runs in the kernels
+// (bf_kernels.cu, bf_sim.cuh, bf_tree.cu); this file only marshals.
 #include <cuda_runtime.h>
 
 #include <atomic>
@@ -10,50 +11,14 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <algorithm>
 #include <string>
 #include <thread>
-#include <algorithm>
 #include <vector>
 
-#include "../../include/bf.h"
-#include "bf_launch.h"
-#include "bf_plan.h"
-#include "bf_tree.h"
+#include "bf_capi_internal.h"
 
-// Per-handle scratch, one block on the device and a pinned mirror on the host:
-// the packed search key, the tree search's best record, bound and counters,
-// and the what-if probe list with its results.
-struct bf_scratch {
-  unsigned long long key;
-  uint32_t survivors;   // pruned search: number of surviving prefixes
-  uint32_t pad;
-  bfk::BestRecord best;      // tree search: best (makespan, index) so far
-  uint32_t bound;            // tree search: makespan bound for pruning
-  uint32_t pad2;
-  unsigned long long appended;  // tree search: nodes appended by all expansions so far
-  bfk::TreeCounters ctr;     // tree search: counters and error bits
-  uint64_t idx[BF_MAX_PROBES];
-  uint32_t ms[BF_MAX_PROBES];
-  uint8_t fe[BF_MAX_PROBES];
-};
-
-struct bf_scenario {
-  bf_scenario_desc desc;
-  bfk::TablesW wide;    // all n tools, 32 slots (index lists and the tree search)
-  bfk::Tables tables;   // all n tools (n <= BF_MAX_TOOLS_ENUM; zero otherwise)
-  bfk::Tables window;   // tools [W0, n), renumbered from 0
-  bfk::Plan plan;       // enumeration split and window (see bfk::Plan), full range
-  int device;
-  bf_scratch* d_scratch;      // device scratch
-  bf_scratch* h_scratch;      // pinned host mirror
-  unsigned long long* d_key;  // &d_scratch->key
-  unsigned long long* h_key;  // &h_scratch->key
-  uint32_t* d_survivors;      // pruned search: 3^P prefix slots, allocated on first use
-  uint32_t* d_levels;         // tree search: node buffers of every level, allocated on first use
-  size_t levels_bytes;
-};
-
-namespace {
+namespace bfcapi {
 
 using bfk::host::build_tables;
 using bfk::host::make_plan;
@@ -304,7 +269,9 @@ int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result
   return BF_OK;
 }
 
-}  // namespace
+}  // namespace bfcapi
+
+using namespace bfcapi;
 
 extern "C" {
 
@@ -584,207 +551,6 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   return BF_OK;
 }
 
-static int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flags, uint64_t hint_index,
-                            bf_result* out, bf_tree_stats* stats, void* cuda_stream) {
-  const char* who = "bf_search_tree";
-  if (!scn_const || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
-  if (space != BF_SPACE_BINARY && space != BF_SPACE_FULL)
-    return fail(BF_EINVAL, "%s: space %u is neither BF_SPACE_BINARY (2) nor BF_SPACE_FULL (3)", who, space);
-  if (flags & ~(uint32_t)BF_TREE_NO_PRUNE) return fail(BF_EINVAL, "%s: unknown flags 0x%x", who, flags);
-  if (const int rc = check_device(scn_const, who)) return rc;
-  // The handle's lazily allocated level buffers are scratch, not state.
-  bf_scenario* scn = const_cast<bf_scenario*>(scn_const);
-  const bfk::TablesW& tb = scn->wide;
-  const uint32_t n = scn->desc.n, R = space;
-  const bool prune = !(flags & BF_TREE_NO_PRUNE);
-  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-
-  // Constants: the leaf depth, the bound's per-tool durations, digit powers.
-  bfk::TreeConsts tc;
-  std::memset(&tc, 0, sizeof tc);
-  tc.n = n;
-  tc.radix = R;
-  tc.D = n < (R == 3 ? 5u : 8u) ? n : (R == 3 ? 5u : 8u);
-  tc.leaf_level = n - tc.D;
-  tc.combos = 1;
-  for (uint32_t i = 0; i < tc.D; ++i) tc.combos *= R;
-  tc.prune = prune ? 1u : 0u;
-  tc.W0 = bfk::host::window_start(tb, tc.leaf_level);
-  {
-    uint32_t anc[bfk::kTreeSlots];
-    bfk::host::ancestors(tb, anc);
-    const uint32_t last = n - 1, others = (last >= 32u) ? ~0u : ((1u << last) - 1u);
-    tc.alone_last = (tc.D >= 1u && (anc[last] & others) == others) ? 1u : 0u;
-    const bool fits = tb.vram[last] <= tb.budget;
-    tc.alone[0] = tb.cpu[last];
-    tc.alone[1] = fits ? tb.wnow[last] >> 10 : 0xFFFFFFFFu;
-    tc.alone[2] = fits ? tb.wq[last] >> 10 : 0xFFFFFFFFu;
-  }
-  {
-    uint64_t down[bfk::kTreeSlots] = {0};
-    for (int v = (int)n - 1; v >= 0; --v) {
-      const uint32_t gpu = tb.wnow[v] >> 10;
-      tc.dmin[v] = tb.cpu[v] < gpu ? tb.cpu[v] : gpu;
-      uint64_t longest = 0;
-      for (uint32_t w = (uint32_t)v + 1; w < n; ++w)
-        if ((tb.succ[v] >> w) & 1u) longest = down[w] > longest ? down[w] : longest;
-      tc.sdown[v] = (uint32_t)(longest < 0xFFFFFFFFull ? longest : 0xFFFFFFFFull);
-      down[v] = tc.dmin[v] + longest;
-    }
-    uint64_t p = 1;
-    for (uint32_t i = 0; i < (uint32_t)bfk::kTreeSlots; ++i, p *= 3) tc.pow3[i] = p;
-  }
-
-  // Level buffers: level d holds up to R * kPop nodes (one pop of its parent
-  // level); nodes are popped from the deepest non-empty level, so no level
-  // ever holds more.
-  constexpr uint32_t kPop = 65536;
-  const uint32_t cap = R * kPop;
-  const uint32_t levels = tc.leaf_level + 1;
-  const size_t level_words = bfk::tree_node_words() * cap;
-  const size_t need = sizeof(uint32_t) * level_words * levels;
-  cudaError_t e = cudaSuccess;
-  if (scn->levels_bytes < need) {
-    if (scn->d_levels) cudaFree(scn->d_levels);
-    scn->d_levels = nullptr;
-    scn->levels_bytes = 0;
-    e = lib_malloc(reinterpret_cast<void**>(&scn->d_levels), need);
-    if (e != cudaSuccess) return cuda_fail(e, who);
-    scn->levels_bytes = need;
-  }
-  auto level = [&](uint32_t d) { return scn->d_levels + level_words * d; };
-
-  bf_scratch* h = scn->h_scratch;
-  bf_scratch* dv = scn->d_scratch;
-  uint32_t launches = 0;
-
-  // 1. Incumbent: the best feasible of a few mappings of the space (the hint
-  //    if it lies in it, all-cpu, all-gpu_now, each tool on its isolated-faster
-  //    device, and all-gpu_queue in the full space).
-  uint32_t bound = 0xFFFFFFFFu;
-  if (prune) {
-    const uint64_t total = pow3(n);
-    uint32_t nc = 0;
-    bool hint_ok = hint_index < total;
-    if (hint_ok && R == 2)
-      for (uint64_t v = hint_index; v; v /= 3) hint_ok = hint_ok && (v % 3 != 2);
-    if (hint_ok) h->idx[nc++] = hint_index;
-    uint64_t now = 0, fast = 0, p = 1;
-    for (uint32_t i = 0; i < n; ++i, p *= 3) {
-      now += p;
-      if ((tb.wnow[i] >> 10) < tb.cpu[i]) fast += p;
-    }
-    h->idx[nc++] = 0;
-    h->idx[nc++] = now;
-    h->idx[nc++] = fast;
-    if (R == 3) h->idx[nc++] = 2 * now;
-    e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
-    if (e == cudaSuccess) e = launch_list(scn, dv->idx, nc, dv->ms, dv->fe, 1, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(h->ms, dv->ms, sizeof(uint32_t) * nc, cudaMemcpyDeviceToHost, st);
-    if (e == cudaSuccess) e = cudaMemcpyAsync(h->fe, dv->fe, nc, cudaMemcpyDeviceToHost, st);
-    if (e != cudaSuccess) return cuda_fail(e, who);
-    const int rc = wait_stream(st, who);
-    if (rc != BF_OK) return rc;
-    ++launches;
-    for (uint32_t j = 0; j < nc; ++j)
-      if (h->fe[j] == 1 && h->ms[j] < bound) bound = h->ms[j];
-  }
-
-  // 2. Reset the record, bound and counters; write the root node.
-  h->best.ms = ~0ull;
-  h->best.idx = ~0ull;
-  h->bound = bound;
-  h->appended = 0;
-  std::memset(&h->ctr, 0, sizeof h->ctr);
-  e = cudaMemcpyAsync(&dv->best, &h->best,
-                      offsetof(bf_scratch, idx) - offsetof(bf_scratch, best), cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) e = bfk::launch_tree_root(tb, level(0), cap, st);
-  if (e != cudaSuccess) return cuda_fail(e, who);
-  ++launches;
-
-  // 3. Depth first over levels: pop up to kPop nodes (a whole leaf-level
-  //    buffer) from the deepest non-empty level, and expand them into the
-  //    next level or enumerate their leaves.  A large tree starts with a
-  //    dive: pops of kDive nodes reach the leaves after one expansion per
-  //    level, and the first leaves' makespans become the bound; the dive's
-  //    other nodes are then dropped and the search restarts from the root
-  //    (the root stays in the level-0 buffer), now pruning the wide levels
-  //    with that bound.  (Measured: 8192 beat 64 and 1024, and beat diving
-  //    without the restart.)
-  constexpr uint32_t kDive = 8192;
-  std::vector<uint32_t> size(levels, 0);
-  size[0] = 1;
-  uint64_t nodes = 1;
-  uint64_t leaf_level_nodes = 1;  // radix^L, saturating
-  for (uint32_t i = 0; i < tc.leaf_level && leaf_level_nodes <= kPop; ++i) leaf_level_nodes *= R;
-  bool diving = prune && leaf_level_nodes > kPop;
-  for (;;) {
-    int d = (int)levels - 1;
-    while (d >= 0 && size[d] == 0) --d;
-    if (d < 0) break;
-    const uint32_t L = (uint32_t)d;
-    const uint32_t pop = diving ? kDive : kPop;
-    const uint32_t take = L == tc.leaf_level ? size[L] : (size[L] < pop ? size[L] : pop);
-    if (diving && L == tc.leaf_level) {
-      e = bfk::launch_tree_leaf(tb, tc, level(L), cap, size[L] - take, take, 16384, &dv->bound, &dv->best, &dv->ctr,
-                                st);
-      if (e != cudaSuccess) return cuda_fail(e, who);
-      ++launches;
-      std::fill(size.begin(), size.end(), 0u);
-      size[0] = 1;
-      diving = false;
-      continue;
-    }
-    const uint32_t lo = size[L] - take;
-    size[L] = lo;
-    if (L == tc.leaf_level) {
-      e = bfk::launch_tree_leaf(tb, tc, level(L), cap, lo, take, 16384, &dv->bound, &dv->best, &dv->ctr, st);
-      if (e != cudaSuccess) return cuda_fail(e, who);
-      ++launches;
-      continue;
-    }
-    const unsigned long long before = h->appended;
-    e = bfk::launch_tree_expand(tb, tc, level(L), cap, lo, take, L, level(L + 1), cap, &dv->appended, before,
-                                &dv->bound, &dv->ctr, st);
-    if (e == cudaSuccess)
-      e = cudaMemcpyAsync(&h->appended, &dv->appended, sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
-    if (e != cudaSuccess) return cuda_fail(e, who);
-    const int rc = wait_stream(st, who);
-    if (rc != BF_OK) return rc;
-    ++launches;
-    const uint32_t added = (uint32_t)(h->appended - before);
-    size[L + 1] = added;
-    nodes += added;
-  }
-
-  // 4. The record.
-  e = cudaMemcpyAsync(&h->best, &dv->best,
-                      offsetof(bf_scratch, idx) - offsetof(bf_scratch, best), cudaMemcpyDeviceToHost, st);
-  if (e != cudaSuccess) return cuda_fail(e, who);
-  const int rc = wait_stream(st, who);
-  if (rc != BF_OK) return rc;
-  if (h->ctr.error) return fail(BF_ECUDA, "%s: internal error 0x%x in the tree kernels", who, h->ctr.error);
-  std::memset(out, 0, sizeof *out);
-  if (h->best.ms >= 0xFFFFFFFFull) {
-    out->makespan_us = 0xFFFFFFFFu;
-  } else {
-    out->index = h->best.idx;
-    out->makespan_us = (uint32_t)h->best.ms;
-    out->feasible = 1;
-    uint64_t idx = out->index;
-    for (uint32_t i = 0; i < n; ++i, idx /= 3) out->mode[i] = (uint8_t)(idx % 3);
-  }
-  if (stats) {
-    stats->nodes = nodes;
-    stats->leaf_nodes = h->ctr.leaf_nodes;
-    stats->leaves = h->ctr.leaves;
-    stats->launches = launches;
-    stats->leaf_depth = tc.D;
-    stats->incumbent_us = bound;
-  }
-  return BF_OK;
-}
-
 static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
   if (count == 0) return BF_OK;
   if (!descs || !out) return fail(BF_EINVAL, "bf_search_batch: NULL argument");
@@ -957,17 +723,6 @@ int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* ou
     return fail(BF_ENOMEM, "bf_search_batch: host allocation failed");
   } catch (const std::exception& ex) {
     return fail(BF_EINVAL, "bf_search_batch: %s", ex.what());
-  }
-}
-
-int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint64_t hint_index, bf_result* out,
-                   bf_tree_stats* stats, void* cuda_stream) {
-  try {
-    return search_tree_impl(scn, space, flags, hint_index, out, stats, cuda_stream);
-  } catch (const std::bad_alloc&) {
-    return fail(BF_ENOMEM, "bf_search_tree: host allocation failed");
-  } catch (const std::exception& ex) {
-    return fail(BF_EINVAL, "bf_search_tree: %s", ex.what());
   }
 }
 
