@@ -251,7 +251,7 @@ typedef struct bf_probe {
 
 #define BF_MAX_PROBES (2 * BF_MAX_TOOLS + BF_MAX_TOOLS * BF_MAX_TOOLS)
 
-/* The what-if probes of Algorithm 1 (lines 4-13, §3.2) around mapping
+/* The what-if probes of Algorithm 1's exploration step (§3.2) around mapping
  * base_index, scored on the model in one launch: for each tool i in index
  * order and each alternative mode a != d_i (in the order cpu, gpu_now,
  * gpu_queue), the single-tool reprobe d[i := a]; when that reprobe moves i to

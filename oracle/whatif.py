@@ -1,6 +1,6 @@
 """Algorithm 1's bounded what-if exploration on the model -- TEST INFRASTRUCTURE.
 
-Lines 4-13 of Algorithm 1 (runtime monitor, §3.2) for a base mapping d: for
+The exploration step of Algorithm 1 (runtime monitor, §3.2) for a base mapping d: for
 each tool i and each alternative mode a != d_i, the single-tool reprobe
 d[i := a]; if that reprobe exceeds the VRAM budget and a is gpu_now, a swap
 reprobe d[i := gpu_now, j := gpu_queue] for each tool j currently on gpu_now.
