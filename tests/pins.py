@@ -273,7 +273,7 @@ ALL_CHECKS = [
 
 
 def check_fig7_whatif(lib):
-    """Figure 7's what-if block: around round 2's mapping (A:GN B:GN C:GQ D:CPU)
+    """Figure 7's what-if block: around the mapping of the monitor's second round (A:GN B:GN C:GQ D:CPU)
     Algorithm 1 reprobes C -> gpu_now, which exceeds 1100 MB, and then swaps C
     with each gpu_now tool; every probe printed there appears with its status
     and, for swaps, the printed full mapping."""

@@ -1,4 +1,4 @@
-"""Host-side fault injection on a GPU machine: failures are made on the host (an
+"""Host-side fault injection with a GPU present: failures are made on the host (an
 allocation the library is told to fail), never on the GPU."""
 import os
 import subprocess
