@@ -289,6 +289,53 @@ def test_non_default_stream():
     assert np.array_equal(ms.cpu().numpy().view(np.uint32).astype(np.uint64), o_ms)
 
 
+def test_concurrent_handles_on_host_threads(golden):
+    """Calls on different handles may run at once: five host threads, each with its own handle
+    (or batch) and its own CUDA stream, repeat full searches, a tree search and a batched search
+    concurrently; every result equals the stored oracle optimum."""
+    import threading
+    import torch
+    with open(os.path.join(GOLDEN, "wide_results.json")) as fh:
+        wide = json.load(fh)["workloads"]["wide28"]
+    batch = S.config4(256)
+    want_batch = [(i, m) for i, m in zip(golden["4"]["best_index"][:256], golden["4"]["best_makespan"][:256])]
+
+    def full(cfg):
+        g = golden[str(cfg)]["summary"]
+        return lambda h, st: (bf.search_best(h, st), (g["best_index"], g["best_makespan"]))
+
+    jobs = [(S.config0(), full(0)), (S.config1(), full(1)), (S.config2(), full(2)),
+            (S.wide28(), lambda h, st: (bf.search_tree(h, bf.SPACE_FULL, True, None, st)[0], tuple(wide["ternary"]))),
+            (None, None)]
+    errors = []
+
+    def worker(scn, call):
+        try:
+            torch.cuda.set_device(0)
+            st = torch.cuda.Stream()
+            if scn is None:
+                for _ in range(4):
+                    got = [(r.index, r.makespan_us) for r in bf.search_batch(batch, st)]
+                    if got != want_batch:
+                        errors.append("batch")
+                return
+            with bf.create_scenario(scn) as h:
+                for _ in range(4):
+                    res, want = call(h, st)
+                    if (res.index, res.makespan_us) != want:
+                        errors.append((scn.n, res.index, res.makespan_us, want))
+        except Exception as exc:  # reported below; a thread's exception would otherwise vanish
+            errors.append(repr(exc))
+
+    threads = [threading.Thread(target=worker, args=job) for job in jobs]
+    for t in threads:
+        t.start()
+    for t in threads:
+        t.join(timeout=300)
+    assert not any(t.is_alive() for t in threads)
+    assert errors == []
+
+
 def test_wait_timeout_is_reported():
     """The host wait is bounded: a 1 ms limit on a ~0.1 s search returns BF_ETIMEOUT, the GPU
     work finishes normally, and the library works afterwards."""
