@@ -94,7 +94,7 @@ __device__ __forceinline__ void prefix_task(const TBF& tb, const SmemTables& sd,
       continue;
     }
     if ((uint64_t)w.T + plan.tail_q > plan.bound) continue;  // pruned at the inner checkpoint
-    if ((w.done | inner_mask) == 0xFFFFFFFFu) {
+    if (plan.I == 1u && (w.done | inner_mask) == 0xFFFFFFFFu) {
       // Everything but the last tool has ended: it runs alone from w.T.
       for (uint32_t i = i_lo; i <= i_hi; ++i) {
         const uint32_t d = plan.alone[i];
@@ -177,7 +177,7 @@ __device__ __forceinline__ void mid_lane_task(const TBF& tb, const SmemTables& s
       for (uint32_t i = 0; i < plan.pow3I; ++i) sink((uint32_t)(base + stride_i * i), kInfeasible);
       continue;
     }
-    if ((w.done | inner_mask) == 0xFFFFFFFFu) {
+    if (plan.I == 1u && (w.done | inner_mask) == 0xFFFFFFFFu) {  // the last tool runs alone
       for (uint32_t i = 0; i < plan.pow3I; ++i) {
         const uint32_t d = plan.alone[i];
         sink((uint32_t)(base + stride_i * i), d == kInfeasible ? kInfeasible : w.T + d);
