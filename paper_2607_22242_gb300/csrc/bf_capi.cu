@@ -24,6 +24,8 @@ using bfk::host::build_tables;
 using bfk::host::make_plan;
 using bfk::host::pow3;
 using bfk::host::split_and_window;
+using bfk::host::split_and_window_batch;
+using bfk::host::split_and_window_pruned;
 
 // Warp tasks a single-scenario launch is split into (several waves of the
 // GPU's resident warps, so that uneven tasks even out).
@@ -198,7 +200,7 @@ void build_records(const bf_scenario_desc* descs, uint32_t count, bfk::BatchReco
       std::memset(&r, 0, sizeof r);
       build_tables(descs + i, &r.full);
       bfk::Plan base;
-      split_and_window(r.full, &base, &r.window);
+      split_and_window_batch(r.full, &base, &r.window);
       r.plan = batch_plan(base, descs[i].n);
       r.mid_lanes = base.W0 == 0u ? 1u : 0u;
       if (r.window.n > part->wmax) part->wmax = r.window.n;
@@ -289,6 +291,7 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   if (desc->n <= BF_MAX_TOOLS_ENUM) {
     build_tables(desc, &s->tables);
     split_and_window(s->tables, &s->plan, &s->window);
+    split_and_window_pruned(s->tables, &s->pplan, &s->pwindow);
   }
   cudaError_t e = cudaGetDevice(&s->device);
   if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_scratch), sizeof(bf_scratch));
@@ -501,7 +504,7 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
     if (h->fe[j] == 1 && h->ms[j] < bound) bound = h->ms[j];
 
   // 2. Keep the prefixes whose checkpoint bound does not exceed the incumbent.
-  bfk::Plan plan = make_plan(scn->plan, 0, total, kSearchTasks);
+  bfk::Plan plan = make_plan(scn->pplan, 0, total, kSearchTasks);
   plan.bound = bound;
   if (!scn->d_survivors) {
     e = lib_malloc(reinterpret_cast<void**>(&scn->d_survivors), sizeof(uint32_t) * plan.pow3P);
@@ -510,7 +513,7 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   e = cudaMemsetAsync(&dv->survivors, 0, sizeof(uint32_t), st);
   if (e == cudaSuccess) {
 #define CALL(NW) launch_prefix_filter_nw##NW(scn->tables, plan, scn->d_survivors, &dv->survivors, st)
-    BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
+    BF_DISPATCH(bfk::bucket_for(scn->pwindow.n), CALL)
 #undef CALL
   }
   if (e == cudaSuccess)
@@ -538,8 +541,8 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
     if (parts < 1) parts = 1;
     plan.m_chunk = (uint32_t)((num_m + parts - 1) / parts);
     plan.m_parts = (uint32_t)((num_m + plan.m_chunk - 1) / plan.m_chunk);
-#define CALL(NW) launch_pruned_search_nw##NW(scn->tables, scn->window, plan, scn->d_survivors, nsurv, scn->d_key, st)
-    BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
+#define CALL(NW) launch_pruned_search_nw##NW(scn->tables, scn->pwindow, plan, scn->d_survivors, nsurv, scn->d_key, st)
+    BF_DISPATCH(bfk::bucket_for(scn->pwindow.n), CALL)
 #undef CALL
   }
   if (e == cudaSuccess)
@@ -682,7 +685,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
       std::memset(&r, 0, sizeof r);
       build_tables(descs + i0 + j, &r.full);
       bfk::Plan plan;
-      split_and_window(r.full, &plan, &r.window);
+      split_and_window_batch(r.full, &plan, &r.window);
       r.plan = batch_plan(plan, descs[i0 + j].n);
       r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
       if (r.window.n > wmax) wmax = r.window.n;

@@ -35,12 +35,14 @@ struct bf_scenario {
   bfk::Tables tables;   // all n tools (n <= BF_MAX_TOOLS_ENUM; zero otherwise)
   bfk::Tables window;   // tools [W0, n), renumbered from 0
   bfk::Plan plan;       // enumeration split and window (see bfk::Plan), full range
+  bfk::Tables pwindow;  // bf_search_pruned: its window (of pplan)
+  bfk::Plan pplan;      // bf_search_pruned: its split (shorter prefixes: fewer to filter)
   int device;
   bf_scratch* d_scratch;      // device scratch
   bf_scratch* h_scratch;      // pinned host mirror
   unsigned long long* d_key;  // &d_scratch->key
   unsigned long long* h_key;  // &h_scratch->key
-  uint32_t* d_survivors;      // pruned search: 3^P prefix slots, allocated on first use
+  uint32_t* d_survivors;      // pruned search: 3^pplan.P prefix slots, allocated on first use
   uint32_t* d_levels;         // tree search: node buffers of every level, allocated on first use
   size_t levels_bytes;
 };

@@ -55,8 +55,9 @@ inline void build_tables(const bf_scenario_desc* d, bfk::TablesT<CAP>* t) {
   t->fmagic[0] = 1ull << 54;
 }
 
-// Number of mid tools M (their modes vary across a warp's lanes): large
-// enough to keep 32 lanes busy, small enough to leave many prefixes (warps).
+// Number of mid tools M when a warp's lanes take mid combinations under one
+// prefix (the batch kernel's whole-DAG windows): large enough to keep 32
+// lanes busy, small enough to leave many prefixes (warps).
 inline uint32_t mid_tools(uint32_t n) {
   if (n >= 13) return 6;   // 729 combinations: 23 rounds of 32 lanes, 1% idle
   if (n >= 9) return 5;    // 243 combinations
@@ -116,31 +117,35 @@ inline void retired_estimate(const TB& t, uint32_t* R) {
   R[n] = n;
 }
 
-// Choose P, M, I and the window start W0 for a scenario, and fill the window
-// tables (tools [W0, n) renumbered from 0).
-inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
-  const uint32_t n = t.n;
-  uint32_t anc[BF_MAX_TOOLS];
-  for (uint32_t v = 0; v < n; ++v) {
+// Ancestor masks of every tool (anc[v] = all tools with a path to v).
+template <typename TB>
+inline void ancestors(const TB& t, uint32_t* anc) {
+  for (uint32_t v = 0; v < t.n; ++v) {
     anc[v] = t.pred[v];
     for (uint32_t u = 0; u < v; ++u)
       if (t.pred[v] & (1u << u)) anc[v] |= anc[u];
   }
-  const uint32_t M = mid_tools(n);
+}
+
+// The plan for M mid tools: the inner level I, P = n - M - I prefix tools,
+// the window start W0, the pruning tails and the lone last tool's durations;
+// the window tables (tools [W0, n) renumbered from 0) are filled too.  anc:
+// ancestor masks; R: retired_estimate.
+inline void plan_for(const bfk::Tables& t, const uint32_t* anc, const uint32_t* R, uint32_t M, bfk::Plan* pl,
+                     bfk::Tables* w) {
+  const uint32_t n = t.n;
   // The inner level: the last I tools, whose modes each lane runs from a
   // second snapshot taken when the first of them can become ready; it pays
-  // when that snapshot comes after most of the events.  With R estimated
-  // below:
-  //  - the last tool waits for every other tool (R[n-1] = n-1): I = 1, and
-  //    the kernels end that tool in closed form;
+  // when that snapshot comes after most of the events.  With R:
+  //  - every other tool has ended when the last one can start (R[n-1] =
+  //    n-1): I = 1, and the kernels end the last tool in closed form
+  //    whenever it runs alone;
   //  - the snapshot would settle fewer than 2 tools: no inner level;
   //  - otherwise I = 1, or 2 when the earlier snapshot of two inner tools
   //    settles as many tools and keeps the same window, which shares the
   //    events before it among 9 mappings instead of 3.
   // Full search of the 16-tool layered workload: I = 2 3.4 ms, I = 1
   // 5.6 ms, I = 0 11.9 ms.
-  uint32_t R[BF_MAX_TOOLS + 1];
-  retired_estimate(t, R);
   uint32_t I = 0;
   if (n >= M + 1) {
     if (R[n - 1] + 1u == n) {
@@ -209,14 +214,57 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
   }
 }
 
-// Ancestor masks of every tool (anc[v] = all tools with a path to v).
-template <typename TB>
-inline void ancestors(const TB& t, uint32_t* anc) {
-  for (uint32_t v = 0; v < t.n; ++v) {
-    anc[v] = t.pred[v];
-    for (uint32_t u = 0; u < v; ++u)
-      if (t.pred[v] & (1u << u)) anc[v] |= anc[u];
+// Plan of a scenario for the kernels whose lanes own prefixes (searches,
+// evaluation, branch and bound).  M = 4 mid tools: a longer prefix settles
+// more of the DAG in each lane's own simulation and often starts the window
+// later (fewer slots per event).  When the last tool waits for every other
+// one (it then ends in closed form and a mapping costs little beyond its mid
+// run), M = 5 if that keeps the window and still leaves P >= 12 prefix tools
+// (3^12 prefixes, many warps per SM): the prefix simulation, which is as long
+// as the prefix, is shared by 3x more mappings.  Full searches, ms
+// (M = 6 / 5 / 4): 19-tool fan-out DAG 17.28 / 16.99 / 17.32; random
+// 20-tool DAG 412 / 416 / 362; layered 17 and 18 tools 14.8 / 14.9 / 13.5
+// and 49.3 / 49.9 / 42.0; segmented 17, 18 and 20 tools 3.66 / 3.78 / 2.98,
+// 3.43 / 2.49 / 1.69 and 14.1 / 10.8 / 10.8; 16-tool layered 3.40 / 3.51 /
+// 3.32.
+inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
+  const uint32_t n = t.n;
+  uint32_t anc[BF_MAX_TOOLS], R[BF_MAX_TOOLS + 1];
+  ancestors(t, anc);
+  retired_estimate(t, R);
+  plan_for(t, anc, R, n < 4 ? n : 4, pl, w);
+  const uint32_t others = n >= 2 ? (1u << (n - 1)) - 1u : 0u;
+  if (n >= 18 && pl->I == 1 && anc[n - 1] == others) {
+    bfk::Plan p5;
+    bfk::Tables w5;
+    plan_for(t, anc, R, 5, &p5, &w5);
+    if (p5.W0 == pl->W0 && p5.I == 1) {
+      *pl = p5;
+      *w = w5;
+    }
   }
+}
+
+// Plan of one scenario of a batch.  A window that is the whole DAG (W0 = 0)
+// runs with lanes taking mid combinations under a shared prefix, which wants
+// mid_tools(n) mid tools to fill the lanes (4096 layered 10-tool DAGs: M = 5
+// 38.2 ms, M = 4 41.1 ms); other scenarios take the search plan.
+inline void split_and_window_batch(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
+  uint32_t anc[BF_MAX_TOOLS], R[BF_MAX_TOOLS + 1];
+  ancestors(t, anc);
+  retired_estimate(t, R);
+  plan_for(t, anc, R, mid_tools(t.n), pl, w);
+  if (pl->W0 != 0u) split_and_window(t, pl, w);
+}
+
+// Plan of bf_search_pruned: mid_tools(n) mid tools, so that fewer, shorter
+// prefixes go through its prefix filter (19-tool fan-out DAG: 0.26 ms with
+// 3^12 prefixes, 0.52 ms with 3^13).
+inline void split_and_window_pruned(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
+  uint32_t anc[BF_MAX_TOOLS], R[BF_MAX_TOOLS + 1];
+  ancestors(t, anc);
+  retired_estimate(t, R);
+  plan_for(t, anc, R, mid_tools(t.n), pl, w);
 }
 
 // Lowest tool not certainly done when the first tool of [from, n) becomes ready.
