@@ -162,18 +162,16 @@ void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* 
   }
 }
 
-#define BF_DISPATCH(NT_VAL, CALL)                         \
-  switch (NT_VAL) {                                       \
-    case 4: { e = bfk::CALL(4); } break;                  \
-    case 6: { e = bfk::CALL(6); } break;                  \
-    case 8: { e = bfk::CALL(8); } break;                  \
-    case 10: { e = bfk::CALL(10); } break;                \
-    case 12: { e = bfk::CALL(12); } break;                \
-    case 14: { e = bfk::CALL(14); } break;                \
-    case 16: { e = bfk::CALL(16); } break;                \
-    case 18: { e = bfk::CALL(18); } break;                \
-    case 19: { e = bfk::CALL(19); } break;                \
-    default: { e = bfk::CALL(20); } break;                \
+// One case per compiled window width (BF_FOR_EACH_BUCKET); CALL(NW) is a
+// macro defined at the use site.  Every bucket_for value has a case.
+#define BF_DISPATCH_CASE(NW) \
+  case NW: {                 \
+    e = bfk::CALL(NW);       \
+  } break;
+#define BF_DISPATCH(NT_VAL, CALL)                  \
+  switch (NT_VAL) {                                \
+    BF_FOR_EACH_BUCKET(BF_DISPATCH_CASE)           \
+    default: { e = cudaErrorInvalidValue; } break; \
   }
 
 // Plan of one scenario of a batch (one block of kThreads / 32 warps each): a

@@ -39,7 +39,7 @@ __device__ __forceinline__ bool prefix_checkpoint(const TBF& tb, const SmemTable
   const uint32_t later = tb.all_mask & ~((1u << plan.P) - 1u);
   if (run<NP>(s, tb, sd, rt, *dgp, later) != kRunStopped) return false;
   *T_check = s.T;
-  if (slotA) save_prefix_window<NP, NW>(s, plan.W0, tb.n - plan.W0, slotA, stride);
+  if (slotA) save_prefix_window<NP, NW>(s, plan.W0, tb.n - plan.W0 - plan.last_apart, slotA, stride);
   return true;
 }
 
@@ -89,12 +89,14 @@ __device__ __forceinline__ void prefix_task(const TBF& tb, const SmemTables& sd,
       sink((uint32_t)base, r == kRunFinished ? w.T : kInfeasible);
       continue;
     }
-    if (r != kRunStopped) {  // infeasible before any inner tool started
+    // The run stops when an inner tool would become ready; with the last tool
+    // apart (the window lacks it) it ends when every other tool has ended.
+    if (r != (plan.last_apart ? kRunFinished : kRunStopped)) {  // infeasible before that
       for (uint32_t i = i_lo; i <= i_hi; ++i) sink((uint32_t)(base + stride_i * i), kInfeasible);
       continue;
     }
     if ((uint64_t)w.T + plan.tail_q > plan.bound) continue;  // pruned at the inner checkpoint
-    if (plan.I == 1u && (w.done | inner_mask) == 0xFFFFFFFFu) {
+    if (plan.last_apart || (plan.I == 1u && (w.done | inner_mask) == 0xFFFFFFFFu)) {
       // Everything but the last tool has ended: it runs alone from w.T.
       for (uint32_t i = i_lo; i <= i_hi; ++i) {
         const uint32_t d = plan.alone[i];
@@ -173,11 +175,11 @@ __device__ __forceinline__ void mid_lane_task(const TBF& tb, const SmemTables& s
       sink((uint32_t)base, r == kRunFinished ? w.T : kInfeasible);
       continue;
     }
-    if (r != kRunStopped) {
+    if (r != (plan.last_apart ? kRunFinished : kRunStopped)) {
       for (uint32_t i = 0; i < plan.pow3I; ++i) sink((uint32_t)(base + stride_i * i), kInfeasible);
       continue;
     }
-    if (plan.I == 1u && (w.done | inner_mask) == 0xFFFFFFFFu) {  // the last tool runs alone
+    if (plan.last_apart || (plan.I == 1u && (w.done | inner_mask) == 0xFFFFFFFFu)) {  // the last tool runs alone
       for (uint32_t i = 0; i < plan.pow3I; ++i) {
         const uint32_t d = plan.alone[i];
         sink((uint32_t)(base + stride_i * i), d == kInfeasible ? kInfeasible : w.T + d);

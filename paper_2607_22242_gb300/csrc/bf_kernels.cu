@@ -103,9 +103,9 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) eval_kernel(const __g
 // warps/SM instead of 24), for the 8-slot window, where that measured 3 %
 // faster; the common shape elsewhere (wider windows spill at that register
 // count).
-constexpr int kSearchThreads = BF_NW == 8 ? 128 : kThreads;
+constexpr int kSearchThreads = (BF_NW == 7 || BF_NW == 8) ? 128 : kThreads;
 constexpr int kSearchWarps = kSearchThreads / 32;
-constexpr int kSearchMinBlocks = BF_NW == 8 ? 7 : BF_MIN_BLOCKS;
+constexpr int kSearchMinBlocks = (BF_NW == 7 || BF_NW == 8) ? 7 : BF_MIN_BLOCKS;
 constexpr size_t kSearchSmemBytes = sizeof(uint32_t) * 2 * kLaneWords * kSearchThreads;
 
 template <int NP>

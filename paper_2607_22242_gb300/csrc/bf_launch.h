@@ -38,17 +38,6 @@ struct BatchRecord {
   uint32_t mid_lanes;
 };
 
-// Window-width buckets: kernels are compiled for NW in this list; a plan whose
-// window has w tools runs the smallest NW >= w (slots w..NW-1 count as done).
-#define BF_FOR_EACH_BUCKET(X) X(4) X(6) X(8) X(10) X(12) X(14) X(16) X(18) X(19) X(20)
-
-inline int bucket_for(uint32_t w) {
-  const int b[] = {4, 6, 8, 10, 12, 14, 16, 18, 19, 20};
-  for (int v : b)
-    if ((int)w <= v) return v;
-  return -1;
-}
-
 #define BF_DECLARE_BUCKET(NW)                                                                       \
   cudaError_t launch_eval_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan, uint32_t* ms, \
                                  uint8_t* fe, cudaStream_t st);                                     \

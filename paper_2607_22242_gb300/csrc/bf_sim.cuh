@@ -109,7 +109,24 @@ struct Plan {
   // the model's one remaining event ends it exactly this long after it is
   // ready.
   uint32_t alone[3];
+  // 1 when the last tool waits for every other tool (then I = 1) and leaving
+  // it out narrows the window to a smaller compiled width: the window holds
+  // tools [W0, n-1), its run ends when they have all ended -- the instant the
+  // last tool becomes ready -- and the last tool then runs alone, ending
+  // alone[a] later in mode a.
+  uint32_t last_apart;
 };
+
+// Window-width buckets: kernels are compiled for NW in this list; a plan whose
+// window has w tools runs the smallest NW >= w (slots w..NW-1 count as done).
+#define BF_FOR_EACH_BUCKET(X) X(4) X(6) X(7) X(8) X(10) X(12) X(14) X(16) X(18) X(19) X(20)
+
+inline int bucket_for(uint32_t w) {
+  const int b[] = {4, 6, 7, 8, 10, 12, 14, 16, 18, 19, 20};
+  for (int v : b)
+    if ((int)w <= v) return v;
+  return -1;
+}
 
 // Tables read with a per-thread (dynamic) index, staged in shared memory:
 // the per-k slowdown constants and the predecessor masks.
