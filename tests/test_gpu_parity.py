@@ -337,7 +337,7 @@ def test_concurrent_handles_on_host_threads(golden):
 
 
 def test_wait_timeout_is_reported():
-    """The host wait is bounded: a 1 ms limit on a ~0.1 s search returns BF_ETIMEOUT, the GPU
+    """The host wait is bounded: a 1 ms limit on a 16 ms search returns BF_ETIMEOUT, the GPU
     work finishes normally, and the library works afterwards."""
     import torch
     scn = S.config3()
