@@ -490,35 +490,33 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
     h->idx[nc++] = que;
     h->idx[nc++] = fast;
   }
-  e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess) e = launch_list(scn, dv->idx, nc, dv->ms, dv->fe, 1, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(h->ms, dv->ms, sizeof(uint32_t) * nc, cudaMemcpyDeviceToHost, st);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(h->fe, dv->fe, nc, cudaMemcpyDeviceToHost, st);
-  if (e != cudaSuccess) return cuda_fail(e, who);
-  int rc = wait_stream(st, who);
-  if (rc != BF_OK) return rc;
-  uint32_t bound = 0xFFFFFFFFu;
-  for (uint32_t j = 0; j < nc; ++j)
-    if (h->fe[j] == 1 && h->ms[j] < bound) bound = h->ms[j];
-
-  // 2. Keep the prefixes whose checkpoint bound does not exceed the incumbent.
-  bfk::Plan plan = make_plan(scn->pplan, 0, total, kSearchTasks);
-  plan.bound = bound;
   if (!scn->d_survivors) {
-    e = lib_malloc(reinterpret_cast<void**>(&scn->d_survivors), sizeof(uint32_t) * plan.pow3P);
+    e = lib_malloc(reinterpret_cast<void**>(&scn->d_survivors), sizeof(uint32_t) * scn->pplan.pow3P);
     if (e != cudaSuccess) return cuda_fail(e, who);
   }
-  e = cudaMemsetAsync(&dv->survivors, 0, sizeof(uint32_t), st);
+  e = cudaMemcpyAsync(dv->idx, h->idx, sizeof(uint64_t) * nc, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess) e = launch_list(scn, dv->idx, nc, dv->ms, dv->fe, 1, st);
+
+  // 2. Keep the prefixes whose checkpoint bound does not exceed the incumbent;
+  //    the filter kernel takes the incumbent from the list kernel's output and
+  //    hands it back with the survivor count (one host round trip for both).
+  bfk::Plan plan = make_plan(scn->pplan, 0, total, kSearchTasks);
+  if (e == cudaSuccess) e = cudaMemsetAsync(&dv->survivors, 0, sizeof(uint32_t), st);
   if (e == cudaSuccess) {
-#define CALL(NW) launch_prefix_filter_nw##NW(scn->tables, plan, scn->d_survivors, &dv->survivors, st)
+#define CALL(NW)                                                                                          \
+  launch_prefix_filter_nw##NW(scn->tables, plan, dv->ms, dv->fe, nc, scn->d_survivors, &dv->survivors, \
+                              &dv->pruned_bound, st)
     BF_DISPATCH(bfk::bucket_for(scn->pwindow.n), CALL)
 #undef CALL
   }
+  static_assert(offsetof(bf_scratch, pruned_bound) == offsetof(bf_scratch, survivors) + sizeof(uint32_t),
+                "survivors and pruned_bound are copied together");
   if (e == cudaSuccess)
-    e = cudaMemcpyAsync(&h->survivors, &dv->survivors, sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
+    e = cudaMemcpyAsync(&h->survivors, &dv->survivors, 2 * sizeof(uint32_t), cudaMemcpyDeviceToHost, st);
   if (e != cudaSuccess) return cuda_fail(e, who);
-  rc = wait_stream(st, who);
+  int rc = wait_stream(st, who);
   if (rc != BF_OK) return rc;
+  plan.bound = h->pruned_bound;
   const uint32_t nsurv = h->survivors;
   // A weak prefix bound (no cut points in the DAG) keeps most prefixes; the
   // tree search, whose expansions bound every node with the forward

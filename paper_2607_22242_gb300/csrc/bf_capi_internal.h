@@ -18,7 +18,7 @@
 struct bf_scratch {
   unsigned long long key;
   uint32_t survivors;   // pruned search: number of surviving prefixes
-  uint32_t pad;
+  uint32_t pruned_bound;  // pruned search: the incumbent's makespan (set with survivors)
   bfk::BestRecord best;      // tree search: best (makespan, index) so far
   uint32_t bound;            // tree search: makespan bound for pruning
   uint32_t pad2;

@@ -206,23 +206,33 @@ __global__ void __launch_bounds__(kThreads) list_kernel(const __grid_constant__ 
 }
 
 // Pruned search, pass 1: one thread per prefix; keeps the prefixes whose
-// checkpoint time plus the tail bound does not exceed plan.bound.
+// checkpoint time plus the tail bound does not exceed the incumbent, the
+// lowest feasible makespan among the ncand candidates the list kernel scored
+// just before on the same stream (cand_ms / cand_fe).  Block 0's thread 0 also
+// stores that bound for the host, which reads it with the survivor count.
 template <int NP>
 __global__ void __launch_bounds__(kThreads) prefix_filter_kernel(const __grid_constant__ Tables tb,
                                                                  const __grid_constant__ Plan plan,
+                                                                 const uint32_t* __restrict__ cand_ms,
+                                                                 const uint8_t* __restrict__ cand_fe, uint32_t ncand,
                                                                  uint32_t* __restrict__ survivors,
-                                                                 uint32_t* __restrict__ count) {
+                                                                 uint32_t* __restrict__ count,
+                                                                 uint32_t* __restrict__ bound_out) {
   __shared__ SmemTables sd;
   __shared__ uint32_t rt[ReadyTable<NP>::size];
   load_smem_tables(tb, sd);
   fill_ready_table<NP>(tb, rt);
   __syncthreads();
+  uint32_t bound = kInfeasible;
+  for (uint32_t j = 0; j < ncand; ++j)
+    if (cand_fe[j] == 1u && cand_ms[j] < bound) bound = cand_ms[j];
+  if (blockIdx.x == 0 && threadIdx.x == 0) *bound_out = bound;
   const uint64_t p = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (p >= plan.pow3P) return;
   Digits dgp;
   uint32_t T = 0u;
   if (prefix_checkpoint<NP, BF_NW>(tb, sd, rt, plan, (uint32_t)p, &dgp, &T, nullptr, 0u) &&
-      (uint64_t)T + plan.tail_p <= plan.bound)
+      (uint64_t)T + plan.tail_p <= bound)
     survivors[atomicAdd(count, 1u)] = (uint32_t)p;
 }
 
@@ -298,13 +308,16 @@ cudaError_t BF_PASTE(launch_search_nw, BF_NW)(const Tables& tb, const Tables& tw
   return cudaGetLastError();
 }
 
-cudaError_t BF_PASTE(launch_prefix_filter_nw, BF_NW)(const Tables& tb, const Plan& plan, uint32_t* survivors,
-                                                     uint32_t* count, cudaStream_t st) {
+cudaError_t BF_PASTE(launch_prefix_filter_nw, BF_NW)(const Tables& tb, const Plan& plan, const uint32_t* cand_ms,
+                                                     const uint8_t* cand_fe, uint32_t ncand, uint32_t* survivors,
+                                                     uint32_t* count, uint32_t* bound_out, cudaStream_t st) {
   const unsigned grid = (unsigned)(((uint64_t)plan.pow3P + kThreads - 1) / kThreads);
   if (tb.n <= (uint32_t)BF_NW)
-    prefix_filter_kernel<BF_NW><<<grid, kThreads, 0, st>>>(tb, plan, survivors, count);
+    prefix_filter_kernel<BF_NW><<<grid, kThreads, 0, st>>>(tb, plan, cand_ms, cand_fe, ncand, survivors, count,
+                                                           bound_out);
   else
-    prefix_filter_kernel<kMaxTools><<<grid, kThreads, 0, st>>>(tb, plan, survivors, count);
+    prefix_filter_kernel<kMaxTools><<<grid, kThreads, 0, st>>>(tb, plan, cand_ms, cand_fe, ncand, survivors, count,
+                                                               bound_out);
   return cudaGetLastError();
 }
 

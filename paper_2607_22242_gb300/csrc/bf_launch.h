@@ -48,8 +48,9 @@ struct BatchRecord {
                                   unsigned long long* keys, cudaStream_t st);                        \
   cudaError_t launch_list_nw##NW(const Tables& tb, uint64_t total, const uint64_t* idx, uint64_t count, \
                                  uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st);             \
-  cudaError_t launch_prefix_filter_nw##NW(const Tables& tb, const Plan& plan, uint32_t* survivors,   \
-                                          uint32_t* count, cudaStream_t st);                         \
+  cudaError_t launch_prefix_filter_nw##NW(const Tables& tb, const Plan& plan, const uint32_t* cand_ms,   \
+                                          const uint8_t* cand_fe, uint32_t ncand, uint32_t* survivors,   \
+                                          uint32_t* count, uint32_t* bound_out, cudaStream_t st);        \
   cudaError_t launch_pruned_search_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan,       \
                                           const uint32_t* survivors, uint32_t nsurv,                 \
                                           unsigned long long* key, cudaStream_t st);
