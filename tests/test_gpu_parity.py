@@ -106,6 +106,36 @@ def test_every_bucket_edge(n):
         assert (r.index, r.makespan_us) == oracle.search(scn, THREADS)
 
 
+@pytest.mark.parametrize("n", [5, 6, 8, 9, 10, 12, 14])
+def test_last_tool_waiting_for_all(n):
+    """A last tool that every other tool precedes: the kernels leave it out of the window when
+    that narrows the compiled width, and end it in closed form.  Full space (n <= 12) or head,
+    tail and middle ranges element by element, ranges that cut the last tool's modes apart, and
+    the exhaustive and branch-and-bound searches, against the oracle."""
+    rng = np.random.default_rng(700 + n)
+    base = S.random_small(rng, n, edge_p=0.25, tight=bool(n % 2), max_time=60)
+    pred = list(base.pred_mask)
+    pred[n - 1] = (1 << (n - 1)) - 1
+    scn = S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
+                     base.vram_budget_mib, base.slowdown_q10)
+    total = 3 ** n
+    third = 3 ** (n - 1)
+    with bf.create_scenario(scn) as h:
+        if total <= 600_000:
+            assert_same(h, scn, 0, total)
+        else:
+            for first in (0, total // 2 - 77_777, total - 150_001):
+                assert_same(h, scn, first, 150_001)
+        for first, count in ((third - 5, 11), (2 * third - 1, 2), (third + 1, third - 2)):
+            if count <= 600_000:
+                assert_same(h, scn, first, count)
+        want = oracle.search(scn, THREADS)
+        r = bf.search_best(h)
+        assert (r.index, r.makespan_us) == want
+        rp = bf.search_pruned(h)
+        assert (rp.index, rp.makespan_us) == want
+
+
 def test_degenerate_budgets_all_paths():
     """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
     the batch, the branch and bound and the tree search, against the oracle."""
