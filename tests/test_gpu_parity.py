@@ -136,6 +136,32 @@ def test_last_tool_waiting_for_all(n):
         assert (rp.index, rp.makespan_us) == want
 
 
+@pytest.mark.parametrize("n", [8, 12])
+def test_magnitudes_at_the_validation_bounds(n):
+    """Durations near the validated limits: GPU work of almost 2^32 units per tool (the virtual
+    clock wraps modulo 2^32 about once per GPU tool), slowdowns up to 64x, CPU times of up to
+    a minute, makespans up to about 10^8 microseconds.  Every mapping element by element, and
+    every search path, against the oracle's 64-bit arithmetic."""
+    rng = np.random.default_rng(900 + n)
+    base = S.random_small(rng, n, edge_p=0.3, tight=True, max_time=50)
+    big = (1 << 22) - 1
+    g = [int(v) for v in rng.integers(big // 2, big // 2 + big // 4, n)]
+    x = [int(v) for v in rng.integers(0, big // 8, n)]
+    l = [int(v) for v in rng.integers(0, big // 8, n)]
+    c = [int(v) for v in rng.integers(1, 300_000_000 // n, n)]
+    f = [0, 1024] + [min(65536, 1024 + (65536 - 1024) * (k - 1) // (n - 1)) for k in range(2, 21)]
+    scn = S.Scenario(n, base.pred_mask, c, g, x, l, base.vram_mib, base.vram_budget_mib, f)
+    bf.validate_desc(scn)
+    with bf.create_scenario(scn) as h:
+        assert_same(h, scn, 0, 3 ** n)
+        want = oracle.search(scn, THREADS)
+        for res in (bf.search_best(h), bf.search_pruned(h), bf.search_tree(h, bf.SPACE_FULL, True)[0],
+                    bf.search_tree(h, bf.SPACE_FULL, False)[0]):
+            assert (res.index, res.makespan_us) == want
+        binary = bf.search_tree(h, bf.SPACE_BINARY, True)[0]
+        assert (binary.index, binary.makespan_us) == oracle.search_binary(scn, THREADS)
+
+
 def test_degenerate_budgets_all_paths():
     """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
     the batch, the branch and bound and the tree search, against the oracle."""
