@@ -26,6 +26,8 @@ using bfk::host::pow3;
 using bfk::host::split_and_window;
 using bfk::host::split_and_window_batch;
 using bfk::host::split_and_window_pruned;
+using bfk::host::relabel_sources_first;
+using bfk::host::renumbering_helps;
 
 // Warp tasks a single-scenario launch is split into (several waves of the
 // GPU's resident warps, so that uneven tasks even out).
@@ -177,6 +179,23 @@ void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* 
 // Plan of one scenario of a batch (one block of kThreads / 32 warps each): a
 // scenario with fewer prefix groups than warps splits its mid combinations
 // so that as many warps as possible share it.
+// Tables, split and window of one scenario of a batch (a whole-space search):
+// renumbered with the sources first when that gives a better split.
+void batch_split(const bf_scenario_desc* d, bfk::Tables* tb, bfk::Plan* plan, bfk::Tables* tw) {
+  bfk::Tables rt, rw;
+  bfk::Plan rp;
+  build_tables(d, tb);
+  split_and_window_batch(*tb, plan, tw);
+  if (relabel_sources_first(*tb, &rt)) {
+    split_and_window_batch(rt, &rp, &rw);
+    if (renumbering_helps(*tb, *plan, *tw, rt, rp, rw)) {
+      *tb = rt;
+      *plan = rp;
+      *tw = rw;
+    }
+  }
+}
+
 bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n) {
   constexpr uint32_t kWarps = bfk::kThreads / 32;
   const uint32_t groups = (base.pow3P + 31u) / 32u;
@@ -196,9 +215,8 @@ void build_records(const bf_scenario_desc* descs, uint32_t count, bfk::BatchReco
     for (uint32_t i = lo; i < hi; ++i) {
       bfk::BatchRecord& r = recs[i];
       std::memset(&r, 0, sizeof r);
-      build_tables(descs + i, &r.full);
       bfk::Plan base;
-      split_and_window_batch(r.full, &base, &r.window);
+      batch_split(descs + i, &r.full, &base, &r.window);
       r.plan = batch_plan(base, descs[i].n);
       r.mid_lanes = base.W0 == 0u ? 1u : 0u;
       if (r.window.n > part->wmax) part->wmax = r.window.n;
@@ -255,9 +273,14 @@ int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result
   cudaError_t e = cudaMemsetAsync(scn->d_key, 0xFF, sizeof(unsigned long long), st);
   if (e != cudaSuccess) return cuda_fail(e, who);
   if (count) {
-    const bfk::Plan plan = make_plan(scn->plan, first, count, kSearchTasks);
-#define CALL(NW) launch_search_nw##NW(scn->tables, scn->window, plan, scn->d_key, st)
-    BF_DISPATCH(bfk::bucket_for(scn->window.n), CALL)
+    // The whole space runs on the renumbered tables; a part of it keeps the
+    // scenario's numbering, in which an index range is a box of the split.
+    const bool whole = first == 0 && count == pow3(scn->desc.n);
+    const bfk::Tables& tb = whole ? scn->rtables : scn->tables;
+    const bfk::Tables& tw = whole ? scn->rwindow : scn->window;
+    const bfk::Plan plan = make_plan(whole ? scn->rplan : scn->plan, first, count, kSearchTasks);
+#define CALL(NW) launch_search_nw##NW(tb, tw, plan, scn->d_key, st)
+    BF_DISPATCH(bfk::bucket_for(tw.n), CALL)
 #undef CALL
     if (e != cudaSuccess) return cuda_fail(e, who);
   }
@@ -289,7 +312,14 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   if (desc->n <= BF_MAX_TOOLS_ENUM) {
     build_tables(desc, &s->tables);
     split_and_window(s->tables, &s->plan, &s->window);
-    split_and_window_pruned(s->tables, &s->pplan, &s->pwindow);
+    if (relabel_sources_first(s->tables, &s->rtables)) split_and_window(s->rtables, &s->rplan, &s->rwindow);
+    if (!s->rtables.relabeled ||
+        !renumbering_helps(s->tables, s->plan, s->window, s->rtables, s->rplan, s->rwindow)) {
+      s->rtables = s->tables;
+      s->rplan = s->plan;
+      s->rwindow = s->window;
+    }
+    split_and_window_pruned(s->rtables, &s->pplan, &s->pwindow);
   }
   cudaError_t e = cudaGetDevice(&s->device);
   if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_scratch), sizeof(bf_scratch));
@@ -504,7 +534,7 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   if (e == cudaSuccess) e = cudaMemsetAsync(&dv->survivors, 0, sizeof(uint32_t), st);
   if (e == cudaSuccess) {
 #define CALL(NW)                                                                                          \
-  launch_prefix_filter_nw##NW(scn->tables, plan, dv->ms, dv->fe, nc, scn->d_survivors, &dv->survivors, \
+  launch_prefix_filter_nw##NW(scn->rtables, plan, dv->ms, dv->fe, nc, scn->d_survivors, &dv->survivors, \
                               &dv->pruned_bound, st)
     BF_DISPATCH(bfk::bucket_for(scn->pwindow.n), CALL)
 #undef CALL
@@ -537,7 +567,7 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
     if (parts < 1) parts = 1;
     plan.m_chunk = (uint32_t)((num_m + parts - 1) / parts);
     plan.m_parts = (uint32_t)((num_m + plan.m_chunk - 1) / plan.m_chunk);
-#define CALL(NW) launch_pruned_search_nw##NW(scn->tables, scn->pwindow, plan, scn->d_survivors, nsurv, scn->d_key, st)
+#define CALL(NW) launch_pruned_search_nw##NW(scn->rtables, scn->pwindow, plan, scn->d_survivors, nsurv, scn->d_key, st)
     BF_DISPATCH(bfk::bucket_for(scn->pwindow.n), CALL)
 #undef CALL
   }
@@ -679,9 +709,8 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
     for (uint32_t j = 0; j < nrec; ++j) {
       bfk::BatchRecord& r = chunk[j];
       std::memset(&r, 0, sizeof r);
-      build_tables(descs + i0 + j, &r.full);
       bfk::Plan plan;
-      split_and_window_batch(r.full, &plan, &r.window);
+      batch_split(descs + i0 + j, &r.full, &plan, &r.window);
       r.plan = batch_plan(plan, descs[i0 + j].n);
       r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
       if (r.window.n > wmax) wmax = r.window.n;

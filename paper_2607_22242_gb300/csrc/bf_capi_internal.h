@@ -35,7 +35,13 @@ struct bf_scenario {
   bfk::Tables tables;   // all n tools (n <= BF_MAX_TOOLS_ENUM; zero otherwise)
   bfk::Tables window;   // tools [W0, n), renumbered from 0
   bfk::Plan plan;       // enumeration split and window (see bfk::Plan), full range
-  bfk::Tables pwindow;  // bf_search_pruned: its window (of pplan)
+  // Searches of the whole space: the tools renumbered with the sources first
+  // (bf_plan.h relabel_sources_first; equal to the above when that order is
+  // the scenario's own), with their split and window.
+  bfk::Tables rtables;
+  bfk::Tables rwindow;
+  bfk::Plan rplan;
+  bfk::Tables pwindow;  // bf_search_pruned: its window (of pplan, on rtables)
   bfk::Plan pplan;      // bf_search_pruned: its split (shorter prefixes: fewer to filter)
   int device;
   bf_scratch* d_scratch;      // device scratch

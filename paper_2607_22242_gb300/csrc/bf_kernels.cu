@@ -75,8 +75,13 @@ __device__ __forceinline__ void block_min_to(unsigned long long v, unsigned long
 // the prefix checkpoint, and a second one for the inner checkpoint when the
 // plan has an inner level; [word][thread] layout.
 constexpr int kLaneWords = LaneWords<BF_NW>::value;
+// Dynamic shared memory: the mid-part table (mid_part_words(3^M) words; the
+// batch kernel reserves the largest) followed by the lane states.
 constexpr size_t kDynSmemBytes = sizeof(uint32_t) * 2 * kLaneWords * kThreads;
-inline size_t dyn_smem_bytes(uint32_t inner_levels) { return inner_levels ? kDynSmemBytes : kDynSmemBytes / 2; }
+constexpr size_t kDynSmemMaxBytes = sizeof(uint32_t) * kMaxMidPartWords + kDynSmemBytes;
+inline size_t dyn_smem_bytes(uint32_t inner_levels, uint32_t mid_words) {
+  return sizeof(uint32_t) * mid_words + (inner_levels ? kDynSmemBytes : kDynSmemBytes / 2);
+}
 
 template <int NP>
 __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) eval_kernel(const __grid_constant__ Tables tb,
@@ -95,7 +100,8 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) eval_kernel(const __g
   const uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5);
   if (task >= plan.groups * plan.m_parts) return;  // no block-level synchronisation follows
   StoreSink sink{plan.first, ms_out, fe_out};
-  warp_task<NP, BF_NW>(tb, sd, rt, tw, sdw, rtw, plan, task / plan.m_parts, task % plan.m_parts,
+  // Index ranges are always in the scenario's numbering.
+  warp_task<NP, BF_NW, false>(tb, sd, rt, tw, sdw, rtw, plan, nullptr, task / plan.m_parts, task % plan.m_parts,
                        lane_state + threadIdx.x, lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
 }
 
@@ -107,24 +113,30 @@ constexpr int kSearchThreads = (BF_NW == 7 || BF_NW == 8) ? 128 : kThreads;
 constexpr int kSearchWarps = kSearchThreads / 32;
 constexpr int kSearchMinBlocks = (BF_NW == 7 || BF_NW == 8) ? 7 : BF_MIN_BLOCKS;
 constexpr size_t kSearchSmemBytes = sizeof(uint32_t) * 2 * kLaneWords * kSearchThreads;
+constexpr size_t kSearchSmemMaxBytes = sizeof(uint32_t) * kMaxMidPartWords + kSearchSmemBytes;
 
-template <int NP>
+// RL: renumbered tables (whole-space searches, Plan::relabeled); the mid-part
+// table then precedes the lane states in dynamic shared memory.
+template <int NP, bool RL>
 __global__ void __launch_bounds__(kSearchThreads, kSearchMinBlocks) search_kernel(const __grid_constant__ Tables tb,
                                                                                   const __grid_constant__ Tables tw,
                                                                                   const __grid_constant__ Plan plan,
                                                                                   unsigned long long* key) {
-  extern __shared__ uint32_t lane_state[];
+  extern __shared__ uint32_t dyn_smem[];
+  uint32_t* const mpart = dyn_smem;
+  uint32_t* const lane_state = dyn_smem + (RL ? mid_part_words(plan.pow3M) : 0u);
   __shared__ SmemTables sd, sdw;
   __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
   fill_ready_table<NP>(tb, rt);
   fill_ready_table<BF_NW>(tw, rtw);
+  if constexpr (RL) fill_mid_parts(plan, mpart);
   __syncthreads();
   const uint32_t task = blockIdx.x * kSearchWarps + (threadIdx.x >> 5);
   MinKeySink sink;
   if (task < plan.groups * plan.m_parts)
-    warp_task<NP, BF_NW>(tb, sd, rt, tw, sdw, rtw, plan, task / plan.m_parts, task % plan.m_parts,
+    warp_task<NP, BF_NW, RL>(tb, sd, rt, tw, sdw, rtw, plan, mpart, task / plan.m_parts, task % plan.m_parts,
                          lane_state + threadIdx.x, lane_state + kLaneWords * kSearchThreads + threadIdx.x,
                          kSearchThreads, sink);
   block_min_to<kSearchWarps>(sink.best, key);
@@ -135,7 +147,9 @@ template <int NP>
 __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(const BatchRecord* __restrict__ recs,
                                                                               uint32_t blocks_per_scenario,
                                                                               unsigned long long* keys) {
-  extern __shared__ uint32_t lane_state[];
+  extern __shared__ uint32_t dyn_smem[];  // mid-part table (3^6 entries at most), then the lane states
+  uint32_t* const mpart = dyn_smem;
+  uint32_t* const lane_state = dyn_smem + kMaxMidPartWords;
   __shared__ BatchRecord rec;
   __shared__ SmemTables sd, sdw;
   __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
@@ -151,6 +165,7 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
   load_smem_tables(rec.window, sdw);
   fill_ready_table<NP>(rec.full, rt);
   fill_ready_table<BF_NW>(rec.window, rtw);
+  fill_mid_parts(rec.plan, mpart);
   __syncthreads();
   const uint32_t warp = b * kWarps + (threadIdx.x >> 5);
   MinKeySink sink;
@@ -161,14 +176,15 @@ __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(co
     // spills at 2 blocks/SM; 2.5 % faster on 4096 layered 10-tool DAGs).
     for (uint32_t p = warp; p < rec.plan.pow3P; p += blocks_per_scenario * kWarps) {
       if constexpr (NP == BF_NW)
-        mid_lane_task<NP, BF_NW>(rec.full, sd, rt, rec.full, sd, rt, rec.plan, p, lane_state + threadIdx.x,
+        mid_lane_task<NP, BF_NW>(rec.full, sd, rt, rec.full, sd, rt, rec.plan, mpart, p, lane_state + threadIdx.x,
                                  lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
       else
-        mid_lane_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, p, lane_state + threadIdx.x,
+        mid_lane_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, mpart, p,
+                                 lane_state + threadIdx.x,
                                  lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
     }
   } else if (warp < rec.plan.groups * rec.plan.m_parts) {
-    warp_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, warp / rec.plan.m_parts,
+    warp_task<NP, BF_NW, true>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, mpart, warp / rec.plan.m_parts,
                          warp % rec.plan.m_parts, lane_state + threadIdx.x,
                          lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
   }
@@ -241,20 +257,23 @@ template <int NP>
 __global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS) pruned_search_kernel(
     const __grid_constant__ Tables tb, const __grid_constant__ Tables tw, const __grid_constant__ Plan plan,
     const uint32_t* __restrict__ survivors, uint32_t nsurv, unsigned long long* key) {
-  extern __shared__ uint32_t lane_state[];
+  extern __shared__ uint32_t dyn_smem[];  // mid-part table, then the lane states
+  uint32_t* const mpart = dyn_smem;
+  uint32_t* const lane_state = dyn_smem + mid_part_words(plan.pow3M);
   __shared__ SmemTables sd, sdw;
   __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
   load_smem_tables(tb, sd);
   load_smem_tables(tw, sdw);
   fill_ready_table<NP>(tb, rt);
   fill_ready_table<BF_NW>(tw, rtw);
+  fill_mid_parts(plan, mpart);
   __syncthreads();
   const uint32_t task = blockIdx.x * kWarps + (threadIdx.x >> 5);
   MinKeySink sink;
   if (task < plan.groups * plan.m_parts) {
     const uint32_t slot = (task / plan.m_parts) * 32u + (threadIdx.x & 31u);
     const bool valid = slot < nsurv;
-    prefix_task<NP, BF_NW>(tb, sd, rt, tw, sdw, rtw, plan, valid ? survivors[slot] : 0u, valid,
+    prefix_task<NP, BF_NW, true>(tb, sd, rt, tw, sdw, rtw, plan, mpart, valid ? survivors[slot] : 0u, valid,
                            task % plan.m_parts, lane_state + threadIdx.x,
                            lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
   }
@@ -272,13 +291,13 @@ static unsigned blocks_for(const Plan& plan) {
 }
 
 // Each launcher picks the prefix width (BF_NW when the scenario fits, else 20).
-#define BF_LAUNCH(KERNEL, FITS, INNER, GRID, ...)                                            \
-  do {                                                                                       \
-    static std::atomic<uint64_t> ready_narrow{0}, ready_wide{0};                           \
-    cudaError_t e_ = (FITS) ? allow_dyn_smem(KERNEL<BF_NW>, kDynSmemBytes, &ready_narrow)   \
-                            : allow_dyn_smem(KERNEL<kMaxTools>, kDynSmemBytes, &ready_wide); \
-    if (e_ != cudaSuccess) return e_;                                                        \
-    const size_t smem_ = dyn_smem_bytes(INNER);                                              \
+#define BF_LAUNCH(KERNEL, FITS, INNER, MIDW, GRID, ...)                                         \
+  do {                                                                                          \
+    static std::atomic<uint64_t> ready_narrow{0}, ready_wide{0};                              \
+    cudaError_t e_ = (FITS) ? allow_dyn_smem(KERNEL<BF_NW>, kDynSmemMaxBytes, &ready_narrow)   \
+                            : allow_dyn_smem(KERNEL<kMaxTools>, kDynSmemMaxBytes, &ready_wide); \
+    if (e_ != cudaSuccess) return e_;                                                           \
+    const size_t smem_ = dyn_smem_bytes(INNER, MIDW);                                           \
     if (FITS)                                                                                \
       KERNEL<BF_NW><<<(GRID), kThreads, smem_, st>>>(__VA_ARGS__);                           \
     else                                                                                     \
@@ -288,23 +307,22 @@ static unsigned blocks_for(const Plan& plan) {
 
 cudaError_t BF_PASTE(launch_eval_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                             uint32_t* ms, uint8_t* fe, cudaStream_t st) {
-  BF_LAUNCH(eval_kernel, tb.n <= (uint32_t)BF_NW, plan.I, blocks_for(plan), tb, tw, plan, ms, fe);
+  BF_LAUNCH(eval_kernel, tb.n <= (uint32_t)BF_NW, plan.I, 0u, blocks_for(plan), tb, tw, plan, ms, fe);
 }
 
 cudaError_t BF_PASTE(launch_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                               unsigned long long* key, cudaStream_t st) {
-  static std::atomic<uint64_t> ready_narrow{0}, ready_wide{0};
-  const bool fits = tb.n <= (uint32_t)BF_NW;
-  cudaError_t e = fits ? allow_dyn_smem(search_kernel<BF_NW>, kSearchSmemBytes, &ready_narrow)
-                       : allow_dyn_smem(search_kernel<kMaxTools>, kSearchSmemBytes, &ready_wide);
+  static std::atomic<uint64_t> ready[4] = {};
+  const bool fits = tb.n <= (uint32_t)BF_NW, rl = plan.relabeled != 0u;
+  auto kernel = fits ? (rl ? search_kernel<BF_NW, true> : search_kernel<BF_NW, false>)
+                     : (rl ? search_kernel<kMaxTools, true> : search_kernel<kMaxTools, false>);
+  cudaError_t e = allow_dyn_smem(kernel, kSearchSmemMaxBytes, &ready[(fits ? 2 : 0) + (rl ? 1 : 0)]);
   if (e != cudaSuccess) return e;
-  const size_t smem = plan.I ? kSearchSmemBytes : kSearchSmemBytes / 2;
+  const size_t smem = sizeof(uint32_t) * (rl ? mid_part_words(plan.pow3M) : 0u) +
+                      (plan.I ? kSearchSmemBytes : kSearchSmemBytes / 2);
   const uint64_t tasks = (uint64_t)plan.groups * plan.m_parts;
   const unsigned grid = (unsigned)((tasks + kSearchWarps - 1) / kSearchWarps);
-  if (fits)
-    search_kernel<BF_NW><<<grid, kSearchThreads, smem, st>>>(tb, tw, plan, key);
-  else
-    search_kernel<kMaxTools><<<grid, kSearchThreads, smem, st>>>(tb, tw, plan, key);
+  kernel<<<grid, kSearchThreads, smem, st>>>(tb, tw, plan, key);
   return cudaGetLastError();
 }
 
@@ -324,8 +342,8 @@ cudaError_t BF_PASTE(launch_prefix_filter_nw, BF_NW)(const Tables& tb, const Pla
 cudaError_t BF_PASTE(launch_pruned_search_nw, BF_NW)(const Tables& tb, const Tables& tw, const Plan& plan,
                                                      const uint32_t* survivors, uint32_t nsurv,
                                                      unsigned long long* key, cudaStream_t st) {
-  BF_LAUNCH(pruned_search_kernel, tb.n <= (uint32_t)BF_NW, plan.I, blocks_for(plan), tb, tw, plan, survivors, nsurv,
-            key);
+  BF_LAUNCH(pruned_search_kernel, tb.n <= (uint32_t)BF_NW, plan.I, mid_part_words(plan.pow3M), blocks_for(plan), tb,
+            tw, plan, survivors, nsurv, key);
 }
 
 // Index lists run the whole scenario in one simulation: this unit handles n <= BF_NW.
@@ -339,7 +357,8 @@ cudaError_t BF_PASTE(launch_batch_nw, BF_NW)(const BatchRecord* d_recs, uint32_t
                                              uint32_t any_inner, uint32_t blocks_per_scenario,
                                              unsigned long long* keys, cudaStream_t st) {
   const unsigned blocks = (unsigned)((uint64_t)count * blocks_per_scenario);
-  BF_LAUNCH(batch_kernel, nmax <= (uint32_t)BF_NW, any_inner, blocks, d_recs, blocks_per_scenario, keys);
+  BF_LAUNCH(batch_kernel, nmax <= (uint32_t)BF_NW, any_inner, kMaxMidPartWords, blocks, d_recs, blocks_per_scenario,
+            keys);
 }
 
 }  // namespace bfk

@@ -65,6 +65,11 @@ struct TablesT {
   uint32_t wnow[CAP];  // (g_i + x_i) * 1024
   uint32_t wq[CAP];    // (l_i + g_i + x_i) * 1024
   uint32_t vram[CAP];  // m_i
+  // Tool v of these tables is tool orig[v] of the scenario (host bookkeeping:
+  // the searches over the whole space may number the tools differently, see
+  // bf_plan.h relabel_sources_first; relabeled = 1 then).
+  uint32_t orig[CAP];
+  uint32_t relabeled;
   uint32_t f[CAP + 1];        // f[k]; f[0] unused
   uint32_t fshift[CAP + 1];   // l - 12
   uint64_t fmagic[CAP + 1];   // ceil(2^(52+l) / f[k])
@@ -115,6 +120,14 @@ struct Plan {
   // last tool becomes ready -- and the last tool then runs alone, ending
   // alone[a] later in mode a.
   uint32_t last_apart;
+  // A mapping's canonical index is the sum over tools v of its mode of v times
+  // pv[v] = 3^orig[v] (3^v unless the tables are relabeled, whole-space
+  // searches only): the prefix part, a mid part per mid combination (a table
+  // in shared memory) and the inner part d0 * pvA + d1 * pvB (pv of the first
+  // and second inner tools, 0 when absent).
+  uint32_t relabeled;
+  uint32_t pvA, pvB;
+  uint32_t pv[kMaxTools];
 };
 
 // Window-width buckets: kernels are compiled for NW in this list; a plan whose
