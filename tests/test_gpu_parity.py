@@ -162,6 +162,31 @@ def test_magnitudes_at_the_validation_bounds(n):
         assert (binary.index, binary.makespan_us) == oracle.search_binary(scn, THREADS)
 
 
+def test_late_sources_renumbered_searches():
+    """DAGs with sources late in the scenario's numbering, which the whole-space searches may
+    renumber (sources first), with small integer times so that queue ties are frequent: the
+    exhaustive search, the branch and bound and the batched search against the oracle."""
+    rng = np.random.default_rng(31)
+    scns = []
+    for t in range(160):
+        n = int(rng.integers(6, 13))
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.3, 0.5])), tight=bool(t % 2),
+                              contention=bool(t % 3), max_time=int(rng.choice([4, 9, 40])))
+        pred = list(base.pred_mask)
+        for v in rng.choice(np.arange(n // 2, n), size=2, replace=False):
+            pred[int(v)] = 0
+        scns.append(S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
+                               base.vram_budget_mib, base.slowdown_q10))
+    want = [oracle.search(scn, THREADS) for scn in scns]
+    for scn, w in zip(scns, want):
+        with bf.create_scenario(scn) as h:
+            r = bf.search_best(h)
+            assert (r.index, r.makespan_us) == w, scn
+            rp = bf.search_pruned(h)
+            assert (rp.index, rp.makespan_us) == w, scn
+    assert [(r.index, r.makespan_us) for r in bf.search_batch(scns)] == want
+
+
 def test_degenerate_budgets_all_paths():
     """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
     the batch, the branch and bound and the tree search, against the oracle."""
