@@ -19,7 +19,7 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(os.path.dirname(HERE), "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(BUILD_DIR, "libbf.so")
-BUCKETS = (4, 6, 7, 8, 10, 12, 14, 16, 18, 19, 20)  # window widths (bf_sim.cuh)
+BUCKETS = tuple(range(4, 21))  # window widths (bf_sim.cuh): one unit per width from 4 to 20
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden",
               f"-I{INCLUDE}"]

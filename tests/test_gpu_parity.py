@@ -89,7 +89,7 @@ def test_random_small_exhaustive(seed):
 
 @pytest.mark.parametrize("n", [1, 2, 9, 11, 13, 15, 17])
 def test_every_bucket_edge(n):
-    """Scenarios whose n sits at or just past a compiled bucket size, realistic magnitudes."""
+    """Scenarios of several sizes (windows across the compiled widths), realistic magnitudes."""
     rng = np.random.default_rng(50 + n)
     base = S.random_small(rng, n, edge_p=0.3, tight=True, max_time=50)
     scale = lambda v: [x * 997 + 1 for x in v]
