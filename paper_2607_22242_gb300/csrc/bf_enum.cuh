@@ -25,7 +25,8 @@ __device__ __forceinline__ bool inner_range(const Plan& plan, uint64_t base, uin
 }
 
 // Canonical index part of `count` tools from `first_tool` on, whose modes are
-// bits 0.. of d, for relabeled plans: sum of mode x 3^orig (plan.pv).
+// bits 0.. of d: the sum of mode x 3^orig (plan.pv; 3^v for tables in the
+// scenario's own numbering).
 __device__ __forceinline__ uint32_t index_part(const Plan& plan, Digits d, uint32_t first_tool, uint32_t count) {
   uint32_t x = 0u;
 #pragma unroll
