@@ -10,6 +10,7 @@ from __future__ import annotations
 
 import concurrent.futures as cf
 import hashlib
+import re
 import os
 import shutil
 import subprocess
@@ -52,13 +53,22 @@ def _fingerprint(extra) -> str:
 KERNEL_UNIT = ("bf_kernels.cu", "bf_enum.cuh", "bf_sim.cuh", "bf_launch.h")
 
 
-def kernel_fingerprint() -> str:
-    """Hash of the enumerating kernels' sources and flags: a profile taken of those kernels stays
-    valid while this is unchanged (changes elsewhere in the library do not touch them)."""
+def _code_only(text: str) -> str:
+    """C++ source without comments and with whitespace runs collapsed (no string literal in the
+    kernel unit contains a comment marker)."""
+    text = re.sub(r"/\*.*?\*/", " ", text, flags=re.S)
+    text = re.sub(r"//[^\n]*", " ", text)
+    return " ".join(text.split())
+
+
+def kernel_fingerprint(csrc: str = CSRC) -> str:
+    """Hash of the enumerating kernels' code (comments and layout ignored) and flags: a profile
+    taken of those kernels stays valid while this is unchanged (changes elsewhere in the library,
+    or to comments, do not touch them)."""
     h = hashlib.sha256()
     for name in KERNEL_UNIT:
-        with open(os.path.join(CSRC, name), "rb") as fh:
-            h.update(name.encode() + fh.read())
+        with open(os.path.join(csrc, name), encoding="utf-8") as fh:
+            h.update(name.encode() + _code_only(fh.read()).encode())
     flags = [f for f in NVCC_FLAGS if not f.startswith("-I")]
     h.update(" ".join(ARCH + flags).encode())
     return h.hexdigest()
