@@ -225,7 +225,10 @@ typedef struct bf_tree_stats {
  * flags: 0 or BF_TREE_NO_PRUNE (every mapping of the space is simulated:
  * full enumeration).  `stats` may be NULL.  Allocates level buffers in the
  * handle on first use (about 1.7 GB for 32 tools in the full space).  Blocks
- * until the result is on the host; every level step is a bounded wait. */
+ * until the result is on the host.  The whole search, not only each level
+ * step, is held to the wait limit (bf_set_wait_timeout_ms): past it the call
+ * returns BF_ETIMEOUT (hard full spaces of 28-32 tools with tight budgets can
+ * take minutes). */
 BF_API int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint64_t hint_index,
                    bf_result* out, bf_tree_stats* stats, void* cuda_stream);
 

@@ -111,6 +111,8 @@ int validate(const bf_scenario_desc* d, const char* who) {
   return BF_OK;
 }
 
+uint32_t wait_limit_ms() { return g_wait_timeout_ms.load(std::memory_order_relaxed); }
+
 int wait_stream(cudaStream_t st, const char* who) {
   const auto t0 = std::chrono::steady_clock::now();
   for (uint32_t polls = 0;; ++polls) {

@@ -64,6 +64,8 @@ cudaError_t lib_malloc(void** p, size_t bytes);
 cudaError_t lib_malloc_host(void** p, size_t bytes);
 // Wait for `st` with the process-wide time limit (BF_ETIMEOUT when it passes).
 int wait_stream(cudaStream_t st, const char* who);
+// That limit in milliseconds (0: none).
+uint32_t wait_limit_ms();
 // BF_EINVAL unless the handle's device is current.
 int check_device(const bf_scenario* scn, const char* who);
 // Makespans of a list of mappings on the index-list kernel for the scenario's width.

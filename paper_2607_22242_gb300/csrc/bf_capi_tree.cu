@@ -8,6 +8,7 @@
 #include <cstddef>
 #include <cstring>
 #include <new>
+#include <chrono>
 #include <vector>
 
 #include "bf_capi_internal.h"
@@ -145,6 +146,9 @@ int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flag
   //    with that bound.  (Measured: 8192 beat 64 and 1024, and beat diving
   //    without the restart.)
   constexpr uint32_t kDive = 8192;
+  // The whole search, not only each wait, is held to the wait limit.
+  const auto t_start = std::chrono::steady_clock::now();
+  const uint32_t limit_ms = wait_limit_ms();
   std::vector<uint32_t> size(levels, 0);
   size[0] = 1;
   uint64_t nodes = 1;
@@ -184,6 +188,11 @@ int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flag
     if (e != cudaSuccess) return cuda_fail(e, who);
     const int rc = wait_stream(st, who);
     if (rc != BF_OK) return rc;
+    if (limit_ms) {
+      const auto ms = std::chrono::duration_cast<std::chrono::milliseconds>(std::chrono::steady_clock::now() - t_start);
+      if (ms.count() > (long long)limit_ms)
+        return fail(BF_ETIMEOUT, "%s: search not finished after %u ms", who, limit_ms);
+    }
     ++launches;
     const uint32_t added = (uint32_t)(h->appended - before);
     size[L + 1] = added;
