@@ -130,9 +130,9 @@ inline void retired_estimate(const TB& t, uint32_t* R) {
 // predecessors) first, each group in the scenario's order.  A topological
 // order, and one that changes no result of the model: its only dependence on
 // numbering is the queue's tie between tools that became ready at the same
-// instant, and a source (ready at time 0) never ties with another tool (ready
-// after a predecessor of at least 1 us has ended), while each group keeps its
-// order.  A late source then settles in the prefix instead of leaving the
+// instant, and a source (ready at time 0) never ties with a tool that has a
+// predecessor (ready only after it has run for at least 1 us), while each
+// group keeps its order.  A late source then settles in the prefix instead of leaving the
 // window open from time 0 (layered DAGs with sources in later layers: 16
 // tools 3.38 -> 2.66 ms, 20 tools 1234 -> 245 ms; 4096 layered 10-tool DAGs
 // 11 % faster).  For searches over the whole space only (the mapping index of
