@@ -1,0 +1,145 @@
+// Host build of the search kernels' enumeration logic (bf_plan.h, bf_enum.cuh,
+// bf_sim.cuh), for tests that run without a GPU: the warp tasks of a plan are
+// executed lane by lane on the CPU with the same code the kernels run, and
+// every mapping's makespan is stored at its canonical index.  Test
+// infrastructure only; the library never runs this.
+#include <algorithm>
+#include <cstdint>
+#include <cstring>
+#include <vector>
+
+#define __device__
+#define __host__
+#define __forceinline__ inline
+using std::min;
+static inline int __popc(unsigned x) { return __builtin_popcount(x); }
+static inline unsigned long long __umul64hi(unsigned long long a, unsigned long long b) {
+  return (unsigned long long)(((unsigned __int128)a * b) >> 64);
+}
+struct HostDim {
+  unsigned x;
+};
+static HostDim threadIdx{0}, blockDim{1};
+
+#include "../paper_2607_22242_gb300/csrc/bf_enum.cuh"
+#include "../paper_2607_22242_gb300/csrc/bf_plan.h"
+
+using namespace bfk;
+
+namespace {
+
+struct StoreAll {
+  uint32_t first;
+  uint32_t* out;
+  void operator()(uint32_t idx, uint32_t ms) { out[idx - first] = ms; }
+};
+
+// Lane states of one emulated warp: [word][lane] as in shared memory, filled
+// with garbage first (shared memory holds stale data on the GPU).
+struct Lanes {
+  std::vector<uint32_t> words;
+  explicit Lanes(int lane_words) : words(2u * (uint32_t)lane_words * 32u, 0xA5A5A5A5u) {}
+};
+
+template <int NP, int NW, bool RL>
+void run_tasks(const Tables& tb, const Tables& tw, const Plan& plan, bool mid_lanes, uint32_t* out) {
+  threadIdx.x = 0;
+  SmemTables sd, sdw;
+  load_smem_tables(tb, sd);
+  load_smem_tables(tw, sdw);
+  std::vector<uint32_t> rt(ReadyTable<NP>::size), rtw(ReadyTable<NW>::size), mpart(kMaxMidPartWords);
+  fill_ready_table<NP>(tb, rt.data());
+  fill_ready_table<NW>(tw, rtw.data());
+  fill_mid_parts(plan, mpart.data());
+  const int lw = LaneWords<NW>::value;
+  StoreAll sink{plan.first, out};
+  if (mid_lanes) {
+    for (uint32_t p = 0; p < plan.pow3P; ++p) {
+      Lanes lanes(lw);
+      for (unsigned lane = 0; lane < 32; ++lane) {
+        threadIdx.x = lane;
+        mid_lane_task<NP, NW>(tb, sd, rt.data(), tw, sdw, rtw.data(), plan, mpart.data(), p, lanes.words.data() + lane,
+                              lanes.words.data() + lw * 32 + lane, 32, sink);
+      }
+    }
+    return;
+  }
+  for (uint32_t g = 0; g < plan.groups; ++g)
+    for (uint32_t part = 0; part < plan.m_parts; ++part) {
+      Lanes lanes(lw);
+      for (unsigned lane = 0; lane < 32; ++lane) {
+        threadIdx.x = lane;
+        warp_task<NP, NW, RL>(tb, sd, rt.data(), tw, sdw, rtw.data(), plan, mpart.data(), g, part,
+                              lanes.words.data() + lane, lanes.words.data() + lw * 32 + lane, 32, sink);
+      }
+    }
+}
+
+template <int NW>
+void run_width(const Tables& tb, const Tables& tw, const Plan& plan, bool mid_lanes, uint32_t* out) {
+  const bool rl = plan.relabeled != 0u;
+  if (tb.n <= (uint32_t)NW) {
+    if (rl) run_tasks<NW, NW, true>(tb, tw, plan, mid_lanes, out);
+    else run_tasks<NW, NW, false>(tb, tw, plan, mid_lanes, out);
+  } else {
+    if (rl) run_tasks<kMaxTools, NW, true>(tb, tw, plan, mid_lanes, out);
+    else run_tasks<kMaxTools, NW, false>(tb, tw, plan, mid_lanes, out);
+  }
+}
+
+}  // namespace
+
+// mode 0: the searches' plan in the scenario's numbering, over [first, first+count).
+// mode 1: the whole space, renumbered with the sources first (when that
+//         changes the order), as the whole-space searches may run it.
+// mode 2: the whole space with a batch record's plan (renumbered when that
+//         improves the split; lanes take mid combinations for whole-DAG windows).
+// Slots beyond a window count as done, so a width of 4, 7, 10, 14 or 20 slots
+// serves every window up to it (the library compiles every width).
+// info[0..5] = P, M, I, W0, window tools, flags (1 renumbered, 2 last tool apart, 4 mid lanes).
+extern "C" int host_eval(const bf_scenario_desc* d, uint64_t first, uint64_t count, uint32_t mode, uint32_t* out,
+                         uint32_t* info) {
+  Tables t0, tb, tw;
+  Plan base;
+  host::build_tables(d, &t0);
+  const uint64_t total = host::pow3(d->n);
+  bool mid_lanes = false;
+  if (mode == 0) {
+    tb = t0;
+    host::split_and_window(tb, &base, &tw);
+  } else {
+    if (first != 0 || count != total) return -1;
+    if (mode == 1) {
+      host::relabel_sources_first(t0, &tb);
+      host::split_and_window(tb, &base, &tw);
+    } else {
+      Tables rt, rw;
+      Plan rp;
+      tb = t0;
+      host::split_and_window_batch(tb, &base, &tw);
+      if (host::relabel_sources_first(t0, &rt)) {
+        host::split_and_window_batch(rt, &rp, &rw);
+        if (host::renumbering_helps(t0, base, tw, rt, rp, rw)) {
+          tb = rt;
+          base = rp;
+          tw = rw;
+        }
+      }
+      mid_lanes = base.W0 == 0u;
+    }
+  }
+  const Plan plan = host::make_plan(base, first, count, mode == 2 ? 8u : 4096u);
+  info[0] = plan.P;
+  info[1] = plan.M;
+  info[2] = plan.I;
+  info[3] = plan.W0;
+  info[4] = tw.n;
+  info[5] = (tb.relabeled ? 1u : 0u) | (plan.last_apart ? 2u : 0u) | (mid_lanes ? 4u : 0u);
+  for (uint64_t j = 0; j < count; ++j) out[j] = 0xDEADBEEFu;
+  if (tw.n <= 4) run_width<4>(tb, tw, plan, mid_lanes, out);
+  else if (tw.n <= 7) run_width<7>(tb, tw, plan, mid_lanes, out);
+  else if (tw.n <= 10) run_width<10>(tb, tw, plan, mid_lanes, out);
+  else if (tw.n <= 14) run_width<14>(tb, tw, plan, mid_lanes, out);
+  else run_width<20>(tb, tw, plan, mid_lanes, out);
+  return 0;
+}
