@@ -143,3 +143,78 @@ extern "C" int host_eval(const bf_scenario_desc* d, uint64_t first, uint64_t cou
   else run_width<20>(tb, tw, plan, mid_lanes, out);
   return 0;
 }
+
+// The branch and bound of bf_search_pruned (its plan on the tables it runs
+// on, renumbered when that improves the split) with incumbent makespan
+// `bound`: pass 1 keeps the prefixes whose checkpoint bound does not exceed
+// it, pass 2 enumerates their mappings with the bound at the inner
+// checkpoint.  Returns the best key, (makespan << 32) | canonical index.
+namespace {
+struct MinKey {
+  unsigned long long best = ~0ull;
+  void operator()(uint32_t idx, uint32_t ms) {
+    const unsigned long long k = ((unsigned long long)ms << 32) | idx;
+    if (k < best) best = k;
+  }
+};
+
+template <int NP, int NW>
+unsigned long long pruned(const Tables& tb, const Tables& tw, Plan plan) {
+  threadIdx.x = 0;
+  SmemTables sd, sdw;
+  load_smem_tables(tb, sd);
+  load_smem_tables(tw, sdw);
+  std::vector<uint32_t> rt(ReadyTable<NP>::size), rtw(ReadyTable<NW>::size), mpart(kMaxMidPartWords), surv;
+  fill_ready_table<NP>(tb, rt.data());
+  fill_ready_table<NW>(tw, rtw.data());
+  fill_mid_parts(plan, mpart.data());
+  for (uint32_t p = 0; p < plan.pow3P; ++p) {
+    Digits dgp;
+    uint32_t T = 0;
+    if (prefix_checkpoint<NP, NW>(tb, sd, rt.data(), plan, p, &dgp, &T, nullptr, 0u) &&
+        (uint64_t)T + plan.tail_p <= plan.bound)
+      surv.push_back(p);
+  }
+  MinKey sink;
+  const int lw = LaneWords<NW>::value;
+  for (size_t g = 0; g < surv.size(); g += 32) {
+    Lanes lanes(lw);
+    for (unsigned lane = 0; lane < 32; ++lane) {
+      threadIdx.x = lane;
+      const bool valid = g + lane < surv.size();
+      prefix_task<NP, NW, true>(tb, sd, rt.data(), tw, sdw, rtw.data(), plan, mpart.data(), valid ? surv[g + lane] : 0u,
+                                valid, 0u, lanes.words.data() + lane, lanes.words.data() + lw * 32 + lane, 32, sink);
+    }
+  }
+  return sink.best;
+}
+
+template <int NW>
+unsigned long long pruned_width(const Tables& tb, const Tables& tw, const Plan& plan) {
+  return tb.n <= (uint32_t)NW ? pruned<NW, NW>(tb, tw, plan) : pruned<kMaxTools, NW>(tb, tw, plan);
+}
+}  // namespace
+
+extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bound) {
+  Tables t0, tb, tw, rt, rw;
+  Plan base, rp;
+  host::build_tables(d, &t0);
+  tb = t0;
+  host::split_and_window(t0, &base, &tw);
+  if (host::relabel_sources_first(t0, &rt)) {
+    host::split_and_window(rt, &rp, &rw);
+    if (host::renumbering_helps(t0, base, tw, rt, rp, rw)) tb = rt;
+  }
+  host::split_and_window_pruned(tb, &base, &tw);
+  Plan plan = host::make_plan(base, 0, host::pow3(d->n), 4096u);
+  plan.bound = bound;
+  plan.m_lo = 0;
+  plan.m_hi = plan.pow3M - 1u;
+  plan.m_chunk = plan.pow3M;
+  plan.m_parts = 1;
+  if (tw.n <= 4) return pruned_width<4>(tb, tw, plan);
+  if (tw.n <= 7) return pruned_width<7>(tb, tw, plan);
+  if (tw.n <= 10) return pruned_width<10>(tb, tw, plan);
+  if (tw.n <= 14) return pruned_width<14>(tb, tw, plan);
+  return pruned_width<20>(tb, tw, plan);
+}

@@ -34,6 +34,8 @@ def host():
     lib.host_eval.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint64, ctypes.c_uint64, ctypes.c_uint32,
                               ctypes.c_void_p, ctypes.c_void_p]
     lib.host_eval.restype = ctypes.c_int
+    lib.host_pruned.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint32]
+    lib.host_pruned.restype = ctypes.c_uint64
 
     def run(scn, first, count, mode):
         d = bf.to_desc(scn)
@@ -41,6 +43,7 @@ def host():
         info = np.zeros(6, np.uint32)
         assert lib.host_eval(ctypes.byref(d), first, count, mode, ms.ctypes.data, info.ctypes.data) == 0
         return ms.astype(np.uint64), info
+    run.pruned = lambda scn, bound: lib.host_pruned(ctypes.byref(bf.to_desc(scn)), bound)
     return run
 
 
@@ -90,3 +93,28 @@ def test_standard_workloads_host(host):
     total = 3 ** scn.n
     for first in (0, total // 2 - 1000, total - 60_001):
         _same(host, scn, first, 60_001, 0)
+
+
+def test_branch_and_bound_host(host):
+    """bf_search_pruned's two passes (checkpoint bound, then the survivors' mappings with the
+    bound at the inner checkpoint) with incumbents at the optimum, above it and absent: always
+    the oracle's optimum, ties to the lowest index."""
+    rng = np.random.default_rng(91)
+    for t in range(150):
+        n = int(rng.integers(1, 10))
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.3, 0.6])), tight=bool(t % 3),
+                              max_time=int(rng.choice([5, 40, 2000])))
+        pred = list(base.pred_mask)
+        if t % 3 == 0 and n > 3:
+            pred[int(rng.integers(n // 2, n))] = 0
+        scn = S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
+                         base.vram_budget_mib, base.slowdown_q10)
+        want = oracle.search(scn)
+        for bound in (want[1], want[1] + int(rng.integers(0, 60)), 0xFFFFFFFF):
+            key = host.pruned(scn, bound)
+            assert (key & 0xFFFFFFFF, key >> 32) == tuple(want), (t, bound)
+    for cfg in (1, 2):
+        scn = S.config(cfg)
+        want = oracle.search(scn, THREADS)
+        key = host.pruned(scn, want[1])
+        assert (key & 0xFFFFFFFF, key >> 32) == tuple(want)
