@@ -28,7 +28,14 @@ int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flag
   if (const int rc = check_device(scn_const, who)) return rc;
   // The handle's lazily allocated level buffers are scratch, not state.
   bf_scenario* scn = const_cast<bf_scenario*>(scn_const);
-  const bfk::TablesW& tb = scn->wide;
+  // The tree runs on the tools renumbered with the sources first
+  // (relabel_sources_first): a source in a later layer is then decided near
+  // the root instead of keeping every node's window open from time 0, and the
+  // model's results do not change.  Indices stay canonical: slot v holds tool
+  // tb.orig[v], whose digit weighs 3^orig[v].
+  bfk::TablesW renumbered;
+  const bool relabeled = bfk::host::relabel_sources_first(scn->wide, &renumbered);
+  const bfk::TablesW& tb = relabeled ? renumbered : scn->wide;
   const uint32_t n = scn->desc.n, R = space;
   const bool prune = !(flags & BF_TREE_NO_PRUNE);
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
@@ -65,8 +72,8 @@ int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flag
       tc.sdown[v] = (uint32_t)(longest < 0xFFFFFFFFull ? longest : 0xFFFFFFFFull);
       down[v] = tc.dmin[v] + longest;
     }
-    uint64_t p = 1;
-    for (uint32_t i = 0; i < (uint32_t)bfk::kTreeSlots; ++i, p *= 3) tc.pow3[i] = p;
+    for (uint32_t i = 0; i < (uint32_t)bfk::kTreeSlots; ++i) tc.pow3[i] = pow3(i < n ? tb.orig[i] : i);
+    tc.relabeled = relabeled ? 1u : 0u;
   }
 
   // Level buffers: level d holds up to R * kPop nodes (one pop of its parent
@@ -103,10 +110,11 @@ int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flag
     if (hint_ok && R == 2)
       for (uint64_t v = hint_index; v; v /= 3) hint_ok = hint_ok && (v % 3 != 2);
     if (hint_ok) h->idx[nc++] = hint_index;
+    const bfk::TablesW& tsc = scn->wide;  // the scenario's numbering
     uint64_t now = 0, fast = 0, p = 1;
     for (uint32_t i = 0; i < n; ++i, p *= 3) {
       now += p;
-      if ((tb.wnow[i] >> 10) < tb.cpu[i]) fast += p;
+      if ((tsc.wnow[i] >> 10) < tsc.cpu[i]) fast += p;
     }
     h->idx[nc++] = 0;
     h->idx[nc++] = now;

@@ -159,7 +159,7 @@ __global__ void __launch_bounds__(LeafShape<NW>::threads, LeafShape<NW>::min_blo
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) {
     const LaneBest other = shfl_best(lb, o);
-    lb.offer(other.ms, other.dg);
+    lb.offer(other.ms, other.dg, tc.tie_pow3());
   }
   if (lane == 0) {
     wb_ms[warp] = lb.ms;
@@ -169,7 +169,7 @@ __global__ void __launch_bounds__(LeafShape<NW>::threads, LeafShape<NW>::min_blo
   __syncthreads();
   if (threadIdx.x == 0) {
     LaneBest b;
-    for (int w = 0; w < LeafShape<NW>::warps; ++w) b.offer(wb_ms[w], Digits{wb_now[w], wb_que[w]});
+    for (int w = 0; w < LeafShape<NW>::warps; ++w) b.offer(wb_ms[w], Digits{wb_now[w], wb_que[w]}, tc.tie_pow3());
     if (b.ms != kInfeasible) {
       atomicMin(bound, b.ms);
       best_min(best, b.ms, index_of(b.dg, tc.pow3), ctr);

@@ -43,7 +43,12 @@ struct TreeConsts {
   uint32_t alone[3];
   uint32_t dmin[kTreeSlots];   // min(c, g + x): no mode runs tool v faster
   uint32_t sdown[kTreeSlots];  // longest path in dmin through v's successors (0 for a sink)
-  uint64_t pow3[kTreeSlots];
+  // 1 when the tools are renumbered (sources first): tree slot v holds tool
+  // orig[v] of the scenario, and ties compare canonical indices.
+  uint32_t relabeled;
+  uint64_t pow3[kTreeSlots];   // 3^(scenario position) of each slot's tool
+  // pow3 when ties need it (renumbered tools), else nullptr.
+  __device__ __forceinline__ const uint64_t* tie_pow3() const { return relabeled ? pow3 : nullptr; }
 };
 
 // A saved node: the state's words, then the digit masks; [word][node] layout
@@ -291,12 +296,15 @@ __device__ __forceinline__ bool index_less(Digits a, Digits b) {
   return da < db;
 }
 
-// Best mapping seen: lowest makespan, ties to the lowest index.
+// Best mapping seen: lowest makespan, ties to the lowest canonical index.
+// pow3 (TreeConsts::tie_pow3) is nullptr when slot order is the scenario's
+// order; otherwise ties compare the canonical indices it gives.
 struct LaneBest {
   uint32_t ms = kInfeasible;
   Digits dg{0u, 0u};
-  __device__ __forceinline__ void offer(uint32_t m, Digits d) {
-    if (m < ms || (m == ms && m != kInfeasible && index_less(d, dg))) {
+  __device__ __forceinline__ void offer(uint32_t m, Digits d, const uint64_t* pow3) {
+    if (m < ms ||
+        (m == ms && m != kInfeasible && (pow3 ? index_of(d, pow3) < index_of(dg, pow3) : index_less(d, dg)))) {
       ms = m;
       dg = d;
     }
@@ -329,8 +337,9 @@ __device__ __forceinline__ void leaf_combos(const TBW& tw, const SD& sdw, const 
       const Digits full{dg.now | (dc.now << W0), dg.que | (dc.que << W0)};
       for (uint32_t a = 0; a < tc.radix; ++a) {
         if (tc.alone[a] == kInfeasible) continue;
-        best.offer(w.T + tc.alone[a], Digits{full.now | (a == 1u ? 1u << last : 0u),
-                                               full.que | (a == 2u ? 1u << last : 0u)});
+        best.offer(w.T + tc.alone[a],
+                   Digits{full.now | (a == 1u ? 1u << last : 0u), full.que | (a == 2u ? 1u << last : 0u)},
+                   tc.tie_pow3());
       }
     }
     return;
@@ -343,7 +352,7 @@ __device__ __forceinline__ void leaf_combos(const TBW& tw, const SD& sdw, const 
     State<NW> w;
     load_lane(slot, stride, w);
     if (run<NW>(w, tw, sdw, rtw, sim, 0u) != kRunFinished) continue;
-    best.offer(w.T, Digits{dg.now | (dc.now << W0), dg.que | (dc.que << W0)});
+    best.offer(w.T, Digits{dg.now | (dc.now << W0), dg.que | (dc.que << W0)}, tc.tie_pow3());
   }
 }
 

@@ -165,7 +165,8 @@ def test_magnitudes_at_the_validation_bounds(n):
 def test_late_sources_renumbered_searches():
     """DAGs with sources late in the scenario's numbering, which the whole-space searches may
     renumber (sources first), with small integer times so that queue ties are frequent: the
-    exhaustive search, the branch and bound and the batched search against the oracle."""
+    exhaustive search, the branch and bound, the batched search and the tree search (which always
+    renumbers; both spaces) against the oracle."""
     rng = np.random.default_rng(31)
     scns = []
     for t in range(160):
@@ -184,6 +185,10 @@ def test_late_sources_renumbered_searches():
             assert (r.index, r.makespan_us) == w, scn
             rp = bf.search_pruned(h)
             assert (rp.index, rp.makespan_us) == w, scn
+            rt, _ = bf.search_tree(h, bf.SPACE_FULL, True)
+            assert (rt.index, rt.makespan_us) == w, scn
+            rb, _ = bf.search_tree(h, bf.SPACE_BINARY, True)
+            assert (rb.index, rb.makespan_us) == oracle.search_binary(scn, THREADS), scn
     assert [(r.index, r.makespan_us) for r in bf.search_batch(scns)] == want
 
 
