@@ -42,39 +42,7 @@ int search_tree_impl(const bf_scenario* scn_const, uint32_t space, uint32_t flag
 
   // Constants: the leaf depth, the bound's per-tool durations, digit powers.
   bfk::TreeConsts tc;
-  std::memset(&tc, 0, sizeof tc);
-  tc.n = n;
-  tc.radix = R;
-  tc.D = n < (R == 3 ? 5u : 8u) ? n : (R == 3 ? 5u : 8u);
-  tc.leaf_level = n - tc.D;
-  tc.combos = 1;
-  for (uint32_t i = 0; i < tc.D; ++i) tc.combos *= R;
-  tc.prune = prune ? 1u : 0u;
-  tc.W0 = bfk::host::window_start(tb, tc.leaf_level);
-  {
-    uint32_t anc[bfk::kTreeSlots];
-    bfk::host::ancestors(tb, anc);
-    const uint32_t last = n - 1, others = (last >= 32u) ? ~0u : ((1u << last) - 1u);
-    tc.alone_last = (tc.D >= 1u && (anc[last] & others) == others) ? 1u : 0u;
-    const bool fits = tb.vram[last] <= tb.budget;
-    tc.alone[0] = tb.cpu[last];
-    tc.alone[1] = fits ? tb.wnow[last] >> 10 : 0xFFFFFFFFu;
-    tc.alone[2] = fits ? tb.wq[last] >> 10 : 0xFFFFFFFFu;
-  }
-  {
-    uint64_t down[bfk::kTreeSlots] = {0};
-    for (int v = (int)n - 1; v >= 0; --v) {
-      const uint32_t gpu = tb.wnow[v] >> 10;
-      tc.dmin[v] = tb.cpu[v] < gpu ? tb.cpu[v] : gpu;
-      uint64_t longest = 0;
-      for (uint32_t w = (uint32_t)v + 1; w < n; ++w)
-        if ((tb.succ[v] >> w) & 1u) longest = down[w] > longest ? down[w] : longest;
-      tc.sdown[v] = (uint32_t)(longest < 0xFFFFFFFFull ? longest : 0xFFFFFFFFull);
-      down[v] = tc.dmin[v] + longest;
-    }
-    for (uint32_t i = 0; i < (uint32_t)bfk::kTreeSlots; ++i) tc.pow3[i] = pow3(i < n ? tb.orig[i] : i);
-    tc.relabeled = relabeled ? 1u : 0u;
-  }
+  bfk::host::tree_consts(tb, R, prune, &tc);
 
   // Level buffers: level d holds up to R * kPop nodes (one pop of its parent
   // level); nodes are popped from the deepest non-empty level, so no level

@@ -238,9 +238,6 @@ cudaError_t launch_tree_expand(const TablesW& tb, const TreeConsts& tc, const ui
   return cudaGetLastError();
 }
 
-// Window buckets of the leaf kernel.
-#define BF_TREE_BUCKETS(X) X(8) X(12) X(16) X(20) X(24) X(32)
-
 template <int NW>
 static cudaError_t leaf_launch(const TablesW& tb, const TreeConsts& tc, const uint32_t* src, uint32_t src_cap,
                                uint32_t lo, uint32_t cnt, uint32_t parts, uint32_t chunk, unsigned grid,

@@ -19,6 +19,7 @@
 // search returns the same (makespan, lowest index) as full enumeration.
 #pragma once
 
+#include "bf_plan.h"
 #include "bf_sim.cuh"
 
 namespace bfk {
@@ -26,6 +27,10 @@ namespace bfk {
 constexpr int kTreeSlots = 32;
 using TablesW = TablesT<kTreeSlots>;
 using SmemTablesW = SmemTablesT<kTreeSlots>;
+
+// Leaf window widths compiled for the leaf kernel: a window of nw tools runs
+// in the narrowest that holds it.
+#define BF_TREE_BUCKETS(X) X(8) X(12) X(16) X(20) X(24) X(32)
 
 // Per-scenario constants of a tree search.
 struct TreeConsts {
@@ -356,4 +361,49 @@ __device__ __forceinline__ void leaf_combos(const TBW& tw, const SD& sdw, const 
   }
 }
 
+namespace host {
+
+// Constants of a search over tables tb (the scenario's tools, renumbered or
+// not) in the space of radix R (2: binary, 3: full): the leaf depth D (5 tools
+// in the full space, 8 in the binary one, all of them for smaller scenarios),
+// the leaf window, the lone last tool's durations, the per-tool minimum
+// durations and downstream paths of the bounds, and each slot's place value
+// in the canonical index.
+inline void tree_consts(const TablesW& tb, uint32_t R, bool prune, TreeConsts* out) {
+  TreeConsts& tc = *out;
+  std::memset(&tc, 0, sizeof tc);
+  const uint32_t n = tb.n;
+  tc.n = n;
+  tc.radix = R;
+  tc.D = n < (R == 3 ? 5u : 8u) ? n : (R == 3 ? 5u : 8u);
+  tc.leaf_level = n - tc.D;
+  tc.combos = 1;
+  for (uint32_t i = 0; i < tc.D; ++i) tc.combos *= R;
+  tc.prune = prune ? 1u : 0u;
+  tc.W0 = window_start(tb, tc.leaf_level);
+  {
+    uint32_t anc[kTreeSlots];
+    ancestors(tb, anc);
+    const uint32_t last = n - 1, others = (last >= 32u) ? ~0u : ((1u << last) - 1u);
+    tc.alone_last = (tc.D >= 1u && (anc[last] & others) == others) ? 1u : 0u;
+    const bool fits = tb.vram[last] <= tb.budget;
+    tc.alone[0] = tb.cpu[last];
+    tc.alone[1] = fits ? tb.wnow[last] >> 10 : 0xFFFFFFFFu;
+    tc.alone[2] = fits ? tb.wq[last] >> 10 : 0xFFFFFFFFu;
+  }
+  uint64_t down[kTreeSlots] = {0};
+  for (int v = (int)n - 1; v >= 0; --v) {
+    const uint32_t gpu = tb.wnow[v] >> 10;
+    tc.dmin[v] = tb.cpu[v] < gpu ? tb.cpu[v] : gpu;
+    uint64_t longest = 0;
+    for (uint32_t w = (uint32_t)v + 1; w < n; ++w)
+      if ((tb.succ[v] >> w) & 1u) longest = down[w] > longest ? down[w] : longest;
+    tc.sdown[v] = (uint32_t)(longest < 0xFFFFFFFFull ? longest : 0xFFFFFFFFull);
+    down[v] = tc.dmin[v] + longest;
+  }
+  for (uint32_t i = 0; i < (uint32_t)kTreeSlots; ++i) tc.pow3[i] = pow3(i < n ? tb.orig[i] : i);
+  tc.relabeled = tb.relabeled ? 1u : 0u;
+}
+
+}  // namespace host
 }  // namespace bfk
