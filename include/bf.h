@@ -195,7 +195,7 @@ BF_API int bf_search_pruned(const bf_scenario* scn, uint64_t hint_index, bf_resu
 
 /* What a tree search did (bf_search_tree, optional). */
 typedef struct bf_tree_stats {
-  uint64_t nodes;         /* prefix nodes created (tools assigned in index order), root included */
+  uint64_t nodes;         /* prefix nodes created (tools assigned in the search's order), root included */
   uint64_t leaf_nodes;    /* nodes whose last leaf_depth tools were enumerated */
   uint64_t leaves;        /* mappings simulated to the end (at most leaf_nodes * modes^leaf_depth) */
   uint32_t launches;      /* kernel launches */
@@ -207,9 +207,12 @@ typedef struct bf_tree_stats {
 /* The optimum of a decision space -- the feasible mapping of lowest makespan,
  * ties to the lowest canonical index, exactly as full enumeration would give
  * it -- for scenarios of up to 32 tools (3^32 ~ 1.9e15 mappings), by depth-
- * first branch and bound over the modes of tools 0, 1, 2, ... in index order.
- * A node (the modes of tools [0, d)) carries the simulation state at the
- * first instant a tool >= d could become ready, shared by all its mappings.
+ * first branch and bound over the modes of the tools in a topological order:
+ * the sources (tools without predecessors) first, then the others, each group
+ * in index order (the model's results do not depend on that order; the index
+ * returned is the canonical one).  A node (the modes of the first d tools of
+ * that order) carries the simulation state at the first instant a later tool
+ * could become ready, shared by all its mappings.
  * A node is dropped when a lower bound on all of its mappings' makespans
  * exceeds the best makespan known (strictly, so the optimum and its ties
  * survive): running tools end no earlier than their remaining work at
@@ -227,8 +230,8 @@ typedef struct bf_tree_stats {
  * handle on first use (about 1.7 GB for 32 tools in the full space).  Blocks
  * until the result is on the host.  The whole search, not only each level
  * step, is held to the wait limit (bf_set_wait_timeout_ms): past it the call
- * returns BF_ETIMEOUT (hard full spaces of 28-32 tools with tight budgets can
- * take minutes). */
+ * returns BF_ETIMEOUT (an unpruned full space of 28 or more tools takes
+ * hours). */
 BF_API int bf_search_tree(const bf_scenario* scn, uint32_t space, uint32_t flags, uint64_t hint_index,
                    bf_result* out, bf_tree_stats* stats, void* cuda_stream);
 

@@ -3,6 +3,10 @@
 // tool) or the binary cpu/gpu_now space (§4.1: S1-S10 choose between CPU and
 // GPU only).
 //
+// Tools are numbered as in the tables the search runs on (the scenario's
+// tools with the sources first, host::relabel_sources_first); results carry
+// canonical indices (TreeConsts::pow3).
+//
 // A node at level d assigns modes to tools [0, d) and holds the simulation
 // state at its checkpoint: the first instant at which a tool >= d would
 // become ready (bf_sim.cuh, resumable runs).  Until then no tool >= d has
@@ -291,7 +295,8 @@ __device__ __forceinline__ uint64_t index_of(Digits dg, const uint64_t* pow3) {
   return idx;
 }
 
-// a < b in canonical index order: the highest tool whose digits differ decides.
+// a < b in slot order: the highest slot whose digits differ decides (the
+// canonical order when the slots are not renumbered).
 __device__ __forceinline__ bool index_less(Digits a, Digits b) {
   const uint32_t diff = (a.now ^ b.now) | (a.que ^ b.que);
   if (diff == 0u) return false;
