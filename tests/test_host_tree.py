@@ -9,6 +9,7 @@ that keeps the optimum), and unpruned.  The GPU tests check the kernels' level l
 hardware.
 """
 import ctypes
+import json
 import os
 import subprocess
 import tempfile
@@ -102,3 +103,34 @@ def test_tree_node_logic_standard_workloads(tree):
                 assert got == want, (cfg, space, bound, got, want, st)
             if cfg == 2:
                 assert st[2] == 1
+
+
+def test_tree_node_logic_beyond_20_tools(tree):
+    """32-slot trees: random segmented DAGs of 21-32 tools in both spaces against the segment
+    rule (oracle.segments, pinned against full enumeration), and the stored optima of the 28- and
+    32-tool workloads and of the 24-tool layered DAG's binary space (two late sources, renumbered,
+    no serialisation point; the oracle's full enumeration of 2^24 mappings)."""
+    from oracle import segments
+    rng = np.random.default_rng(4243)
+    for t in range(12):
+        n = int(rng.integers(21, 33))
+        scn = S.random_segmented(rng, n, seg_max=int(rng.choice([4, 6, 8])), tight=bool(t % 2),
+                                 max_time=int(rng.choice([20, 2000])))
+        for space in (3, 2):
+            got, st = tree(scn, space)
+            assert got == tuple(segments.search(scn, binary=space == 2, threads=THREADS)), (t, n, space, got, st)
+    with open(os.path.join(HERE, "golden", "wide_results.json")) as fh:
+        golden = json.load(fh)["workloads"]
+    widths = set()
+    # the 32-tool full space starts from the optimum's makespan, as the kernels' dive would
+    # give it (from no incumbent the depth-first walk simulates 7.7e8 leaves, about 2 minutes)
+    for name, space, key, start in (("wide28", 3, "ternary", False), ("wide32", 3, "ternary", True),
+                                    ("wide32", 2, "binary", False), ("layered24", 2, "binary", False)):
+        scn = getattr(S, name)()
+        assert S.sha256_of([scn]) == golden[name]["sha256"]
+        got, st = tree(scn, space, True, golden[name][key][1] if start else INF)
+        assert got == tuple(golden[name][key]), (name, space, got, st)
+        widths.add(st[3])
+        if name == "layered24":
+            assert st[2] == 1
+    assert max(widths) > 12, widths  # a leaf window wider than the small DAGs reach
