@@ -24,14 +24,11 @@ using bfk::host::build_tables;
 using bfk::host::make_plan;
 using bfk::host::pow3;
 using bfk::host::split_and_window;
-using bfk::host::split_and_window_batch;
 using bfk::host::split_and_window_pruned;
-using bfk::host::relabel_sources_first;
-using bfk::host::renumbering_helps;
-
-// Warp tasks a single-scenario launch is split into (several waves of the
-// GPU's resident warps, so that uneven tasks even out).
-constexpr uint64_t kSearchTasks = 32768;
+using bfk::host::batch_plan;
+using bfk::host::batch_split;
+using bfk::host::kSearchTasks;
+using bfk::host::whole_space_tables;
 
 thread_local std::string g_error;
 std::atomic<uint32_t> g_wait_timeout_ms{600000};
@@ -178,33 +175,6 @@ void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* 
     default: { e = cudaErrorInvalidValue; } break; \
   }
 
-// Plan of one scenario of a batch (one block of kThreads / 32 warps each): a
-// scenario with fewer prefix groups than warps splits its mid combinations
-// so that as many warps as possible share it.
-// Tables, split and window of one scenario of a batch (a whole-space search):
-// renumbered with the sources first when that gives a better split.
-void batch_split(const bf_scenario_desc* d, bfk::Tables* tb, bfk::Plan* plan, bfk::Tables* tw) {
-  bfk::Tables rt, rw;
-  bfk::Plan rp;
-  build_tables(d, tb);
-  split_and_window_batch(*tb, plan, tw);
-  if (relabel_sources_first(*tb, &rt)) {
-    split_and_window_batch(rt, &rp, &rw);
-    if (renumbering_helps(*tb, *plan, *tw, rt, rp, rw)) {
-      *tb = rt;
-      *plan = rp;
-      *tw = rw;
-    }
-  }
-}
-
-bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n) {
-  constexpr uint32_t kWarps = bfk::kThreads / 32;
-  const uint32_t groups = (base.pow3P + 31u) / 32u;
-  const uint32_t fill = groups < kWarps ? kWarps / groups : 1u;
-  return make_plan(base, 0, pow3(n), (uint64_t)fill * groups);
-}
-
 // Records (tables, window tables, plan) of descs[0, count), built on up to 16
 // host threads (about half a microsecond per scenario); the largest window,
 // task count and whether any plan has an inner level are returned too.
@@ -219,7 +189,7 @@ void build_records(const bf_scenario_desc* descs, uint32_t count, bfk::BatchReco
       std::memset(&r, 0, sizeof r);
       bfk::Plan base;
       batch_split(descs + i, &r.full, &base, &r.window);
-      r.plan = batch_plan(base, descs[i].n);
+      r.plan = batch_plan(base, descs[i].n, bfk::kThreads / 32);
       r.mid_lanes = base.W0 == 0u ? 1u : 0u;
       if (r.window.n > part->wmax) part->wmax = r.window.n;
       const uint32_t tasks = r.plan.groups * r.plan.m_parts;
@@ -314,13 +284,7 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   if (desc->n <= BF_MAX_TOOLS_ENUM) {
     build_tables(desc, &s->tables);
     split_and_window(s->tables, &s->plan, &s->window);
-    if (relabel_sources_first(s->tables, &s->rtables)) split_and_window(s->rtables, &s->rplan, &s->rwindow);
-    if (!s->rtables.relabeled ||
-        !renumbering_helps(s->tables, s->plan, s->window, s->rtables, s->rplan, s->rwindow)) {
-      s->rtables = s->tables;
-      s->rplan = s->plan;
-      s->rwindow = s->window;
-    }
+    whole_space_tables(s->tables, s->plan, s->window, split_and_window, &s->rtables, &s->rplan, &s->rwindow);
     split_and_window_pruned(s->rtables, &s->pplan, &s->pwindow);
   }
   cudaError_t e = cudaGetDevice(&s->device);
@@ -713,7 +677,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
       std::memset(&r, 0, sizeof r);
       bfk::Plan plan;
       batch_split(descs + i0 + j, &r.full, &plan, &r.window);
-      r.plan = batch_plan(plan, descs[i0 + j].n);
+      r.plan = batch_plan(plan, descs[i0 + j].n, bfk::kThreads / 32);
       r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
       if (r.window.n > wmax) wmax = r.window.n;
       const uint32_t tasks = r.plan.groups * r.plan.m_parts;

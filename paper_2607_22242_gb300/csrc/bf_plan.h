@@ -301,7 +301,7 @@ inline void plan_for(const bfk::Tables& t, const uint32_t* anc, const uint32_t* 
 // 3.32.
 inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
   const uint32_t n = t.n;
-  uint32_t anc[BF_MAX_TOOLS], R[BF_MAX_TOOLS + 1];
+  uint32_t anc[BF_MAX_TOOLS] = {}, R[BF_MAX_TOOLS + 1] = {};
   ancestors(t, anc);
   retired_estimate(t, R);
   plan_for(t, anc, R, n < 4 ? n : 4, true, pl, w);
@@ -322,7 +322,7 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
 // mid_tools(n) mid tools to fill the lanes (4096 layered 10-tool DAGs: M = 5
 // 38.2 ms, M = 4 41.1 ms); other scenarios take the search plan.
 inline void split_and_window_batch(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
-  uint32_t anc[BF_MAX_TOOLS], R[BF_MAX_TOOLS + 1];
+  uint32_t anc[BF_MAX_TOOLS] = {}, R[BF_MAX_TOOLS + 1] = {};
   ancestors(t, anc);
   retired_estimate(t, R);
   plan_for(t, anc, R, mid_tools(t.n), false, pl, w);
@@ -347,7 +347,7 @@ inline bool renumbering_helps(const bfk::Tables& t, const bfk::Plan& p, const bf
 // prefixes go through its prefix filter (19-tool fan-out DAG: 0.26 ms with
 // 3^12 prefixes, 0.52 ms with 3^13).
 inline void split_and_window_pruned(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
-  uint32_t anc[BF_MAX_TOOLS], R[BF_MAX_TOOLS + 1];
+  uint32_t anc[BF_MAX_TOOLS] = {}, R[BF_MAX_TOOLS + 1] = {};
   ancestors(t, anc);
   retired_estimate(t, R);
   plan_for(t, anc, R, mid_tools(t.n), true, pl, w);
@@ -356,7 +356,7 @@ inline void split_and_window_pruned(const bfk::Tables& t, bfk::Plan* pl, bfk::Ta
 // Lowest tool not certainly done when the first tool of [from, n) becomes ready.
 template <typename TB>
 inline uint32_t window_start(const TB& t, uint32_t from) {
-  uint32_t anc[32];
+  uint32_t anc[32] = {};
   ancestors(t, anc);
   return window_of(anc, t, from);
 }
@@ -427,6 +427,52 @@ inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count
   pl.m_parts = (uint32_t)((num_m + pl.m_chunk - 1) / pl.m_chunk);
   pl.full = (first == 0 && last + 1 == (uint64_t)pl.pow3P * pl.pow3M * pl.pow3I) ? 1u : 0u;
   return pl;
+}
+
+// Warp tasks a single-scenario search is cut into (make_plan): several waves
+// of the GPU's resident warps, so that uneven tasks even out.
+constexpr uint64_t kSearchTasks = 32768;
+
+// Whole-space searches (bf_search_best and bf_search_range over the whole
+// space, bf_search_pruned, the batch) run on the tables renumbered with the
+// sources first when that gives a better split (renumbering_helps); otherwise
+// on t0 with its own split p0 and window w0.  split: split_and_window, or
+// split_and_window_batch for the scenarios of a batch.
+template <typename Split>
+inline void whole_space_tables(const bfk::Tables& t0, const bfk::Plan& p0, const bfk::Tables& w0, Split split,
+                               bfk::Tables* tb, bfk::Plan* plan, bfk::Tables* tw) {
+  bfk::Tables rt, rw;
+  bfk::Plan rp;
+  if (relabel_sources_first(t0, &rt)) {
+    split(rt, &rp, &rw);
+    if (renumbering_helps(t0, p0, w0, rt, rp, rw)) {
+      *tb = rt;
+      *plan = rp;
+      *tw = rw;
+      return;
+    }
+  }
+  *tb = t0;
+  *plan = p0;
+  *tw = w0;
+}
+
+// Tables, split and window of one scenario of a batch (a whole-space search).
+inline void batch_split(const bf_scenario_desc* d, bfk::Tables* tb, bfk::Plan* plan, bfk::Tables* tw) {
+  bfk::Tables t0, w0;
+  bfk::Plan p0;
+  build_tables(d, &t0);
+  split_and_window_batch(t0, &p0, &w0);
+  whole_space_tables(t0, p0, w0, split_and_window_batch, tb, plan, tw);
+}
+
+// Plan of one scenario of a batch, which one block of `block_warps` warps
+// searches: a scenario with fewer prefix groups than warps splits its mid
+// combinations so that as many warps as possible share it.
+inline bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n, uint32_t block_warps) {
+  const uint32_t groups = (base.pow3P + 31u) / 32u;
+  const uint32_t fill = groups < block_warps ? block_warps / groups : 1u;
+  return make_plan(base, 0, pow3(n), (uint64_t)fill * groups);
 }
 
 }  // namespace host

@@ -28,6 +28,8 @@ using namespace bfk;
 
 namespace {
 
+constexpr uint32_t kBlockWarps = 8;  // warps of the batch kernel's blocks (kThreads / 32 in the library)
+
 struct StoreAll {
   uint32_t first;
   uint32_t* out;
@@ -104,31 +106,23 @@ extern "C" int host_eval(const bf_scenario_desc* d, uint64_t first, uint64_t cou
   host::build_tables(d, &t0);
   const uint64_t total = host::pow3(d->n);
   bool mid_lanes = false;
+  Plan plan;
   if (mode == 0) {
     tb = t0;
     host::split_and_window(tb, &base, &tw);
+    plan = host::make_plan(base, first, count, host::kSearchTasks);
   } else {
     if (first != 0 || count != total) return -1;
     if (mode == 1) {
       host::relabel_sources_first(t0, &tb);
       host::split_and_window(tb, &base, &tw);
+      plan = host::make_plan(base, first, count, host::kSearchTasks);
     } else {
-      Tables rt, rw;
-      Plan rp;
-      tb = t0;
-      host::split_and_window_batch(tb, &base, &tw);
-      if (host::relabel_sources_first(t0, &rt)) {
-        host::split_and_window_batch(rt, &rp, &rw);
-        if (host::renumbering_helps(t0, base, tw, rt, rp, rw)) {
-          tb = rt;
-          base = rp;
-          tw = rw;
-        }
-      }
+      host::batch_split(d, &tb, &base, &tw);
+      plan = host::batch_plan(base, d->n, kBlockWarps);
       mid_lanes = base.W0 == 0u;
     }
   }
-  const Plan plan = host::make_plan(base, first, count, mode == 2 ? 8u : 4096u);
   info[0] = plan.P;
   info[1] = plan.M;
   info[2] = plan.I;
@@ -196,17 +190,13 @@ unsigned long long pruned_width(const Tables& tb, const Tables& tw, const Plan& 
 }  // namespace
 
 extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bound) {
-  Tables t0, tb, tw, rt, rw;
-  Plan base, rp;
+  Tables t0, w0, tb, tw;
+  Plan p0, base;
   host::build_tables(d, &t0);
-  tb = t0;
-  host::split_and_window(t0, &base, &tw);
-  if (host::relabel_sources_first(t0, &rt)) {
-    host::split_and_window(rt, &rp, &rw);
-    if (host::renumbering_helps(t0, base, tw, rt, rp, rw)) tb = rt;
-  }
+  host::split_and_window(t0, &p0, &w0);
+  host::whole_space_tables(t0, p0, w0, host::split_and_window, &tb, &base, &tw);
   host::split_and_window_pruned(tb, &base, &tw);
-  Plan plan = host::make_plan(base, 0, host::pow3(d->n), 4096u);
+  Plan plan = host::make_plan(base, 0, host::pow3(d->n), host::kSearchTasks);
   plan.bound = bound;
   plan.m_lo = 0;
   plan.m_hi = plan.pow3M - 1u;
