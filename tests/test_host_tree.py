@@ -92,6 +92,27 @@ def test_tree_node_logic_random_dags(tree):
     assert ("renumbered", 1) in seen and ("renumbered", 0) in seen
 
 
+def test_tree_node_logic_queue_bound(tree):
+    """Queue-heavy DAGs (few edges, tight budgets, steep contention, CPU times scaled up to 10x),
+    where the bound's serial queue sum is what prunes: from the optimum's makespan and from no
+    incumbent, the oracle's optimum (a queue sum raised by 1 us per queued tool changes the
+    result of scenario 15 here)."""
+    rng = np.random.default_rng(6)
+    for t in range(40):
+        n = int(rng.integers(6, 11))
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.1, 0.3])), tight=True, contention=True,
+                              max_time=int(rng.choice([3, 10, 100])))
+        cpu = [c * int(rng.choice([1, 3, 10])) for c in base.cpu_us]
+        scn = S.Scenario(n, base.pred_mask, cpu, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
+                         base.vram_budget_mib, base.slowdown_q10)
+        want = oracle.search(scn)
+        if want[0] < 0:
+            continue
+        for bound in (want[1], INF):
+            got, st = tree(scn, 3, True, bound)
+            assert got == want, (t, bound, got, want, st)
+
+
 def test_tree_node_logic_standard_workloads(tree):
     """The 8-, 12- and 16-tool workloads (the 16-tool one has a late source and runs renumbered)
     in both spaces against the oracle, with the bound at the optimum."""
