@@ -19,6 +19,7 @@ import pytest
 import oracle
 from paper_2607_22242_gb300 import bf
 from paper_2607_22242_gb300 import scenarios as S
+from tie_cases import tie_order_scenarios
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
@@ -118,3 +119,18 @@ def test_branch_and_bound_host(host):
         want = oracle.search(scn, THREADS)
         key = host.pruned(scn, want[1])
         assert (key & 0xFFFFFFFF, key >> 32) == tuple(want)
+
+
+def test_tie_order_scenarios_host(host):
+    """Queue-heavy tiny DAGs with late sources, some with tied optima whose lowest member differs
+    between the canonical and the renumbered order: every mapping in all three modes at its
+    canonical index, and bf_search_pruned's optimum (ties to the lowest canonical index) from the
+    optimum's makespan and from no incumbent."""
+    for t, scn in enumerate(tie_order_scenarios()):
+        for mode in (0, 1, 2):
+            _same(host, scn, 0, 3 ** scn.n, mode)
+        want = oracle.search(scn)
+        for bound in (want[1], 0xFFFFFFFF):
+            key = host.pruned(scn, bound)
+            got = (key & 0xFFFFFFFF, key >> 32) if key != 2 ** 64 - 1 else (-1, 0xFFFFFFFF)
+            assert got == tuple(want), (t, bound, got, want)

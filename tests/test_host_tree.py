@@ -20,6 +20,7 @@ import pytest
 import oracle
 from paper_2607_22242_gb300 import bf
 from paper_2607_22242_gb300 import scenarios as S
+from tie_cases import tie_order_scenarios
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 ROOT = os.path.dirname(HERE)
@@ -117,17 +118,7 @@ def test_tree_node_logic_tie_order(tree):
     """Queue-heavy tiny DAGs with late sources, where the tied optima's lowest canonical index
     differs from the lowest index in the renumbered (sources-first) order (scenario 91 here):
     ties must be broken by canonical index, in both spaces."""
-    rng = np.random.default_rng(1)
-    for t in range(120):
-        n = int(rng.integers(3, 8))
-        base = S.random_small(rng, n, edge_p=float(rng.choice([0.1, 0.3, 0.6])), tight=True, contention=True,
-                              max_time=int(rng.choice([2, 3, 10])))
-        cpu = [c * int(rng.choice([1, 3, 10])) for c in base.cpu_us]
-        pred = list(base.pred_mask)
-        for v in rng.choice(np.arange(1, n), size=int(rng.integers(1, n // 2 + 1)), replace=False):
-            pred[int(v)] = 0
-        scn = S.Scenario(n, pred, cpu, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
-                         base.vram_budget_mib, base.slowdown_q10)
+    for t, scn in enumerate(tie_order_scenarios()):
         for space, want in ((3, oracle.search(scn)), (2, oracle.search_binary(scn))):
             got, st = tree(scn, space)
             assert got == want, (t, space, got, want, st)
