@@ -128,7 +128,10 @@ typedef struct bf_scenario bf_scenario;
 /* Validate a desc without touching the GPU.  BF_OK or BF_EINVAL. */
 BF_API int bf_validate_desc(const bf_scenario_desc* desc);
 
-/* Validate `desc`, copy it, allocate the handle's scratch (8-byte device key,
+/* The problem instance of §2.1 -- the tool DAG G=(V,E), each tool's profile
+ * (Table 1 / §3.1: CPU and GPU latency, load-in, VRAM) plus its transfer time,
+ * the VRAM budget M -- with the contention table of §2.3 Factor A.
+ * Validate `desc`, copy it, allocate the handle's scratch (8-byte device key,
  * 8-byte pinned host key) on the current device and return it in *out.
  * The caller releases it with bf_destroy_scenario.  BF_EINVAL, BF_ENOMEM,
  * BF_ECUDA. */
@@ -160,8 +163,11 @@ BF_API int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_str
 BF_API int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
                     bf_result* out, void* cuda_stream);
 
-/* Full search of `count` independent scenarios in one launch (the batched
- * path): out[i] is the result for descs[i].  All descs are validated first;
+/* Full search of `count` independent scenarios in one launch: out[i] is the
+ * brute-force oracle of §2.3/§4.1 (as bf_search_best) for descs[i].  The paper
+ * searches one workflow at a time; running many per launch is this library's
+ * addition, for callers that score many workflows or many candidate
+ * contention tables (the calibration of Table 2's S5 latencies) together.  All descs are validated first;
  * the first invalid one fails the call with BF_EINVAL naming its position.
  * Allocates and frees its device scratch (packed tables + one key per
  * scenario) per call.  Blocks until the results are on the host. */

@@ -24,9 +24,22 @@ segmented DAGs, and the 19-tool workload's stored brute-force optimum).
 """
 from __future__ import annotations
 
-from typing import List, Tuple
+from typing import List, NamedTuple, Tuple
 
 from . import INFEASIBLE, default
+
+
+class SubScenario(NamedTuple):
+    """The oracle's own record of a segment: the fields its flat record reads."""
+    n: int
+    pred_mask: List[int]
+    cpu_us: List[int]
+    gpu_us: List[int]
+    xfer_us: List[int]
+    load_us: List[int]
+    vram_mib: List[int]
+    vram_budget_mib: int
+    slowdown_q10: List[int]
 
 
 def serialisation_points(pred_mask: List[int], n: int) -> List[int]:
@@ -54,11 +67,10 @@ def serialisation_points(pred_mask: List[int], n: int) -> List[int]:
 
 def segment(scn, lo: int, hi: int):
     """The sub-scenario of tools [lo, hi), renumbered from 0 (edges from below lo dropped)."""
-    from paper_2607_22242_gb300.scenarios import Scenario
     m = hi - lo
-    return Scenario(m, [(scn.pred_mask[v] >> lo) & ((1 << m) - 1) for v in range(lo, hi)],
-                    scn.cpu_us[lo:hi], scn.gpu_us[lo:hi], scn.xfer_us[lo:hi], scn.load_us[lo:hi],
-                    scn.vram_mib[lo:hi], scn.vram_budget_mib, scn.slowdown_q10)
+    return SubScenario(m, [(scn.pred_mask[v] >> lo) & ((1 << m) - 1) for v in range(lo, hi)],
+                       scn.cpu_us[lo:hi], scn.gpu_us[lo:hi], scn.xfer_us[lo:hi], scn.load_us[lo:hi],
+                       scn.vram_mib[lo:hi], scn.vram_budget_mib, scn.slowdown_q10)
 
 
 def bounds(scn) -> List[Tuple[int, int]]:

@@ -45,7 +45,7 @@ QUEUE_PRICED_OUT_US = 3_000_000
 
 
 def table(a: float, b: float) -> List[int]:
-    """f[k] = round(1024 (1 + a (k-1)^b)) for k = 1..20; f[0] unused."""
+    """f[k] = round(1024 (1 + a (k-1)^b)) for k = 1..MAX_TOOLS (the desc's 32 slots); f[0] unused."""
     return [0] + [int(round(1024 * (1 + a * (k - 1) ** b))) for k in range(1, MAX_TOOLS + 1)]
 
 

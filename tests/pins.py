@@ -406,3 +406,64 @@ def check_degenerate_budgets(lib, trials=30, seed=24):
 
 
 ALL_CHECKS += [check_wide_closed_forms, check_binary_space, check_segments, check_degenerate_budgets]
+
+
+# ---------------------------------------------------------------------------
+# The aggregating entry points that write the full-size expected values: the
+# batch search (per-scenario optima of the 4096-scenario workload) and the
+# range summary (feasible count, makespan sum, order-sensitive hash and argmin
+# of the 8-, 12-, 16- and 19-tool workloads).  Each is checked against plain
+# reductions of the per-mapping makespans, which the pins above fix.
+# ---------------------------------------------------------------------------
+
+def _argmin(ms, fe, first=0):
+    """(index, makespan) of the lowest feasible makespan, lowest index among ties; (-1, INF) if none."""
+    best = None
+    for j in range(len(ms)):
+        if fe[j] and (best is None or int(ms[j]) < best[1]):
+            best = (first + j, int(ms[j]))
+    return best if best is not None else (-1, INF)
+
+
+def check_batch_search(lib, seed=25):
+    """Each scenario of a batch gets the argmin of its own 3^n makespans: batches of mixed sizes (1-7
+    tools, so consecutive records differ), a one-scenario batch, the last scenario alone, and several
+    host threads."""
+    rng = np.random.default_rng(seed)
+    scns = [S.random_small(rng, int(rng.integers(1, 8)), max_time=int(rng.choice([9, 700])))
+            for _ in range(25)]
+    want = []
+    for s in scns:
+        ms, fe = lib.eval_range(s, 0, 3 ** s.n)
+        want.append(_argmin(ms, fe))
+    for lo, hi, threads in ((0, 25, 1), (0, 25, 4), (0, 1, 1), (24, 25, 1), (7, 19, 3)):
+        idx, ms = lib.search_batch(scns[lo:hi], threads)
+        got = [(int(i), int(m)) for i, m in zip(idx, ms)]
+        assert got == want[lo:hi], (lo, hi, threads)
+
+
+def check_summary_range(lib, trials=30, seed=26):
+    """The range summary equals plain reductions of the range's makespans: the feasible count, the sum of
+    feasible makespans, the hash sum_j makespan(j) * (j * 2654435761 + 1) mod 2^64 (infeasible counted
+    as 0xFFFFFFFF), summed here in Python integers, and the argmin; on random sub-ranges and over one
+    and several host threads."""
+    rng = np.random.default_rng(seed)
+    for t in range(trials):
+        n = int(rng.integers(1, 8))
+        scn = S.random_small(rng, n, max_time=int(rng.choice([9, 700])))
+        total = 3 ** n
+        first = int(rng.integers(0, total)) if t % 3 else 0
+        count = int(rng.integers(1, total - first + 1)) if t % 3 else total
+        ms, fe = lib.eval_range(scn, first, count)
+        got = lib.summary_range(scn, first, count, int(rng.choice([1, 3])))
+        feas = [int(m) for m, f in zip(ms, fe) if f]
+        assert got["feasible"] == len(feas), (scn, first, count)
+        assert got["makespan_sum"] == sum(feas), (scn, first, count)
+        h = sum(int(m) * ((first + j) * 2654435761 + 1) for j, m in enumerate(ms)) % (1 << 64)
+        assert got["hash"] == h, (scn, first, count)
+        best = _argmin(ms, fe, first)
+        want = (best[0] if best[0] >= 0 else (1 << 64) - 1, best[1])
+        assert (got["best_index"], got["best_makespan"]) == want, (scn, first, count)
+
+
+ALL_CHECKS += [check_batch_search, check_summary_range]

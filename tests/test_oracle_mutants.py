@@ -35,6 +35,12 @@ MUTANTS = {
                                          "for (int i = 0; i + 1 < n; ++i, p *= 3)\n    if ((b >> i) & 1) idx += p;"),
     "edges out of tool 30 ignored": ("if (((s.pred[v] >> u) & 1u) && status[u] != kDone) return false;",
                                      "if (u != 30 && ((s.pred[v] >> u) & 1u) && status[u] != kDone) return false;"),
+    "batch record indexed from the thread's first": ("unpack(flats + j * kFlatWords)", "unpack(flats + (j - lo) * kFlatWords)"),
+    "summary hash multiplier mistyped": ("hash[t] += ms * (idx * 2654435761ull + 1);",
+                                         "hash[t] += ms * (idx * 2654435769ull + 1);"),
+    "summary counts infeasible mappings": ("        if (ms != kInfeasibleMakespan) {\n          feasible[t] += 1;",
+                                           "        if (true) {\n          feasible[t] += 1;"),
+    "summary keeps one thread's sum": ("out[1] += total[t];", "out[1] = total[t];"),
 }
 
 
