@@ -288,10 +288,15 @@ BF_API int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out,
  * scenario, about 2 MiB for BF_NOALLOC_MAX_SCENARIOS) is a fixed array in
  * the library's device image, held on every GPU that loads the library until
  * the process exits.  count > BF_NOALLOC_MAX_SCENARIOS fails with BF_EINVAL.
- * The first call on a device resolves that array's device address; make it
- * before any stream capture.  All calls share the one array, so calls whose
- * GPU work overlaps (other threads, other streams) race and must be
- * serialised by the caller.  Blocks until the results are on the host. */
+ * The first call on a device (and the first after a device reset) resolves
+ * that array's device address; make it before any stream capture.
+ * All calls share the one array, which keeps the last call's contents (each
+ * call resets its keys), so two calls whose GPU work overlapped would race.
+ * The library prevents that: calls on one device are serialised by a host
+ * lock, and after a call returns BF_ETIMEOUT its kernel may still be using
+ * the array, so the next call first waits (bounded) for that call's stream to
+ * finish and returns BF_ETIMEOUT if it does not; keep that stream alive until
+ * then.  Blocks until the results are on the host. */
 BF_API int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                             void* cuda_stream);
 

@@ -336,7 +336,8 @@ def search_batch_noalloc(scns: Sequence[Scenario], stream=None) -> List[Result]:
     memory belongs to another allocator's pool, or a cudaMalloc/cudaFree pair
     would synchronise the device inside a latency-critical loop).  The scratch is
     a fixed array in the library's device image; at most NOALLOC_MAX_SCENARIOS
-    scenarios per call, and calls that overlap on the GPU must not be issued.
+    scenarios per call.  Calls on one device are serialised; after a call that
+    timed out, the next one first waits for that call's stream.
     """
     return _batch_call(load().bf_search_batch_noalloc, scns, stream)
 

@@ -2,6 +2,7 @@
 // device-format tables, launches and bounded waits (the tree search's host
 // side is in bf_capi_tree.cu).  All search arithmetic runs in the kernels
 // (bf_kernels.cu, bf_sim.cuh, bf_tree.cu); this file only marshals.
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <atomic>
@@ -12,6 +13,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <algorithm>
+#include <mutex>
 #include <string>
 #include <thread>
 #include <vector>
@@ -615,60 +617,100 @@ static __device__ __align__(256) unsigned char bf_noalloc_scratch[kNoAllocBytes]
 namespace {
 
 constexpr int kNoAllocMaxDevices = 64;
-std::atomic<unsigned char*> g_noalloc_base[kNoAllocMaxDevices];
 
-// Device address of bf_noalloc_scratch on the current device.  In host code
-// the array's name only stands in for it; the address is resolved once per
-// device, with that device current.
-int noalloc_scratch(unsigned char** base, const char* who) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return cuda_fail(e, who);
-  if (dev < 0 || dev >= kNoAllocMaxDevices)
-    return fail(BF_EINVAL, "%s: device %d is beyond the %d devices this entry point supports", who, dev,
-                kNoAllocMaxDevices);
-  unsigned char* p = g_noalloc_base[dev].load(std::memory_order_acquire);
-  if (!p) {
-    void* addr = nullptr;
-    e = cudaGetSymbolAddress(&addr, bf_noalloc_scratch);
-    if (e != cudaSuccess) return cuda_fail(e, who);
-    p = static_cast<unsigned char*>(addr);
-    g_noalloc_base[dev].store(p, std::memory_order_release);
-  }
-  *base = p;
+// Per-device bookkeeping of the array.  `base` is its device address, resolved
+// with that device current in the context whose ID is `ctx_id` (a device reset
+// destroys the context and the module with it, so a new context resolves the
+// address again).  `pending` is set when a call returned BF_ETIMEOUT: its
+// kernel may still be reading the array on `pending_stream`, so the next call
+// waits for that stream before reusing the array.  `mu` serialises the calls
+// on one device: they all share the one array.
+struct NoAllocDevice {
+  std::mutex mu;
+  unsigned long long ctx_id = 0;
+  unsigned char* base = nullptr;
+  bool pending = false;
+  cudaStream_t pending_stream = nullptr;
+};
+NoAllocDevice g_noalloc[kNoAllocMaxDevices];
+
+// The driver's cuCtxGetCurrent and cuCtxGetId, looked up through the runtime
+// (the library links no driver library).
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+struct CtxFns {
+  CtxGetCurrentFn get_current = nullptr;
+  CtxGetIdFn get_id = nullptr;
+};
+
+const CtxFns& ctx_fns() {
+  static const CtxFns fns = [] {
+    CtxFns f;
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetCurrent", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      f.get_current = reinterpret_cast<CtxGetCurrentFn>(p);
+    p = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuCtxGetId", &p, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      f.get_id = reinterpret_cast<CtxGetIdFn>(p);
+    return f;
+  }();
+  return fns;
+}
+
+// ID of the current context, 0 when none is current yet.
+int current_ctx_id(unsigned long long* id, const char* who) {
+  const CtxFns& f = ctx_fns();
+  if (!f.get_current || !f.get_id) return fail(BF_ECUDA, "%s: cuCtxGetCurrent/cuCtxGetId not available", who);
+  CUcontext ctx = nullptr;
+  if (f.get_current(&ctx) != CUDA_SUCCESS) return fail(BF_ECUDA, "%s: cuCtxGetCurrent failed", who);
+  *id = 0;
+  if (ctx && f.get_id(ctx, id) != CUDA_SUCCESS) return fail(BF_ECUDA, "%s: cuCtxGetId failed", who);
   return BF_OK;
 }
 
-}  // namespace
-
-extern "C" {
-
-int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
-  const char* who = "bf_search_batch_noalloc";
-  if (count == 0) return BF_OK;
-  if (!descs || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
-  if (count > BF_NOALLOC_MAX_SCENARIOS)
-    return fail(BF_EINVAL, "%s: %u scenarios exceed this entry point's fixed scratch of %d scenarios; split the "
-                "batch or use bf_search_batch", who, count, BF_NOALLOC_MAX_SCENARIOS);
-  uint32_t nmax = 0;
-  for (uint32_t i = 0; i < count; ++i) {
-    int rc = validate(descs + i, who);
-    if (rc == BF_OK) rc = require_enum(descs[i], who);
-    if (rc != BF_OK) return fail(rc, "%s: descs[%u]: %s", who, i, g_error.c_str());
-    if (descs[i].n > nmax) nmax = descs[i].n;
-  }
-  unsigned char* base = nullptr;
-  int rc = noalloc_scratch(&base, who);
+// Set-up of the current device, done by the first call on it (and again in a
+// new context after a device reset): the device address of bf_noalloc_scratch.
+// In host code the array's name only stands in for it.  Called with the
+// device's lock held.
+int noalloc_setup(NoAllocDevice& d, const char* who) {
+  unsigned long long id = 0;
+  int rc = current_ctx_id(&id, who);
   if (rc != BF_OK) return rc;
-  bfk::BatchRecord* d_recs = reinterpret_cast<bfk::BatchRecord*>(base);
-  unsigned long long* d_keys = reinterpret_cast<unsigned long long*>(base + kNoAllocKeyOffset);
-  cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  if (id != 0 && id == d.ctx_id) return BF_OK;
+  void* addr = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&addr, bf_noalloc_scratch);  // creates the context if needed
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  rc = current_ctx_id(&id, who);
+  if (rc != BF_OK) return rc;
+  d.base = static_cast<unsigned char*>(addr);
+  d.ctx_id = id;
+  d.pending = false;  // work of an earlier context ended with it
+  return BF_OK;
+}
+
+int search_batch_noalloc_locked(NoAllocDevice& dv, const bf_scenario_desc* descs, uint32_t count, bf_result* out,
+                                cudaStream_t st, const char* who) {
+  int rc = noalloc_setup(dv, who);
+  if (rc != BF_OK) return rc;
+  if (dv.pending) {  // a timed-out call's kernel may still read the array
+    rc = wait_stream(dv.pending_stream, who);
+    if (rc == BF_ETIMEOUT)
+      return fail(BF_ETIMEOUT, "%s: the kernel of an earlier call that timed out is still using the fixed scratch",
+                  who);
+    if (rc != BF_OK) return rc;
+    dv.pending = false;
+  }
+  bfk::BatchRecord* d_recs = reinterpret_cast<bfk::BatchRecord*>(dv.base);
+  unsigned long long* d_keys = reinterpret_cast<unsigned long long*>(dv.base + kNoAllocKeyOffset);
 
   // Pack the records a few at a time through a stack buffer (a copy from
   // pageable memory has left the buffer when cudaMemcpyAsync returns).
   constexpr uint32_t kChunk = 8;
   bfk::BatchRecord chunk[kChunk];
-  uint32_t wmax = 0, pmax = 0, any_inner = 0;
+  uint32_t nmax = 0, wmax = 0, pmax = 0, any_inner = 0;
   cudaError_t e = cudaSuccess;
   for (uint32_t i0 = 0; i0 < count && e == cudaSuccess; i0 += kChunk) {
     const uint32_t nrec = (count - i0 < kChunk) ? (count - i0) : kChunk;
@@ -679,6 +721,7 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
       batch_split(descs + i0 + j, &r.full, &plan, &r.window);
       r.plan = batch_plan(plan, descs[i0 + j].n, bfk::kThreads / 32);
       r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
+      if (descs[i0 + j].n > nmax) nmax = descs[i0 + j].n;
       if (r.window.n > wmax) wmax = r.window.n;
       const uint32_t tasks = r.plan.groups * r.plan.m_parts;
       if (tasks > pmax) pmax = tasks;
@@ -696,6 +739,10 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
   }
   if (e != cudaSuccess) return cuda_fail(e, who);
   rc = wait_stream(st, who);
+  if (rc == BF_ETIMEOUT) {
+    dv.pending = true;
+    dv.pending_stream = st;
+  }
   if (rc != BF_OK) return rc;
   constexpr uint32_t kKeyChunk = 256;
   unsigned long long keys[kKeyChunk];
@@ -707,6 +754,33 @@ int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_re
     for (uint32_t j = 0; j < nk; ++j) fill_result(keys[j], descs[i0 + j].n, 0, out + i0 + j);
   }
   return BF_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int bf_search_batch_noalloc(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
+  const char* who = "bf_search_batch_noalloc";
+  if (count == 0) return BF_OK;
+  if (!descs || !out) return fail(BF_EINVAL, "%s: NULL argument", who);
+  if (count > BF_NOALLOC_MAX_SCENARIOS)
+    return fail(BF_EINVAL, "%s: %u scenarios exceed this entry point's fixed scratch of %d scenarios; split the "
+                "batch or use bf_search_batch", who, count, BF_NOALLOC_MAX_SCENARIOS);
+  for (uint32_t i = 0; i < count; ++i) {
+    int rc = validate(descs + i, who);
+    if (rc == BF_OK) rc = require_enum(descs[i], who);
+    if (rc != BF_OK) return fail(rc, "%s: descs[%u]: %s", who, i, g_error.c_str());
+  }
+  int dev = 0;
+  const cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_fail(e, who);
+  if (dev < 0 || dev >= kNoAllocMaxDevices)
+    return fail(BF_EINVAL, "%s: device %d is beyond the %d devices this entry point supports", who, dev,
+                kNoAllocMaxDevices);
+  NoAllocDevice& dv = g_noalloc[dev];
+  std::lock_guard<std::mutex> lock(dv.mu);
+  return search_batch_noalloc_locked(dv, descs, count, out, static_cast<cudaStream_t>(cuda_stream), who);
 }
 
 // Entry points that allocate host memory keep C++ exceptions inside the library.

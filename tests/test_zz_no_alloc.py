@@ -4,19 +4,26 @@ Some callers cannot allocate device memory at the moment they search -- their
 process has given all GPU memory to another allocator's pool, or a
 cudaMalloc/cudaFree pair would synchronise the device inside a latency-critical
 scheduling loop.  This entry point keeps its scratch in a fixed array inside the
-library's device image.  The test calls it through the C ABI twice in a row,
-with batches of different sizes and contents, and checks each result against
-the allocating entry point bf_search_batch (exact: makespans and indices are
-integers).  Collected last so that a run stopping at the first failure has
-already run every other test.
+library's device image.  The tests call it through the C ABI twice in a row,
+with batches of different sizes and contents (the second on a stream of its
+own), and check each result against the allocating entry point bf_search_batch
+and against the oracle (exact: makespans and indices are integers).  Collected
+last so that a run stopping at the first failure has already run every other
+test.
 """
+import json
+import os
+
 import numpy as np
 import pytest
 
+import oracle
 from paper_2607_22242_gb300 import bf
 from paper_2607_22242_gb300 import scenarios as S
 
 pytestmark = pytest.mark.gpu
+
+GOLDEN = os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", "config_results.json")
 
 
 @pytest.fixture(scope="module", autouse=True)
@@ -34,15 +41,60 @@ def _same(a, b):
            [(r.index, r.makespan_us, r.feasible, r.modes) for r in b]
 
 
-def test_noalloc_matches_allocating_batch_on_two_calls():
+def _batches():
     first = S.config4(bf.NOALLOC_MAX_SCENARIOS)          # the largest batch it accepts
     rng = np.random.default_rng(2024)
     second = [S.random_small(rng, int(rng.integers(1, 12)), max_time=int(rng.choice([9, 700])))
               for _ in range(301)]                           # smaller, mixed sizes: stale keys must not leak
-    for batch in (first, second):
-        got = bf.search_batch_noalloc(batch)
-        want = bf.search_batch(batch)
-        assert _same(got, want)
+    return first, second
+
+
+def _oracle_optima(first, second):
+    with open(GOLDEN) as fh:
+        g = json.load(fh)["configs"]["4"]
+    want_first = list(zip(g["best_index"][:len(first)], g["best_makespan"][:len(first)]))
+    idx, ms = oracle.search_batch(second, oracle.default_threads())
+    return want_first, [(int(i), int(m)) for i, m in zip(idx, ms)]
+
+
+def test_noalloc_matches_allocating_batch_and_oracle_on_two_calls():
+    import torch
+    first, second = _batches()
+    want_first, want_second = _oracle_optima(first, second)
+    side = torch.cuda.Stream()
+    for batch, stream, want in ((first, None, want_first), (second, side, want_second)):
+        got = bf.search_batch_noalloc(batch, stream)
+        assert [(r.index, r.makespan_us) for r in got] == want
+        assert _same(got, bf.search_batch(batch, stream))
+
+
+def test_noalloc_waits_for_a_timed_out_call():
+    """A call that times out leaves its kernel reading the shared array; the next call must not reuse it
+    until that kernel has finished.  64 copies of the 16-tool layered workload (about 0.2 s of kernel)
+    outlast a 1 ms wait limit."""
+    import torch
+    with open(GOLDEN) as fh:
+        g = json.load(fh)["configs"]["2"]["summary"]
+    heavy = [S.config2()] * 64
+    want_heavy = [(g["best_index"], g["best_makespan"])] * len(heavy)
+    _, second = _batches()
+    _, want_second = _oracle_optima([], second)
+    busy = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    try:
+        bf.set_wait_timeout_ms(1)
+        with pytest.raises(bf.BfError) as ei:
+            bf.search_batch_noalloc(heavy, busy)
+        assert ei.value.code == bf.BF_ETIMEOUT
+        with pytest.raises(bf.BfError) as ei:               # the earlier call's kernel is still running
+            bf.search_batch_noalloc(second)
+        assert ei.value.code == bf.BF_ETIMEOUT and "earlier call" in ei.value.message
+    finally:
+        bf.set_wait_timeout_ms(600000)
+    got = bf.search_batch_noalloc(second)                   # waits for the timed-out call, then runs
+    assert [(r.index, r.makespan_us) for r in got] == want_second
+    got = bf.search_batch_noalloc(heavy, busy)
+    assert [(r.index, r.makespan_us) for r in got] == want_heavy
 
 
 def test_noalloc_rejects_oversized_batch():
