@@ -15,9 +15,11 @@ scenario from host tables, search, result back on the host, release).
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl bf|reference]
 
 With --impl reference the CPU oracle is timed instead (rank 0 only), on
-bounded samples of the same workload.  Under torchrun each rank searches the
-same scenario independently (replicas, no collective on the data path); the
-step time is the max over ranks.
+bounded samples of the same workload.  Under torchrun (N > 1) one step is
+still one search of all 3^19 mappings, split into N contiguous index ranges
+(bf_search_range on each rank's GPU) and reduced by one all-gather of an
+8-byte key per rank; the step time is the max over ranks and `value` counts
+the 3^19 mappings once (strong scaling).
 """
 from __future__ import annotations
 
@@ -42,32 +44,43 @@ WORKLOAD = ("config3: N=19 tools (spine of 7 + two fan-outs of 6; 11 GPU-preferr
 # N-wide next-completion scan and an N-wide readiness scan (2 N^2).
 N_TOOLS = 19
 OPS_PER_MAPPING = 2 * N_TOOLS * N_TOOLS
-INT_LANES_PER_SM = 128  # 4 SMSPs x 32 lanes issue one integer op each per clock
+INT_LANES_PER_SM = 128  # 4 SMSPs x 32 lanes: one thread instruction each per clock at full issue
+
+# Committed ncu summaries of the enumerating kernels, one per standard workload.
+PROFILES = {"config0": "search_kernel_config0_n8.md", "config1": "search_kernel_config1_n12.md",
+            "config2": "search_kernel_config2_n16.md", "config3": "search_kernel_config3_n19.md",
+            "config4_batch": "batch_kernel_config4.md"}
+PROFILE_KEYS = ("source_fingerprint", "dram_bytes_per_launch", "thread_instructions_per_mapping", "issue_active",
+                "warp_efficiency", "kernel_ms")
 
 
-PROFILE_SUMMARY = os.path.join(ROOT, "profiles", "search_kernel_config3_n19.md")
-
-
-def profiled_fields():
-    """Fields of the committed ncu summary of the search kernel (DRAM bytes per launch, executed
-    thread instructions per mapping, issue-slot utilisation), or {} when the search kernel's
-    translation unit changed since that capture."""
+def profiled_fields(workload: str = "config3"):
+    """Fields of the committed ncu summary of `workload`'s kernel (DRAM bytes per launch, executed
+    thread instructions per mapping, issue-slot utilisation, warp execution efficiency), or {} when
+    the summary is missing or the enumerating kernels' translation unit changed since that capture."""
     from paper_2607_22242_gb300 import _build
     try:
-        text = open(PROFILE_SUMMARY).read()
+        text = open(os.path.join(ROOT, "profiles", PROFILES[workload])).read()
     except OSError:
         return {}
-    keys = ("source_fingerprint", "dram_bytes_per_launch", "thread_instructions_per_mapping", "issue_active")
-    fields = dict(line.split(": ", 1) for line in text.splitlines() if line.startswith(tuple(k + ": " for k in keys)))
+    fields = dict(line.split(": ", 1) for line in text.splitlines()
+                  if line.startswith(tuple(k + ": " for k in PROFILE_KEYS)))
     if fields.get("source_fingerprint", "").strip() != _build.kernel_fingerprint():
         return {}
-    return fields
+    return {k: v.strip() for k, v in fields.items()}
 
 
-def profiled_traffic():
-    """DRAM bytes per launch of the search kernel from the committed ncu summary, or None when stale."""
-    f = profiled_fields()
-    return int(f["dram_bytes_per_launch"]) if "dram_bytes_per_launch" in f else None
+def issue_roofline(fields, mappings_per_s: float, peak_ops: float):
+    """The instruction-issue roofline of one workload: executed thread instructions per mapping (ncu) x
+    mappings/s against SMs x 128 lanes x clock, with the ncu issue-slot share and warp efficiency."""
+    if "thread_instructions_per_mapping" not in fields:
+        return {}
+    inst = float(fields["thread_instructions_per_mapping"])
+    out = {"thread_instructions_per_mapping": inst, "issue_frac": inst * mappings_per_s / peak_ops}
+    for key, name in (("issue_active", "issue_active_frac"), ("warp_efficiency", "warp_efficiency")):
+        if key in fields:
+            out[name] = float(fields[key])
+    return out
 
 
 def dist_env():
@@ -310,6 +323,15 @@ def oracle_single_core(S, seconds_per_config: float = 1.5):
     return out
 
 
+def sharded_step(search_range, total: int):
+    """The multi-GPU step: this rank searches its contiguous share of [0, total) with
+    ``search_range(first, count) -> (index, makespan, feasible)``, then one all-gather of one 8-byte key
+    per rank gives the optimum (index, makespan) of the whole space on every rank."""
+    from paper_2607_22242_gb300 import shard
+    idx, ms, _ = shard.sharded_search(search_range, total)
+    return idx, ms
+
+
 def run_gpu(args):
     import torch
     rank, world, local = dist_env()
@@ -325,11 +347,24 @@ def run_gpu(args):
     __graft_entry__.build()
     from paper_2607_22242_gb300 import bf
     from paper_2607_22242_gb300 import scenarios as S
+    from paper_2607_22242_gb300 import shard
 
     scn = S.config3()
     total = 3 ** scn.n
+    with open(os.path.join(ROOT, "tests", "golden", "config_results.json")) as fh:
+        summ = json.load(fh)["configs"]["3"]["summary"]
+    want = (summ["best_index"], summ["best_makespan"])
     stream = torch.cuda.current_stream()
     flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.int32, device="cuda")  # > 129 MB L2
+
+    def search_step(handle):
+        """One search of all 3^19 mappings: on one GPU the whole space (bf_search_best); on N ranks
+        each searches its contiguous index range (bf_search_range) and one all-gather of 8-byte keys
+        gives every rank the optimum."""
+        if world == 1:
+            r = bf.search_best(handle, stream)
+            return r.index, r.makespan_us
+        return sharded_step(shard.gpu_search_range(handle, stream), total)
 
     def barrier():
         if world > 1:
@@ -338,29 +373,29 @@ def run_gpu(args):
 
     h = bf.create_scenario(scn)
     for _ in range(args.warmup):
-        res = bf.search_best(h, stream)
+        res = search_step(h)
+    assert res == want, (res, want)
 
     # ---- timed region: K full searches, L2 flushed between them -------------
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     sampler = ClockSampler(device_id_for_smi(torch, dev))
+    results = []
     with sampler:
         barrier()
         wall0 = time.perf_counter()
         for i in range(args.steps):
             flush.zero_()
             starts[i].record(stream)
-            res = bf.search_best(h, stream)
+            results.append(search_step(h))
             ends[i].record(stream)
         barrier()
         wall = time.perf_counter() - wall0
+    assert all(r == want for r in results), results
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
     mean_ms = statistics.mean(step_ms)
-    worst_ms = mean_ms
-    if world > 1:
-        from paper_2607_22242_gb300 import shard
-        worst_ms = shard.max_over_ranks(mean_ms)
-    value = world * total / (worst_ms / 1e3)
+    worst_ms = shard.max_over_ranks(mean_ms) if world > 1 else mean_ms
+    value = total / (worst_ms / 1e3)  # the 3^19 mappings of one search, counted once
     clocks = sampler.summary()
 
     # ---- end to end through the host-buffer API ------------------------------
@@ -369,35 +404,38 @@ def run_gpu(args):
     for _ in range(max(3, args.steps // 4)):
         t0 = time.perf_counter()
         with bf.create_scenario(scn) as h2:       # host tables in, validated, scratch allocated
-            r2 = bf.search_best(h2, stream)       # tables travel with the launch; 8-byte key back
+            r2 = search_step(h2)                   # tables travel with the launch; 8-byte key back
         e2e_times.append(time.perf_counter() - t0)
-        assert (r2.index, r2.makespan_us) == (res.index, res.makespan_us)
-    e2e_value = world * total / statistics.mean(e2e_times)
+        assert r2 == want
+    e2e_mean = statistics.mean(e2e_times)
+    if world > 1:
+        e2e_mean = shard.max_over_ranks(e2e_mean)
+    e2e_value = total / e2e_mean
 
-    # ---- the same optimum by branch and bound (reported beside, not as `value`) ---
-    pruned_ms = []
-    for _ in range(max(3, args.steps // 4)):
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        rp = bf.search_pruned(h, None, stream)
-        b.record(stream)
-        b.synchronize()
-        pruned_ms.append(a.elapsed_time(b))
-        assert (rp.index, rp.makespan_us) == (res.index, res.makespan_us)
+    extras = {}
+    if world == 1:
+        # ---- the same optimum by branch and bound (reported beside, not as `value`) ---
+        pruned_ms = []
+        for _ in range(max(3, args.steps // 4)):
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            rp = bf.search_pruned(h, None, stream)
+            b.record(stream)
+            b.synchronize()
+            pruned_ms.append(a.elapsed_time(b))
+            assert (rp.index, rp.makespan_us) == want
+        # ---- host wall time of the blocking call, scenario already created ----------
+        host_ms = []
+        for _ in range(10):
+            t0 = time.perf_counter()
+            bf.search_best(h, stream)
+            host_ms.append((time.perf_counter() - t0) * 1e3)
+        extras = {"pruned_ms": pruned_ms, "host_ms": host_ms,
+                  # ---- every standard workload, and beyond 20 tools the tree search ---------
+                  "per_config": per_config_times(torch, bf, S, stream),
+                  "tree": tree_search_times(torch, bf, S, stream),
+                  "modes": bf.search_best(h, stream).modes}
     h.close()
-
-    # ---- host wall time of the blocking call, scenario already created ----------
-    h = bf.create_scenario(scn)
-    host_ms = []
-    for _ in range(10):
-        t0 = time.perf_counter()
-        bf.search_best(h, stream)
-        host_ms.append((time.perf_counter() - t0) * 1e3)
-    h.close()
-
-    # ---- every standard workload, and beyond 20 tools the tree search ---------------
-    per_config = per_config_times(torch, bf, S, stream)
-    tree = tree_search_times(torch, bf, S, stream)
 
     if rank != 0:
         torch.distributed.destroy_process_group()
@@ -406,45 +444,60 @@ def run_gpu(args):
     sm_count = torch.cuda.get_device_properties(dev).multi_processor_count
     clk_mhz = clocks["sm_mhz"] or 2070.0
     peak_ops = sm_count * INT_LANES_PER_SM * clk_mhz * 1e6
-    achieved_ops = OPS_PER_MAPPING * total / (mean_ms / 1e3)
-    roofline = {"bound": "alu", "achieved": achieved_ops / 1e12, "peak": peak_ops / 1e12, "unit": "Tops/s",
-                "frac": achieved_ops / peak_ops, "traffic": profiled_traffic(),
-                "peak_basis": f"{sm_count} SMs x {INT_LANES_PER_SM} int lanes x "
-                              f"{clk_mhz:.0f} MHz ({'sampled median under load' if clocks['sm_mhz'] else 'max clock, no samples'})",
-                "ops_per_mapping": OPS_PER_MAPPING}
-    prof = profiled_fields()
-    if prof:
-        roofline["executed_thread_instructions_per_mapping"] = float(prof["thread_instructions_per_mapping"])
-        roofline["issue_active_frac"] = float(prof["issue_active"])
-    roofline["note"] = ("achieved counts the naive per-mapping work (2 N^2 integer ops for a from-scratch "
-                        "simulation); the enumeration resumes each mapping from checkpoints shared with its "
-                        "neighbours, so it executes fewer instructions per mapping and frac can exceed 1; "
-                        "issue_active_frac is the measured share of issue slots used (ncu)")
+    per_gpu = value / world  # mappings/s of one GPU's kernel
+    prof = profiled_fields("config3")
+    issue = issue_roofline(prof, per_gpu, peak_ops)
+    roofline = {"bound": "alu",
+                "achieved": issue["thread_instructions_per_mapping"] * per_gpu / 1e12 if issue else None,
+                "peak": peak_ops / 1e12, "unit": "T thread-instructions/s",
+                "frac": issue.get("issue_frac"),
+                "traffic": int(prof["dram_bytes_per_launch"]) if "dram_bytes_per_launch" in prof else None,
+                "peak_basis": f"{sm_count} SMs x {INT_LANES_PER_SM} lanes (4 SMSPs x 32) x "
+                              f"{clk_mhz:.0f} MHz ({'sampled median under load' if clocks['sm_mhz'] else 'max clock, no samples'}); "
+                              "derived from unit counts and the sampled clock (no integer peak is measured)",
+                "executed_thread_instructions_per_mapping": issue.get("thread_instructions_per_mapping"),
+                "issue_active_frac": issue.get("issue_active_frac"),
+                "warp_efficiency": issue.get("warp_efficiency"),
+                "algorithmic_ops_per_mapping": OPS_PER_MAPPING,
+                "algorithmic_frac": OPS_PER_MAPPING * per_gpu / peak_ops,
+                "note": ("frac = executed thread instructions per mapping (ncu, committed summary whose kernel "
+                         "fingerprint matches the built kernels; null when stale) x mappings/s / peak; "
+                         "algorithmic_frac counts 2 N^2 integer ops per mapping (a from-scratch simulation), "
+                         "which the checkpointed enumeration does not execute")}
 
     out = {"metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-           "warmup": args.warmup, "ms_per_step": mean_ms, "higher_is_better": True, "scaling": "weak",
+           "warmup": args.warmup, "ms_per_step": worst_ms, "higher_is_better": True,
+           "scaling": "strong" if world > 1 else "weak",
            "vs_baseline": None, "dtype": "u32", "data": "synthetic",
-           "config": {"workload": WORKLOAD, "mappings_per_step": total, "parallelism": f"replicas x{world}",
+           "config": {"workload": WORKLOAD, "mappings_per_step": total,
+                      "parallelism": f"index-range shards x{world}" if world > 1 else "single GPU",
                       "l2": "flushed between steps (256 MiB write, outside the timed events)"},
            "wall_time_to_optimum_ms": {"median": statistics.median(step_ms), "min": min(step_ms),
-                                       "max": max(step_ms),
-                                       "host_median": statistics.median(host_ms),
-                                       "host_note": "bf_search_best call as seen by the host (blocks until the "
-                                                    "result is in pinned host memory), median of 10"},
-           "per_config": per_config,
-           "pruned_wall_time_to_optimum_ms": {
-               "median": statistics.median(pruned_ms), "min": min(pruned_ms),
-               "note": "bf_search_pruned: exact branch and bound, same optimum; not a full enumeration"},
-           "result": {"index": res.index, "makespan_us": res.makespan_us, "modes": res.modes},
-           "tree_search": tree,
+                                       "max": max(step_ms)},
+           "result": {"index": want[0], "makespan_us": want[1], "checked": "equals the oracle's stored optimum"},
            "roofline": roofline,
            "e2e": {"value": e2e_value, "unit": UNIT, "h2d_bytes_per_step": ctypes.sizeof(bf.Desc),
                    "d2h_bytes_per_step": 8,
-                   "path": "bf_create_scenario(host desc) + bf_search_best + bf_destroy_scenario",
-                   "bytes_note": "in: the step's input, one bf_scenario_desc (its derived tables reach the GPU "
-                                 "as kernel parameters); out: the 8-byte result key"},
-           "gpu_launches": args.steps,  # one search kernel per timed step
+                   "path": "bf_create_scenario(host desc) + " + ("bf_search_best" if world == 1 else
+                           "bf_search_range on each rank's index range + all-gather of 8-byte keys") +
+                           " + bf_destroy_scenario",
+                   "bytes_note": "in: the step's input, one bf_scenario_desc per GPU (its derived tables reach "
+                                 "the GPU as kernel parameters); out: the 8-byte result key"},
+           "gpu_launches": args.steps,  # one search kernel per timed step (per GPU)
            "clocks": clocks, "timed_wall_s": wall, "sm_count": sm_count}
+    if world == 1:
+        for name, entry in extras["per_config"].items():
+            entry.update(issue_roofline(profiled_fields(name), entry["mappings_per_s"], peak_ops))
+        out["wall_time_to_optimum_ms"].update(
+            host_median=statistics.median(extras["host_ms"]),
+            host_note="bf_search_best call as seen by the host (blocks until the result is in pinned host "
+                      "memory), median of 10")
+        out["per_config"] = extras["per_config"]
+        out["pruned_wall_time_to_optimum_ms"] = {
+            "median": statistics.median(extras["pruned_ms"]), "min": min(extras["pruned_ms"]),
+            "note": "bf_search_pruned: exact branch and bound, same optimum; not a full enumeration"}
+        out["tree_search"] = extras["tree"]
+        out["result"]["modes"] = extras["modes"]
     if world == 1 and not args.no_cpu_baseline:
         import oracle
         oracle.build()

@@ -119,3 +119,49 @@ def test_sharded_batch_equals_single_process(count, world):
     want = [(int(i), int(m), True) for i, m in zip(idx, ms)]
     for rank, got in results:
         assert got == want, rank
+
+
+def _bench_worker(rank, world, port, out):
+    import torch.distributed as dist
+    import oracle
+    import bench
+    from paper_2607_22242_gb300 import scenarios as S
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port))
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        scn = S.config(1)
+        total = 3 ** scn.n
+        seen = []
+
+        def search_range(first, count):
+            seen.append((first, count))
+            idx, ms = oracle.search_range(scn, first, count)
+            return (idx, ms, True) if idx >= 0 else (first, shard.INFEASIBLE, False)
+        out.put((rank, bench.sharded_step(search_range, total), seen))
+    finally:
+        dist.destroy_process_group()
+
+
+def test_bench_sharded_step_two_ranks():
+    """The benchmark's multi-GPU step with the oracle standing in for each rank's GPU range search:
+    two ranks search the two halves of the 12-tool workload's index space, once each, and both get
+    the single-process optimum."""
+    import oracle
+    from paper_2607_22242_gb300 import scenarios as S
+    oracle.build()
+    ctx = mp.get_context("spawn")
+    out = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_bench_worker, args=(r, 2, port, out)) for r in range(2)]
+    for p in procs:
+        p.start()
+    results = sorted(out.get(timeout=120) for _ in range(2))
+    for p in procs:
+        p.join(timeout=60)
+        assert p.exitcode == 0
+    scn = S.config(1)
+    want = oracle.search(scn)
+    total = 3 ** scn.n
+    assert [seen for _, _, seen in results] == [[shard.shard_range(total, r, 2)] for r in range(2)]
+    for rank, got, _ in results:
+        assert got == want, rank
