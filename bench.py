@@ -49,7 +49,9 @@ INT_LANES_PER_SM = 128  # 4 SMSPs x 32 lanes: one thread instruction each per cl
 # Committed ncu summaries of the enumerating kernels, one per standard workload.
 PROFILES = {"config0": "search_kernel_config0_n8.md", "config1": "search_kernel_config1_n12.md",
             "config2": "search_kernel_config2_n16.md", "config3": "search_kernel_config3_n19.md",
-            "config4_batch": "batch_kernel_config4.md"}
+            "config4_batch": "lanetree_kernel_config4.md"}
+# Translation unit each summary's fingerprint covers (_build.kernel_fingerprint).
+PROFILE_UNITS = {"config4_batch": "LANETREE_UNIT"}
 PROFILE_KEYS = ("source_fingerprint", "dram_bytes_per_launch", "thread_instructions_per_mapping", "issue_active",
                 "warp_efficiency", "kernel_ms")
 
@@ -65,7 +67,8 @@ def profiled_fields(workload: str = "config3"):
         return {}
     fields = dict(line.split(": ", 1) for line in text.splitlines()
                   if line.startswith(tuple(k + ": " for k in PROFILE_KEYS)))
-    if fields.get("source_fingerprint", "").strip() != _build.kernel_fingerprint():
+    unit = getattr(_build, PROFILE_UNITS.get(workload, "KERNEL_UNIT"))
+    if fields.get("source_fingerprint", "").strip() != _build.kernel_fingerprint(unit=unit):
         return {}
     return {k: v.strip() for k, v in fields.items()}
 

@@ -61,12 +61,18 @@ def _code_only(text: str) -> str:
     return " ".join(text.split())
 
 
-def kernel_fingerprint(csrc: str = CSRC) -> str:
-    """Hash of the enumerating kernels' code (comments and layout ignored) and flags: a profile
-    taken of those kernels stays valid while this is unchanged (changes elsewhere in the library,
-    or to comments, do not touch them)."""
+# Sources of the lane-tree batch kernel's translation unit.
+LANETREE_UNIT = ("bf_lanetree.cu", "bf_lanetree.cuh", "bf_lanetree_launch.h", "bf_enum.cuh", "bf_sim.cuh",
+                 "bf_launch.h")
+
+
+def kernel_fingerprint(csrc: str = CSRC, unit=KERNEL_UNIT) -> str:
+    """Hash of a kernel translation unit's code (comments and layout ignored) and flags -- by default
+    the enumerating kernels', LANETREE_UNIT for the lane-tree batch kernel: a profile taken of those
+    kernels stays valid while this is unchanged (changes elsewhere in the library, or to comments,
+    do not touch them)."""
     h = hashlib.sha256()
-    for name in KERNEL_UNIT:
+    for name in unit:
         with open(os.path.join(csrc, name), encoding="utf-8") as fh:
             h.update(name.encode() + _code_only(fh.read()).encode())
     flags = [f for f in NVCC_FLAGS if not f.startswith("-I")]
@@ -89,7 +95,7 @@ def build(force: bool = False, extra_flags=(), verbose: bool = False) -> str:
         obj = os.path.join(BUILD_DIR, f"bf_kernels_nw{nt}.o")
         jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, f"-DBF_NW={nt}", "-c",
                      os.path.join(CSRC, "bf_kernels.cu"), "-o", obj])
-    for unit in ("bf_tree", "bf_capi", "bf_capi_tree"):
+    for unit in ("bf_tree", "bf_lanetree", "bf_capi", "bf_capi_tree"):
         jobs.append([cc, *ARCH, *NVCC_FLAGS, *extra_flags, "-c", os.path.join(CSRC, unit + ".cu"), "-o",
                      os.path.join(BUILD_DIR, unit + ".o")])
 

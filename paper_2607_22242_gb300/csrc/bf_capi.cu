@@ -31,6 +31,7 @@ using bfk::host::batch_plan;
 using bfk::host::batch_split;
 using bfk::host::kSearchTasks;
 using bfk::host::whole_space_tables;
+using bfk::host::lanetree_record;
 
 thread_local std::string g_error;
 std::atomic<uint32_t> g_wait_timeout_ms{600000};
@@ -177,57 +178,118 @@ void fill_result(unsigned long long key, uint32_t n, uint64_t first, bf_result* 
     default: { e = cudaErrorInvalidValue; } break; \
   }
 
-// Records (tables, window tables, plan) of descs[0, count), built on up to 16
-// host threads (about half a microsecond per scenario); the largest window,
-// task count and whether any plan has an inner level are returned too.
-void build_records(const bf_scenario_desc* descs, uint32_t count, bfk::BatchRecord* recs, uint32_t* wmax,
-                   uint32_t* pmax, uint32_t* any_inner) {
+// Run work(lo, hi, &parts[t]) over [0, count) on up to 16 host threads (a
+// thread is worth starting for a few hundred scenarios; about half a
+// microsecond of host work per scenario); parts gets one entry per thread.
+template <typename Part, typename Work>
+void parallel_parts(uint32_t count, std::vector<Part>& parts, Work work) {
+  const unsigned hw = std::thread::hardware_concurrency();
+  uint32_t nthreads = count / 256u;
+  if (nthreads > 16u) nthreads = 16u;
+  if (hw && nthreads > hw) nthreads = hw;
+  parts.assign(nthreads > 1 ? nthreads : 1, Part{});
+  if (nthreads <= 1) {
+    work(0u, count, &parts[0]);
+    return;
+  }
+  std::vector<std::thread> pool;
+  bool threads_ok = true;
+  try {
+    for (uint32_t t = 0; t < nthreads; ++t)
+      pool.emplace_back(work, (uint32_t)((uint64_t)count * t / nthreads),
+                        (uint32_t)((uint64_t)count * (t + 1) / nthreads), &parts[t]);
+  } catch (const std::exception&) {
+    threads_ok = false;  // no more threads: finish on this one
+  }
+  for (auto& th : pool) th.join();
+  if (!threads_ok) {
+    parts.assign(1, Part{});
+    work(0u, count, &parts[0]);
+  }
+}
+
+// Batch-kernel records (tables, window tables, plan) of descs[ids[j]], j <
+// count; the largest window, task count and whether any plan has an inner
+// level are returned too.
+void build_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count, bfk::BatchRecord* recs,
+                   uint32_t* wmax, uint32_t* pmax, uint32_t* any_inner) {
   struct Part {
     uint32_t wmax = 0, pmax = 0, inner = 0;
   };
-  auto work = [&](uint32_t lo, uint32_t hi, Part* part) {
-    for (uint32_t i = lo; i < hi; ++i) {
-      bfk::BatchRecord& r = recs[i];
+  std::vector<Part> parts;
+  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part* part) {
+    for (uint32_t j = lo; j < hi; ++j) {
+      bfk::BatchRecord& r = recs[j];
       std::memset(&r, 0, sizeof r);
       bfk::Plan base;
-      batch_split(descs + i, &r.full, &base, &r.window);
-      r.plan = batch_plan(base, descs[i].n, bfk::kThreads / 32);
+      batch_split(descs + ids[j], &r.full, &base, &r.window);
+      r.plan = batch_plan(base, descs[ids[j]].n, bfk::kThreads / 32);
       r.mid_lanes = base.W0 == 0u ? 1u : 0u;
       if (r.window.n > part->wmax) part->wmax = r.window.n;
       const uint32_t tasks = r.plan.groups * r.plan.m_parts;
       if (tasks > part->pmax) part->pmax = tasks;
       part->inner |= r.plan.I;
     }
-  };
-  const unsigned hw = std::thread::hardware_concurrency();
-  uint32_t nthreads = count / 256u;  // a thread is worth starting for a few hundred scenarios
-  if (nthreads > 16u) nthreads = 16u;
-  if (hw && nthreads > hw) nthreads = hw;
-  std::vector<Part> parts(nthreads > 1 ? nthreads : 1);
-  if (nthreads <= 1) {
-    work(0, count, &parts[0]);
-  } else {
-    std::vector<std::thread> pool;
-    bool threads_ok = true;
-    try {
-      for (uint32_t t = 0; t < nthreads; ++t)
-        pool.emplace_back(work, (uint32_t)((uint64_t)count * t / nthreads),
-                          (uint32_t)((uint64_t)count * (t + 1) / nthreads), &parts[t]);
-    } catch (const std::exception&) {
-      threads_ok = false;  // no more threads: finish on this one
-    }
-    for (auto& th : pool) th.join();
-    if (!threads_ok) {
-      parts.assign(1, Part{});
-      work(0, count, &parts[0]);
-    }
-  }
+  });
   for (const Part& p : parts) {
     *wmax = p.wmax > *wmax ? p.wmax : *wmax;
     *pmax = p.pmax > *pmax ? p.pmax : *pmax;
     *any_inner |= p.inner;
   }
 }
+
+// Lane-tree records of descs[ids[j]], j < count.
+void build_lanetree_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count,
+                            bfk::LaneTreeRecord* recs) {
+  struct Part {};
+  std::vector<Part> parts;
+  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part*) {
+    for (uint32_t j = lo; j < hi; ++j) lanetree_record(descs + ids[j], recs + j);
+  });
+}
+
+// Where a batch's scenarios go: up to kLtBatchTools tools the lane-tree
+// kernel (bf_lanetree.cuh), above it the batch kernel (bf_kernels.cu).  The
+// keys of the first group come first in the key array.
+struct BatchSplit {
+  uint32_t ns = 0, nl = 0;            // scenarios in each group
+  uint32_t nmax_small = 0, nmax_large = 0;
+};
+
+template <typename Ids>
+BatchSplit split_batch(const bf_scenario_desc* descs, uint32_t count, Ids& small, Ids& large) {
+  BatchSplit b;
+  for (uint32_t i = 0; i < count; ++i) {
+    const uint32_t n = descs[i].n;
+    if (n <= bfk::kLtBatchTools) {
+      small[b.ns++] = i;
+      b.nmax_small = n > b.nmax_small ? n : b.nmax_small;
+    } else {
+      large[b.nl++] = i;
+      b.nmax_large = n > b.nmax_large ? n : b.nmax_large;
+    }
+  }
+  return b;
+}
+
+// Launch both groups of a batch on `st` (records already on the device; keys
+// reset to ~0): keys[0, ns) for the lane-tree group, keys[ns, ns + nl) for
+// the other.
+cudaError_t launch_batch_groups(const BatchSplit& b, const bfk::LaneTreeRecord* d_lt, const uint32_t* d_first_block,
+                                uint32_t lt_blocks, const bfk::BatchRecord* d_bk, uint32_t wmax, uint32_t pmax,
+                                uint32_t any_inner, unsigned long long* d_keys, cudaStream_t st) {
+  cudaError_t e = cudaSuccess;
+  if (b.ns) e = bfk::launch_lanetree(d_lt, d_first_block, b.ns, lt_blocks, b.nmax_small, d_keys, st);
+  if (e == cudaSuccess && b.nl) {
+    const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
+#define CALL(NW) launch_batch_nw##NW(d_bk, b.nl, b.nmax_large, any_inner, bps, d_keys + b.ns, st)
+    BF_DISPATCH(bfk::bucket_for(wmax), CALL)
+#undef CALL
+  }
+  return e;
+}
+
+inline size_t align256(size_t x) { return (x + 255) / 256 * 256; }
 
 // Index-list evaluation: the 20-slot kernels up to 20 tools, the 32-slot one above.
 cudaError_t launch_list(const bf_scenario* scn, const uint64_t* idx, uint64_t count, uint32_t* ms, uint8_t* fe,
@@ -551,32 +613,41 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
 static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
   if (count == 0) return BF_OK;
   if (!descs || !out) return fail(BF_EINVAL, "bf_search_batch: NULL argument");
-  uint32_t nmax = 0;
   for (uint32_t i = 0; i < count; ++i) {
     int rc = validate(descs + i, "bf_search_batch");
     if (rc == BF_OK) rc = require_enum(descs[i], "bf_search_batch");
     if (rc != BF_OK) return fail(rc, "bf_search_batch: descs[%u]: %s", i, g_error.c_str());
-    if (descs[i].n > nmax) nmax = descs[i].n;
   }
-  std::vector<bfk::BatchRecord> recs(count);
+  std::vector<uint32_t> small(count), large(count);
+  const BatchSplit b = split_batch(descs, count, small, large);
+  std::vector<bfk::LaneTreeRecord> lt(b.ns);
+  std::vector<uint32_t> first_block(b.ns + 1, 0u);
+  std::vector<bfk::BatchRecord> bk(b.nl);
+  build_lanetree_records(descs, small.data(), b.ns, lt.data());
+  for (uint32_t j = 0; j < b.ns; ++j) first_block[j + 1] = first_block[j] + lt[j].nblocks;
   uint32_t wmax = 0, pmax = 0, any_inner = 0;
-  build_records(descs, count, recs.data(), &wmax, &pmax, &any_inner);
+  build_records(descs, large.data(), b.nl, bk.data(), &wmax, &pmax, &any_inner);
+
+  // One device allocation: lane-tree records, their first blocks, batch
+  // records, keys.
+  const size_t lt_bytes = sizeof(bfk::LaneTreeRecord) * b.ns, fb_bytes = sizeof(uint32_t) * (b.ns + 1);
+  const size_t bk_bytes = sizeof(bfk::BatchRecord) * b.nl, kbytes = sizeof(unsigned long long) * count;
+  const size_t off_fb = align256(lt_bytes), off_bk = off_fb + align256(fb_bytes), off_keys = off_bk + align256(bk_bytes);
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
-  bfk::BatchRecord* d_recs = nullptr;
-  unsigned long long* d_keys = nullptr;
+  unsigned char* d_base = nullptr;
   std::vector<unsigned long long> keys(count);
-  const size_t rbytes = sizeof(bfk::BatchRecord) * count, kbytes = sizeof(unsigned long long) * count;
-  cudaError_t e = lib_malloc(reinterpret_cast<void**>(&d_recs), rbytes);
-  if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&d_keys), kbytes);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(d_recs, recs.data(), rbytes, cudaMemcpyHostToDevice, st);
+  cudaError_t e = lib_malloc(reinterpret_cast<void**>(&d_base), off_keys + kbytes);
+  auto* d_lt = reinterpret_cast<bfk::LaneTreeRecord*>(d_base);
+  auto* d_fb = reinterpret_cast<uint32_t*>(d_base + off_fb);
+  auto* d_bk = reinterpret_cast<bfk::BatchRecord*>(d_base + off_bk);
+  auto* d_keys = reinterpret_cast<unsigned long long*>(d_base + off_keys);
+  if (e == cudaSuccess && b.ns) e = cudaMemcpyAsync(d_lt, lt.data(), lt_bytes, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && b.ns) e = cudaMemcpyAsync(d_fb, first_block.data(), fb_bytes, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && b.nl) e = cudaMemcpyAsync(d_bk, bk.data(), bk_bytes, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, kbytes, st);
+  if (e == cudaSuccess)
+    e = launch_batch_groups(b, d_lt, d_fb, first_block[b.ns], d_bk, wmax, pmax, any_inner, d_keys, st);
   int rc = BF_OK;
-  if (e == cudaSuccess) {
-    const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
-#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, any_inner, bps, d_keys, st)
-    BF_DISPATCH(bfk::bucket_for(wmax), CALL)
-#undef CALL
-  }
   if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
   // Bounded wait first: a copy into pageable memory would block without limit.
   if (rc == BF_OK) rc = wait_stream(st, "bf_search_batch");
@@ -585,12 +656,11 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
   }
-  if (rc != BF_ETIMEOUT) {  // on timeout the kernel may still use the scratch: leak it rather than free in-use memory
-    if (d_recs) cudaFree(d_recs);
-    if (d_keys) cudaFree(d_keys);
-  }
+  // On timeout the kernels may still use the scratch: leak it rather than free in-use memory.
+  if (rc != BF_ETIMEOUT && d_base) cudaFree(d_base);
   if (rc != BF_OK) return rc;
-  for (uint32_t i = 0; i < count; ++i) fill_result(keys[i], descs[i].n, 0, out + i);
+  for (uint32_t j = 0; j < b.ns; ++j) fill_result(keys[j], descs[small[j]].n, 0, out + small[j]);
+  for (uint32_t j = 0; j < b.nl; ++j) fill_result(keys[b.ns + j], descs[large[j]].n, 0, out + large[j]);
   return BF_OK;
 }
 
@@ -606,8 +676,14 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
 
 namespace {
 
-constexpr size_t kNoAllocRecordBytes = sizeof(bfk::BatchRecord) * BF_NOALLOC_MAX_SCENARIOS;
-constexpr size_t kNoAllocKeyOffset = (kNoAllocRecordBytes + 255) / 256 * 256;
+// Regions of the array: lane-tree records, their first blocks, batch-kernel
+// records, keys; each sized for BF_NOALLOC_MAX_SCENARIOS scenarios.
+constexpr size_t kNoAllocFirstBlockOffset =
+    (sizeof(bfk::LaneTreeRecord) * BF_NOALLOC_MAX_SCENARIOS + 255) / 256 * 256;
+constexpr size_t kNoAllocRecordOffset =
+    kNoAllocFirstBlockOffset + (sizeof(uint32_t) * (BF_NOALLOC_MAX_SCENARIOS + 1) + 255) / 256 * 256;
+constexpr size_t kNoAllocKeyOffset =
+    kNoAllocRecordOffset + (sizeof(bfk::BatchRecord) * BF_NOALLOC_MAX_SCENARIOS + 255) / 256 * 256;
 constexpr size_t kNoAllocBytes = kNoAllocKeyOffset + sizeof(unsigned long long) * BF_NOALLOC_MAX_SCENARIOS;
 
 }  // namespace
@@ -703,40 +779,56 @@ int search_batch_noalloc_locked(NoAllocDevice& dv, const bf_scenario_desc* descs
     if (rc != BF_OK) return rc;
     dv.pending = false;
   }
-  bfk::BatchRecord* d_recs = reinterpret_cast<bfk::BatchRecord*>(dv.base);
-  unsigned long long* d_keys = reinterpret_cast<unsigned long long*>(dv.base + kNoAllocKeyOffset);
+  auto* d_lt = reinterpret_cast<bfk::LaneTreeRecord*>(dv.base);
+  auto* d_fb = reinterpret_cast<uint32_t*>(dv.base + kNoAllocFirstBlockOffset);
+  auto* d_bk = reinterpret_cast<bfk::BatchRecord*>(dv.base + kNoAllocRecordOffset);
+  auto* d_keys = reinterpret_cast<unsigned long long*>(dv.base + kNoAllocKeyOffset);
+  uint32_t small[BF_NOALLOC_MAX_SCENARIOS], large[BF_NOALLOC_MAX_SCENARIOS];
+  uint32_t first_block[BF_NOALLOC_MAX_SCENARIOS + 1];
+  const BatchSplit b = split_batch(descs, count, small, large);
 
-  // Pack the records a few at a time through a stack buffer (a copy from
+  // Pack the records a few at a time through stack buffers (a copy from
   // pageable memory has left the buffer when cudaMemcpyAsync returns).
   constexpr uint32_t kChunk = 8;
-  bfk::BatchRecord chunk[kChunk];
-  uint32_t nmax = 0, wmax = 0, pmax = 0, any_inner = 0;
   cudaError_t e = cudaSuccess;
-  for (uint32_t i0 = 0; i0 < count && e == cudaSuccess; i0 += kChunk) {
-    const uint32_t nrec = (count - i0 < kChunk) ? (count - i0) : kChunk;
-    for (uint32_t j = 0; j < nrec; ++j) {
-      bfk::BatchRecord& r = chunk[j];
-      std::memset(&r, 0, sizeof r);
-      bfk::Plan plan;
-      batch_split(descs + i0 + j, &r.full, &plan, &r.window);
-      r.plan = batch_plan(plan, descs[i0 + j].n, bfk::kThreads / 32);
-      r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
-      if (descs[i0 + j].n > nmax) nmax = descs[i0 + j].n;
-      if (r.window.n > wmax) wmax = r.window.n;
-      const uint32_t tasks = r.plan.groups * r.plan.m_parts;
-      if (tasks > pmax) pmax = tasks;
-      any_inner |= r.plan.I;
+  first_block[0] = 0u;
+  {
+    bfk::LaneTreeRecord chunk[kChunk];
+    for (uint32_t j0 = 0; j0 < b.ns && e == cudaSuccess; j0 += kChunk) {
+      const uint32_t nrec = (b.ns - j0 < kChunk) ? (b.ns - j0) : kChunk;
+      for (uint32_t j = 0; j < nrec; ++j) {
+        lanetree_record(descs + small[j0 + j], chunk + j);
+        first_block[j0 + j + 1] = first_block[j0 + j] + chunk[j].nblocks;
+      }
+      e = cudaMemcpyAsync(d_lt + j0, chunk, sizeof(bfk::LaneTreeRecord) * nrec, cudaMemcpyHostToDevice, st);
     }
-    e = cudaMemcpyAsync(d_recs + i0, chunk, sizeof(bfk::BatchRecord) * nrec, cudaMemcpyHostToDevice, st);
+  }
+  if (e == cudaSuccess && b.ns)
+    e = cudaMemcpyAsync(d_fb, first_block, sizeof(uint32_t) * (b.ns + 1), cudaMemcpyHostToDevice, st);
+  uint32_t wmax = 0, pmax = 0, any_inner = 0;
+  {
+    bfk::BatchRecord chunk[kChunk];
+    for (uint32_t j0 = 0; j0 < b.nl && e == cudaSuccess; j0 += kChunk) {
+      const uint32_t nrec = (b.nl - j0 < kChunk) ? (b.nl - j0) : kChunk;
+      for (uint32_t j = 0; j < nrec; ++j) {
+        bfk::BatchRecord& r = chunk[j];
+        std::memset(&r, 0, sizeof r);
+        bfk::Plan plan;
+        batch_split(descs + large[j0 + j], &r.full, &plan, &r.window);
+        r.plan = batch_plan(plan, descs[large[j0 + j]].n, bfk::kThreads / 32);
+        r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
+        if (r.window.n > wmax) wmax = r.window.n;
+        const uint32_t tasks = r.plan.groups * r.plan.m_parts;
+        if (tasks > pmax) pmax = tasks;
+        any_inner |= r.plan.I;
+      }
+      e = cudaMemcpyAsync(d_bk + j0, chunk, sizeof(bfk::BatchRecord) * nrec, cudaMemcpyHostToDevice, st);
+    }
   }
   // The keys keep the previous call's values: reset them to "nothing found".
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, sizeof(unsigned long long) * count, st);
-  if (e == cudaSuccess) {
-    const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
-#define CALL(NW) launch_batch_nw##NW(d_recs, count, nmax, any_inner, bps, d_keys, st)
-    BF_DISPATCH(bfk::bucket_for(wmax), CALL)
-#undef CALL
-  }
+  if (e == cudaSuccess)
+    e = launch_batch_groups(b, d_lt, d_fb, first_block[b.ns], d_bk, wmax, pmax, any_inner, d_keys, st);
   if (e != cudaSuccess) return cuda_fail(e, who);
   rc = wait_stream(st, who);
   if (rc == BF_ETIMEOUT) {
@@ -751,7 +843,10 @@ int search_batch_noalloc_locked(NoAllocDevice& dv, const bf_scenario_desc* descs
     e = cudaMemcpyAsync(keys, d_keys + i0, sizeof(unsigned long long) * nk, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return cuda_fail(e, who);
-    for (uint32_t j = 0; j < nk; ++j) fill_result(keys[j], descs[i0 + j].n, 0, out + i0 + j);
+    for (uint32_t j = 0; j < nk; ++j) {
+      const uint32_t k = i0 + j, i = k < b.ns ? small[k] : large[k - b.ns];
+      fill_result(keys[j], descs[i].n, 0, out + i);
+    }
   }
   return BF_OK;
 }

@@ -8,6 +8,7 @@
 #include <stdint.h>
 
 #include "../../include/bf.h"
+#include "bf_lanetree_launch.h"
 #include "bf_launch.h"
 #include "bf_plan.h"
 #include "bf_tree.h"

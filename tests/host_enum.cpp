@@ -13,6 +13,7 @@
 #define __forceinline__ inline
 using std::min;
 static inline int __popc(unsigned x) { return __builtin_popcount(x); }
+static inline int __ffs(unsigned x) { return __builtin_ffs((int)x); }
 static inline unsigned long long __umul64hi(unsigned long long a, unsigned long long b) {
   return (unsigned long long)(((unsigned __int128)a * b) >> 64);
 }
@@ -207,4 +208,48 @@ extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bo
   if (tw.n <= 10) return pruned_width<10>(tb, tw, plan);
   if (tw.n <= 14) return pruned_width<14>(tb, tw, plan);
   return pruned_width<20>(tb, tw, plan);
+}
+
+// The lane-tree batch kernel's search (bf_lanetree.cuh) of one scenario,
+// with the record bf_search_batch builds for it: every block of its roots
+// with `lanes` lanes, lane l taking the block's roots l, l + lanes, ...
+// (the kernel hands roots out from a shared counter; any order gives the
+// same mappings).  Every mapping reported to the sink is stored at its
+// canonical index; out[] starts at 0xFFFFFFFF (infeasible mappings are not
+// reported) and a second report of one index stores 0xDEADBEEF.
+// info[0..2] = x, y, blocks.
+extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint32_t* out, uint32_t* info) {
+  if (d->n > kLtBatchTools || lanes == 0) return -1;
+  LaneTreeRecord rec;
+  host::lanetree_record(d, &rec);
+  info[0] = rec.x;
+  info[1] = rec.y;
+  info[2] = rec.nblocks;
+  const uint64_t total = host::pow3(d->n), roots = host::pow3(rec.x);
+  for (uint64_t j = 0; j < total; ++j) out[j] = 0xFFFFFFFFu;
+  std::vector<LtShared> shared(1);
+  LtShared& S = shared[0];
+  S.rec = rec;
+  threadIdx.x = 0;
+  blockDim.x = 1;
+  lt_fill_tables(S);
+  struct Store {
+    uint32_t* out;
+    void operator()(uint32_t idx, uint32_t ms) { out[idx] = out[idx] == 0xFFFFFFFFu ? ms : 0xDEADBEEFu; }
+  } sink{out};
+  std::vector<uint32_t> rows((size_t)lt_rows(d->n) * lanes, 0xA5A5A5A5u);  // stale shared memory
+  for (uint32_t b = 0; b < rec.nblocks; ++b) {
+    const uint32_t r0 = (uint32_t)(roots * b / rec.nblocks), r1 = (uint32_t)(roots * (b + 1) / rec.nblocks);
+    for (uint32_t lane = 0; lane < lanes; ++lane) {
+      uint32_t next = r0 + lane;
+      lt_lane(S, rows.data() + lane, lanes,
+              [&]() {
+                const uint32_t r = next;
+                next += lanes;
+                return r < r1 ? r : 0xFFFFFFFFu;
+              },
+              sink);
+    }
+  }
+  return 0;
 }

@@ -45,6 +45,15 @@ def host():
         assert lib.host_eval(ctypes.byref(d), first, count, mode, ms.ctypes.data, info.ctypes.data) == 0
         return ms.astype(np.uint64), info
     run.pruned = lambda scn, bound: lib.host_pruned(ctypes.byref(bf.to_desc(scn)), bound)
+    lib.host_lanetree.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]
+    lib.host_lanetree.restype = ctypes.c_int
+
+    def lanetree(scn, lanes):
+        ms = np.zeros(3 ** scn.n, np.uint32)
+        info = np.zeros(3, np.uint32)
+        assert lib.host_lanetree(ctypes.byref(bf.to_desc(scn)), lanes, ms.ctypes.data, info.ctypes.data) == 0
+        return ms.astype(np.uint64), info
+    run.lanetree = lanetree
     return run
 
 
@@ -134,3 +143,47 @@ def test_tie_order_scenarios_host(host):
             key = host.pruned(scn, bound)
             got = (key & 0xFFFFFFFF, key >> 32) if key != 2 ** 64 - 1 else (-1, 0xFFFFFFFF)
             assert got == tuple(want), (t, bound, got, want)
+
+
+def _same_lanetree(host, scn, lanes):
+    got, info = host.lanetree(scn, lanes)
+    want, _ = oracle.eval_range(scn, 0, 3 ** scn.n, THREADS)
+    bad = np.flatnonzero(got != want)
+    assert bad.size == 0, (f"levels x={int(info[0])} y={int(info[1])}, {int(info[2])} blocks: {bad.size} "
+                           f"mismatches, first at index {int(bad[0])}: {int(got[bad[0]])} vs {int(want[bad[0]])}")
+    return info
+
+
+def test_lanetree_random_dags(host):
+    """The lane-tree batch search (roots, then up to two levels of checkpoints per lane) on random DAGs of
+    1-12 tools with small integer times, late sources and last tools that wait for all others: every
+    feasible mapping reported once, at its canonical index, with the oracle's makespan; infeasible ones
+    never; with 1, 3 and 32 lanes."""
+    rng = np.random.default_rng(92)
+    levels = set()
+    for t in range(200):
+        n = int(rng.integers(1, 13)) if t % 5 else int(rng.integers(8, 13))
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.25, 0.5, 0.8])), tight=bool(t % 3),
+                              contention=bool(t % 4), max_time=int(rng.choice([3, 7, 40, 2000])))
+        pred = list(base.pred_mask)
+        if t % 3 == 0 and n > 3:
+            pred[int(rng.integers(n // 2, n))] = 0
+        if t % 4 == 1 and n > 2:
+            pred[n - 1] = (1 << (n - 1)) - 1
+        scn = S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
+                         base.vram_budget_mib, base.slowdown_q10)
+        info = _same_lanetree(host, scn, (1, 3, 32)[t % 3])
+        levels.add(1 + (int(info[0]) < n) + (int(info[1]) < n))
+    assert levels == {1, 2, 3}, levels
+
+
+def test_lanetree_workloads_and_ties(host):
+    """The 8- and 12-tool workloads (the latter over several blocks), the first 48 scenarios of the
+    4096-scenario batch workload and the tie-order scenarios: every mapping against the oracle."""
+    for cfg in (0, 1):
+        info = _same_lanetree(host, S.config(cfg), 32)
+    assert int(info[2]) > 1  # the 12-tool workload's roots span several blocks
+    for scn in S.config4(48):
+        _same_lanetree(host, scn, 32)
+    for scn in tie_order_scenarios():
+        _same_lanetree(host, scn, 3)
