@@ -304,27 +304,28 @@ cudaError_t launch_list(const bf_scenario* scn, const uint64_t* idx, uint64_t co
   return e;
 }
 
+// One launch of the search kernel; its last warp writes the best key into the
+// host mirror (scn->h_scratch->search.key) and resets the launch state.
 int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result* out,
                cudaStream_t st, const char* who) {
-  cudaError_t e = cudaMemsetAsync(scn->d_key, 0xFF, sizeof(unsigned long long), st);
-  if (e != cudaSuccess) return cuda_fail(e, who);
-  if (count) {
-    // The whole space runs on the renumbered tables; a part of it keeps the
-    // scenario's numbering, in which an index range is a box of the split.
-    const bool whole = first == 0 && count == pow3(scn->desc.n);
-    const bfk::Tables& tb = whole ? scn->rtables : scn->tables;
-    const bfk::Tables& tw = whole ? scn->rwindow : scn->window;
-    const bfk::Plan plan = make_plan(whole ? scn->rplan : scn->plan, first, count, kSearchTasks);
-#define CALL(NW) launch_search_nw##NW(tb, tw, plan, scn->d_key, st)
-    BF_DISPATCH(bfk::bucket_for(tw.n), CALL)
-#undef CALL
-    if (e != cudaSuccess) return cuda_fail(e, who);
+  if (count == 0) {
+    fill_result(~0ull, scn->desc.n, first, out);
+    return BF_OK;
   }
-  e = cudaMemcpyAsync(scn->h_key, scn->d_key, sizeof(unsigned long long), cudaMemcpyDeviceToHost, st);
+  // The whole space runs on the renumbered tables; a part of it keeps the
+  // scenario's numbering, in which an index range is a box of the split.
+  const bool whole = first == 0 && count == pow3(scn->desc.n);
+  const bfk::Tables& tb = whole ? scn->rtables : scn->tables;
+  const bfk::Tables& tw = whole ? scn->rwindow : scn->window;
+  const bfk::Plan plan = make_plan(whole ? scn->rplan : scn->plan, first, count, kSearchTasks);
+  cudaError_t e = cudaSuccess;
+#define CALL(NW) launch_search_nw##NW(tb, tw, plan, &scn->d_scratch->search, scn->d_host_search_key, st)
+  BF_DISPATCH(bfk::bucket_for(tw.n), CALL)
+#undef CALL
   if (e != cudaSuccess) return cuda_fail(e, who);
   const int rc = wait_stream(st, who);
   if (rc != BF_OK) return rc;
-  fill_result(*scn->h_key, scn->desc.n, first, out);
+  fill_result(*static_cast<volatile unsigned long long*>(&scn->h_scratch->search.key), scn->desc.n, first, out);
   return BF_OK;
 }
 
@@ -362,6 +363,21 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   }
   s->d_key = &s->d_scratch->key;
   s->h_key = &s->h_scratch->key;
+  // The search kernel's launch state starts as (~0, 0, 0) and every launch
+  // leaves it so; its result goes to the pinned host mirror, which the
+  // device addresses directly.
+  void* mirror = nullptr;
+  e = cudaMemset(&s->d_scratch->search, 0, sizeof(bfk::SearchSync));
+  if (e == cudaSuccess) e = cudaMemset(&s->d_scratch->search.key, 0xFF, sizeof(unsigned long long));
+  if (e == cudaSuccess) e = cudaHostGetDevicePointer(&mirror, s->h_scratch, 0);
+  if (e != cudaSuccess) {
+    const int code = cuda_fail(e, "bf_create_scenario");
+    cudaFree(s->d_scratch);
+    cudaFreeHost(s->h_scratch);
+    delete s;
+    return code;
+  }
+  s->d_host_search_key = &static_cast<bf_scratch*>(mirror)->search.key;
   *out = s;
   return BF_OK;
 }

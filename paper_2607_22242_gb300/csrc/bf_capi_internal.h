@@ -17,6 +17,7 @@
 // the packed search key, the tree search's best record, bound and counters,
 // and the what-if probe list with its results.
 struct bf_scratch {
+  bfk::SearchSync search;  // the search kernel's launch state; search.key of the host mirror receives its result
   unsigned long long key;
   uint32_t survivors;   // pruned search: number of surviving prefixes
   uint32_t pruned_bound;  // pruned search: the incumbent's makespan (set with survivors)
@@ -49,6 +50,7 @@ struct bf_scenario {
   bf_scratch* h_scratch;      // pinned host mirror
   unsigned long long* d_key;  // &d_scratch->key
   unsigned long long* h_key;  // &h_scratch->key
+  unsigned long long* d_host_search_key;  // &h_scratch->search.key as the device addresses it
   uint32_t* d_survivors;      // pruned search: 3^pplan.P prefix slots, allocated on first use
   uint32_t* d_levels;         // tree search: node buffers of every level, allocated on first use
   size_t levels_bytes;

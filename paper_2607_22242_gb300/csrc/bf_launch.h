@@ -28,6 +28,16 @@ inline cudaError_t allow_dyn_smem(K kernel, size_t bytes, std::atomic<uint64_t>*
   return e;
 }
 
+// State of one launch of the search kernel, in device memory: the best key
+// found so far and the blocks that have finished.  It holds (~0, 0) between
+// launches: the last block of a launch writes the result out and puts it
+// back.
+struct SearchSync {
+  unsigned long long key;
+  uint32_t blocks_done;
+  uint32_t pad;
+};
+
 // One scenario of a batched search: its tables, its window tables and plan,
 // and how its warps assign lanes (0: a prefix per lane, warp_task; 1: a mid
 // combination per lane, mid_lane_task).
@@ -42,7 +52,7 @@ struct BatchRecord {
   cudaError_t launch_eval_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan, uint32_t* ms, \
                                  uint8_t* fe, cudaStream_t st);                                     \
   cudaError_t launch_search_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan,             \
-                                   unsigned long long* key, cudaStream_t st);                        \
+                                   SearchSync* sync, unsigned long long* host_key, cudaStream_t st);  \
   cudaError_t launch_batch_nw##NW(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,           \
                                   uint32_t any_inner, uint32_t blocks_per_scenario,                  \
                                   unsigned long long* keys, cudaStream_t st);                        \
