@@ -176,22 +176,23 @@ __device__ __forceinline__ uint32_t lt_step(const LtShared& S, LtState& s, uint3
   // ---- admission at T: newly ready tools start in index order -------------
   if (ready) {
     s.pend &= ~ready;
-    uint32_t qpos = 4u * __popc(s.qset);
-    for (uint32_t m = ready; m; m &= m - 1u) {
-      const uint32_t i = __ffs(m) - 1u, b = 1u << i;
-      const bool isq = (que & b) != 0u, isn = (now & b) != 0u;
+    // cpu: real end T + c; gpu_now: end stamp V + (g + x) * 1024
+    for (uint32_t m = ready & ~que; m; m &= m - 1u) {
+      const uint32_t i = __ffs(m) - 1u;
+      const bool isn = (now >> i) & 1u;
       const uint32_t w = R.dur[isn ? 1 : 0][i];
-      // cpu: real end T + c; gpu_now: end stamp V + (g + x) * 1024 (a queued
-      // tool's row is written when it starts)
       const uint32_t val = (isn ? s.V : s.T) + w;
       e[i * stride] = val;
       const bool first = isn && (!(s.run & gpu) || w < s.gm - s.V);
       s.gm = first ? val : s.gm;
-      s.tc = (isq || isn) ? s.tc : min(s.tc, val);
-      s.run |= isq ? 0u : b;
-      s.qset |= isq ? b : 0u;
-      s.qlist |= isq ? ((uint64_t)(i + 1u) << qpos) : 0ull;
-      qpos += isq ? 4u : 0u;
+      s.tc = isn ? s.tc : min(s.tc, val);
+      s.run |= 1u << i;
+    }
+    // queued: join the FIFO in index order (a row is written when the tool starts)
+    for (uint32_t m = ready & que; m; m &= m - 1u) {
+      const uint32_t i = __ffs(m) - 1u;
+      s.qlist |= (uint64_t)(i + 1u) << (4u * __popc(s.qset));
+      s.qset |= 1u << i;
     }
     if ((ready & now) && lt_vram(S, s.run & gpu) > R.budget) return kLtInfeasible;  // out of memory
   }
@@ -219,13 +220,16 @@ __device__ __forceinline__ uint32_t lt_step(const LtShared& S, LtState& s, uint3
   s.V = gpu_event ? s.gm : (k ? s.V + adv : s.V);
   s.T = gpu_event ? (uint32_t)tg : s.tc;
   // ---- retire everything that ends at T; the next CPU end and GPU stamp -----
-  // (a GPU tool can end only at a GPU event: at a CPU event V stays below
-  // every running GPU tool's stamp)
-  uint32_t ntc = 0xFFFFFFFFu, nrem = 0xFFFFFFFFu, ended = 0u;
-  for (uint32_t m = s.run; m; m &= m - 1u) {
+  // Only tools of the kinds that can end now are scanned: CPU tools when T
+  // reached the earliest CPU end, GPU tools at a GPU event (at a CPU event V
+  // stays below every running GPU tool's stamp); the other kind's earliest
+  // end is unchanged.
+  const bool cpu_event = s.tc == s.T;
+  uint32_t ntc = cpu_event ? 0xFFFFFFFFu : s.tc, nrem = gpu_event ? 0xFFFFFFFFu : s.gm - s.V, ended = 0u;
+  for (uint32_t m = (cpu_event ? s.run & ~gpu : 0u) | (gpu_event ? rg : 0u); m; m &= m - 1u) {
     const uint32_t i = __ffs(m) - 1u, b = 1u << i, end = e[i * stride];
     const bool isc = (gpu & b) == 0u;
-    const bool hit = isc ? end == s.T : (gpu_event && end == s.V);
+    const bool hit = end == (isc ? s.T : s.V);
     ended |= hit ? b : 0u;
     ntc = (isc && !hit) ? min(ntc, end) : ntc;
     nrem = (!isc && !hit) ? min(nrem, end - s.V) : nrem;
@@ -315,14 +319,22 @@ __device__ __forceinline__ void lt_lane(const LtShared& S, uint32_t* rows, uint3
       }
       // Modes and index part of the new job's level: a root's three table
       // parts, or one level combination (the first, all cpu, on a descent).
-      const uint32_t r0 = root % kLtPartCombos, rq = root / kLtPartCombos;
-      const uint32_t pa = L == 0u ? 0u : (L == 1u ? 3u : 4u);
-      const uint32_t ia = L == 0u ? r0 : (L == 1u ? c1 : c2);
-      const uint32_t ib = L == 0u ? rq % kLtPartCombos : 0u, ic = L == 0u ? rq / kLtPartCombos : 0u;
+      uint32_t cn, cq, xi;
+      if (L == 0u) {
+        const uint32_t r0 = root % kLtPartCombos, rq = root / kLtPartCombos;
+        const uint32_t r1 = rq % kLtPartCombos, r2 = rq / kLtPartCombos;
+        cn = S.cnow[0][r0] | S.cnow[1][r1] | S.cnow[2][r2];
+        cq = S.cque[0][r0] | S.cque[1][r1] | S.cque[2][r2];
+        xi = S.cidx[0][r0] + S.cidx[1][r1] + S.cidx[2][r2];
+      } else {
+        const uint32_t pa = L == 1u ? 3u : 4u, ia = L == 1u ? c1 : c2;
+        cn = S.cnow[pa][ia];
+        cq = S.cque[pa][ia];
+        xi = S.cidx[pa][ia];
+      }
       const uint32_t clear = L == 0u ? 0xFFFFFFFFu : (L == 1u ? (lm1 | lm2) : lm2);
-      now = (now & ~clear) | S.cnow[pa][ia] | S.cnow[1][ib] | S.cnow[2][ic];
-      que = (que & ~clear) | S.cque[pa][ia] | S.cque[1][ib] | S.cque[2][ic];
-      const uint32_t xi = S.cidx[pa][ia] + S.cidx[1][ib] + S.cidx[2][ic];
+      now = (now & ~clear) | cn;
+      que = (que & ~clear) | cq;
       idx0 = L == 0u ? xi : idx0;
       idx1 = L == 1u ? xi : (L == 0u ? 0u : idx1);
       idx2 = L == 2u ? xi : 0u;
