@@ -492,7 +492,8 @@ constexpr uint64_t kLtMinRootsPerBlock = 1024;
 // 4096 layered 10-tool DAGs (48 checked by enumeration): 2.9 events per
 // mapping against 2.8 for the best split and 4.1 for the prefix/mid/inner
 // split of the other batch kernel.
-inline void lanetree_split(const bfk::Tables& t, uint32_t* x_out, uint32_t* y_out, uint32_t* nblocks) {
+template <typename TB>
+inline void lanetree_split(const TB& t, uint32_t* x_out, uint32_t* y_out, uint32_t* nblocks) {
   const uint32_t n = t.n;
   uint32_t R[BF_MAX_TOOLS + 1] = {};
   retired_estimate(t, R);
@@ -521,31 +522,59 @@ inline void lanetree_split(const bfk::Tables& t, uint32_t* x_out, uint32_t* y_ou
   *nblocks = (uint32_t)(nb < 1 ? 1 : nb);
 }
 
-// Record of one scenario of the lane-tree batch search: its tables renumbered
-// with the sources first (when that is not already its order) and its levels.
+// The tables a lane-tree record's split estimate reads (n, pred, cpu, wnow).
+struct LtView {
+  uint32_t n;
+  uint32_t pred[BF_MAX_TOOLS], cpu[BF_MAX_TOOLS], wnow[BF_MAX_TOOLS];
+};
+
+// Record of one scenario of the lane-tree batch search: its tools renumbered
+// with the sources first (each group in the scenario's order: the order of
+// relabel_sources_first) and its levels.  Built straight from the desc; the
+// slowdown constants are those of build_tables, taken over from the previous
+// record built on this thread when the slowdown table is the same (the
+// scenarios of a batch usually share one).
 inline void lanetree_record(const bf_scenario_desc* d, bfk::LaneTreeRecord* r) {
-  bfk::Tables t0, rt;
-  build_tables(d, &t0);
-  const bfk::Tables& t = relabel_sources_first(t0, &rt) ? rt : t0;
+  const uint32_t n = d->n;
+  uint32_t order[BF_MAX_TOOLS], pos[BF_MAX_TOOLS], k = 0;
+  for (uint32_t v = 0; v < n; ++v)
+    if (d->pred_mask[v] == 0u) order[k++] = v;
+  for (uint32_t v = 0; v < n; ++v)
+    if (d->pred_mask[v] != 0u) order[k++] = v;
+  for (uint32_t j = 0; j < n; ++j) pos[order[j]] = j;
   std::memset(r, 0, sizeof *r);
-  r->n = t.n;
-  r->budget = t.budget;
-  r->all_mask = t.all_mask;
-  r->big_mask = t.big_mask;
-  for (uint32_t v = 0; v < t.n; ++v) {
-    r->pred[v] = t.pred[v];
-    r->dur[0][v] = t.cpu[v];
-    r->dur[1][v] = t.wnow[v];
-    r->dur[2][v] = t.wq[v];
-    r->vram[v] = t.vram[v];
-    r->pv[v] = (uint32_t)pow3(t.orig[v]);
+  r->n = n;
+  r->budget = d->vram_budget_mib;
+  r->all_mask = (1u << n) - 1u;
+  LtView view;
+  view.n = n;
+  for (uint32_t j = 0; j < n; ++j) {
+    const uint32_t v = order[j];
+    uint32_t pm = 0u;
+    for (uint32_t u = 0; u < v; ++u)
+      if ((d->pred_mask[v] >> u) & 1u) pm |= 1u << pos[u];
+    r->pred[j] = view.pred[j] = pm;
+    r->dur[0][j] = view.cpu[j] = d->cpu_us[v];
+    r->dur[1][j] = view.wnow[j] = (d->gpu_us[v] + d->xfer_us[v]) * 1024u;
+    r->dur[2][j] = (d->load_us[v] + d->gpu_us[v] + d->xfer_us[v]) * 1024u;
+    r->vram[j] = d->vram_mib[v];
+    r->pv[j] = (uint32_t)pow3(v);
+    if (d->vram_mib[v] > d->vram_budget_mib) r->big_mask |= 1u << j;
   }
-  for (uint32_t k = 0; k <= bfk::kLtMaxTools; ++k) {
-    r->f[k] = t.f[k];
-    r->fshift[k] = t.fshift[k];
-    r->fmagic[k] = t.fmagic[k];
+  thread_local uint32_t last_f[BF_MAX_TOOLS + 1] = {0};
+  thread_local uint32_t last_n = 0;
+  thread_local bfk::Tables last;
+  if (last_n != n || std::memcmp(last_f, d->slowdown_q10, sizeof last_f) != 0) {
+    build_tables(d, &last);
+    std::memcpy(last_f, d->slowdown_q10, sizeof last_f);
+    last_n = n;
   }
-  lanetree_split(t, &r->x, &r->y, &r->nblocks);
+  for (uint32_t j = 0; j <= bfk::kLtMaxTools; ++j) {
+    r->f[j] = last.f[j];
+    r->fshift[j] = last.fshift[j];
+    r->fmagic[j] = last.fmagic[j];
+  }
+  lanetree_split(view, &r->x, &r->y, &r->nblocks);
 }
 
 }  // namespace host
