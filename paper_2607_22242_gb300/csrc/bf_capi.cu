@@ -248,6 +248,30 @@ void build_lanetree_records(const bf_scenario_desc* descs, const uint32_t* ids, 
   });
 }
 
+// Where a batch's scenarios go: up to kLtBatchTools tools the lane-tree
+// kernel (bf_lanetree.cuh), above it the batch kernel (bf_kernels.cu).  The
+// keys of the first group come first in the key array.
+struct BatchSplit {
+  uint32_t ns = 0, nl = 0;            // scenarios in each group
+  uint32_t nmax_small = 0, nmax_large = 0;
+};
+
+template <typename Ids>
+BatchSplit split_batch(const bf_scenario_desc* descs, uint32_t count, Ids& small, Ids& large) {
+  BatchSplit b;
+  for (uint32_t i = 0; i < count; ++i) {
+    const uint32_t n = descs[i].n;
+    if (n <= bfk::kLtBatchTools) {
+      small[b.ns++] = i;
+      b.nmax_small = n > b.nmax_small ? n : b.nmax_small;
+    } else {
+      large[b.nl++] = i;
+      b.nmax_large = n > b.nmax_large ? n : b.nmax_large;
+    }
+  }
+  return b;
+}
+
 // Launch both groups of a batch on `st` (records already on the device; keys
 // reset to ~0): keys[0, ns) for the lane-tree group, keys[ns, ns + nl) for
 // the other.
