@@ -14,6 +14,7 @@ import pytest
 
 import oracle
 import pins
+from batch_cases import mixed_group_batch
 from paper_2607_22242_gb300 import bf
 from paper_2607_22242_gb300 import scenarios as S
 
@@ -564,3 +565,42 @@ def test_pruned_search_batch_scenarios(golden):
         with bf.create_scenario(scn) as h:
             r = bf.search_pruned(h)
         assert (r.index, r.makespan_us) == (want_i[k], want_m[k]), k
+
+
+# --------------------------------------------------------------------------- the batch's two kernel groups
+
+def test_batch_two_kernel_groups():
+    """Scenarios of up to 12 tools (lane-tree kernel) interleaved with scenarios of 13 and 14 tools
+    (batch kernel) in one call: every result at its position, equal to the oracle's."""
+    scns = mixed_group_batch()
+    assert {s.n > 12 for s in scns} == {True, False}
+    o_i, o_m = oracle.search_batch(scns, THREADS)
+    res = bf.search_batch(scns)
+    assert [(r.index, r.makespan_us) for r in res] == list(zip(o_i.tolist(), o_m.tolist()))
+
+
+def test_search_launch_state_across_calls():
+    """A search call is one launch whose last block writes the result to the handle's host mirror and
+    resets the launch state: every kind of search, and empty and partial ranges, on one handle and on
+    two streams in turn, must each give the oracle's answer."""
+    import torch
+    scn = S.config1()
+    total = 3 ** scn.n
+    want = oracle.search(scn, THREADS)
+    part = (total // 3, total // 5)
+    want_part = oracle.search_range(scn, part[0], part[1], THREADS)
+    streams = [torch.cuda.current_stream(), torch.cuda.Stream()]
+    with bf.create_scenario(scn) as h:
+        for k in range(3):
+            st = streams[k % 2]
+            r = bf.search_best(h, st)
+            assert (r.index, r.makespan_us) == want
+            empty = bf.search_range(h, 17, 0, st)
+            assert not empty.feasible and empty.index == 17
+            r = bf.search_range(h, part[0], part[1], st)
+            assert (r.index, r.makespan_us) == want_part
+            r = bf.search_pruned(h, None, st)
+            assert (r.index, r.makespan_us) == want
+            rt, _ = bf.search_tree(h, bf.SPACE_FULL, True, None, st)
+            assert (rt.index, rt.makespan_us) == want
+            streams[1 - k % 2].wait_stream(st)

@@ -103,3 +103,13 @@ def test_noalloc_rejects_oversized_batch():
         bf.search_batch_noalloc(batch)
     assert ei.value.code == bf.BF_EINVAL
     assert str(bf.NOALLOC_MAX_SCENARIOS) in ei.value.message
+
+
+def test_noalloc_two_kernel_groups():
+    """Scenarios of up to 12 tools and of 13 and 14 tools interleaved in one call: both regions of the
+    fixed scratch in use, every result at its position, equal to the oracle's."""
+    from batch_cases import mixed_group_batch
+    scns = mixed_group_batch()
+    o_i, o_m = oracle.search_batch(scns, oracle.default_threads())
+    got = bf.search_batch_noalloc(scns)
+    assert [(r.index, r.makespan_us) for r in got] == list(zip(o_i.tolist(), o_m.tolist()))
