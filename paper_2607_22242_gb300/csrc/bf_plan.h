@@ -477,9 +477,12 @@ inline bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n, uint32_t block_wa
 }
 
 // Mappings a block of the lane-tree batch kernel aims to search, and the
-// fewest roots a block hands out (about four per lane of 256).
-constexpr uint64_t kLtBlockMappings = 59049;
-constexpr uint64_t kLtMinRootsPerBlock = 1024;
+// fewest roots a block hands out (two per lane of 256).  Many short blocks
+// keep every SM busy to the end of the launch: 4096 x 3^10 batch call, blocks
+// per scenario (roots per block) 1 (1024+) 16.2 ms, 2 15.4, 4 (512+) 15.1,
+// 8 (512+) 14.8, 8 (256+) 14.8, 16 (256+) 15.8, 32 (128+) 18.0.
+constexpr uint64_t kLtBlockMappings = 7381;
+constexpr uint64_t kLtMinRootsPerBlock = 512;
 
 // The levels of the lane-tree search of one scenario (n <= kLtBatchTools):
 // roots [0, x), then [x, y), then [y, n).  Each level below the root holds at
