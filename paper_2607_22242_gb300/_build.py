@@ -49,8 +49,9 @@ def _fingerprint(extra) -> str:
     return h.hexdigest()
 
 
-# Sources of the enumerating kernels' translation unit (bf_kernels.cu and what it includes).
-KERNEL_UNIT = ("bf_kernels.cu", "bf_enum.cuh", "bf_sim.cuh", "bf_launch.h")
+# Sources of the enumerating kernels' translation unit (bf_kernels.cu and what it includes), and
+# the host planner that chooses their launches (splits, windows, grid sizes).
+KERNEL_UNIT = ("bf_kernels.cu", "bf_enum.cuh", "bf_sim.cuh", "bf_launch.h", "bf_plan.h")
 
 
 def _code_only(text: str) -> str:
@@ -61,9 +62,9 @@ def _code_only(text: str) -> str:
     return " ".join(text.split())
 
 
-# Sources of the lane-tree batch kernel's translation unit.
+# Sources of the lane-tree batch kernel's translation unit, and the planner of its launches.
 LANETREE_UNIT = ("bf_lanetree.cu", "bf_lanetree.cuh", "bf_lanetree_launch.h", "bf_enum.cuh", "bf_sim.cuh",
-                 "bf_launch.h")
+                 "bf_launch.h", "bf_plan.h")
 
 
 def kernel_fingerprint(csrc: str = CSRC, unit=KERNEL_UNIT) -> str:
