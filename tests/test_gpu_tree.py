@@ -241,3 +241,23 @@ def test_tree_search_time_limit():
     want = _golden("wide_results.json")["workloads"]["wide28"]["ternary"]
     res, _ = bf.search_tree(scn, bf.SPACE_FULL, True)
     assert _pair(res) == tuple(want)
+
+
+def test_tie_order_scenarios_every_search():
+    """Queue-heavy tiny DAGs with late sources, among them tied optima whose lowest member differs
+    between the sources-first order the searches may run in and the canonical order (the first is
+    scenario 91): the tree search in both spaces, pruned and unpruned, the exhaustive search, the
+    branch and bound and the batched search (lane-tree kernel) must all return the lowest
+    canonical index among the oracle's optima."""
+    from tie_cases import tie_order_scenarios
+    scns = tie_order_scenarios()
+    want = [oracle.search(s) for s in scns]
+    for t, (scn, w) in enumerate(zip(scns, want)):
+        binary = oracle.search_binary(scn)
+        with bf.create_scenario(scn) as h:
+            for prune in (True, False):
+                assert _pair(bf.search_tree(h, bf.SPACE_FULL, prune)[0]) == w, (t, prune)
+                assert _pair(bf.search_tree(h, bf.SPACE_BINARY, prune)[0]) == binary, (t, prune)
+            assert _pair(bf.search_best(h)) == w, t
+            assert _pair(bf.search_pruned(h)) == w, t
+    assert [_pair(r) for r in bf.search_batch(scns)] == want
