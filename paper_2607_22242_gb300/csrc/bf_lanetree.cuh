@@ -39,7 +39,8 @@
 //   * a lane moves to its next job (a level combination or a new root) the
 //     moment its current one ends, instead of waiting for the warp's slowest
 //     lane; roots come from a per-block counter in shared memory;
-//   * a checkpoint holds the state words plus the rows of running tools only.
+//   * a checkpoint is nine state words: the per-tool words of the tools
+//     running at it are never written again while it can still be resumed.
 // Arithmetic is that of bf_sim.cuh: u32 real time, virtual clock modulo 2^32,
 // GPU completion ceil(rem * f[k] / 2^20), the CPU-event advance
 // floor(dt * 2^20 / f[k]) by the per-k reciprocal of Granlund and Montgomery
@@ -102,10 +103,14 @@ struct LtState {
   uint32_t gm;     // end stamp of the running GPU tool that ends first (when one runs)
 };
 
-// Rows of one lane ([row][thread], `stride` threads): the current per-tool
-// words [0, n); checkpoint 1: words [n, 2n), state [2n, 2n + 9); checkpoint
-// 2: words [2n + 9, 3n + 9), state [3n + 9, 3n + 18).
-__host__ __device__ inline uint32_t lt_rows(uint32_t n) { return 3u * n + 2u * kLtStateWords; }
+// Rows of one lane ([row][thread], `stride` threads): the per-tool words
+// [0, n), then the state words of checkpoint 1 [n, n + 9) and of checkpoint
+// 2 [n + 9, n + 18).  One set of per-tool words serves every level: a tool's
+// word is written once per simulation, when it starts, and only read after
+// that; a job resumed from a checkpoint starts only tools that were pending
+// there, so it never overwrites the word of a tool running at any checkpoint
+// it or a later job may resume from.  A checkpoint is its state words alone.
+__host__ __device__ inline uint32_t lt_rows(uint32_t n) { return n + 2u * kLtStateWords; }
 
 __device__ __forceinline__ uint32_t lt_ready(const LtShared& S, uint32_t pend, uint32_t done) {
   return pend & S.rt[0][done & (kLtChunk - 1u)] & S.rt[1][(done >> kLtChunkBits) & (kLtChunk - 1u)];
@@ -256,7 +261,7 @@ template <typename TakeRoot, typename Sink>
 __device__ __forceinline__ void lt_lane(const LtShared& S, uint32_t* rows, uint32_t stride, TakeRoot take_root,
                                         Sink& sink) {
   const LaneTreeRecord& R = S.rec;
-  const uint32_t n = R.n, blk = n + kLtStateWords;
+  const uint32_t n = R.n;
   uint32_t* const cur = rows;
   const uint32_t stop0 = R.all_mask & ~((1u << R.x) - 1u);
   const uint32_t stop1 = R.all_mask & ~((1u << R.y) - 1u);
@@ -285,9 +290,8 @@ __device__ __forceinline__ void lt_lane(const LtShared& S, uint32_t* rows, uint3
         root = take_root();
         if (root == 0xFFFFFFFFu) return;
       }
-      uint32_t* const ck = rows + (L == 2u ? 2u * n + kLtStateWords : n) * stride;  // words, then state
-      uint32_t* const cw = ck + n * stride;
-      if (descend) {  // save: the state words and the rows of the running tools
+      uint32_t* const cw = rows + (L == 2u ? n + kLtStateWords : n) * stride;  // checkpoint L's state words
+      if (descend) {  // save the state words
         cw[0] = s.pend;
         cw[stride] = s.run;
         cw[2u * stride] = s.qset;
@@ -297,11 +301,7 @@ __device__ __forceinline__ void lt_lane(const LtShared& S, uint32_t* rows, uint3
         cw[6u * stride] = s.V;
         cw[7u * stride] = s.tc;
         cw[8u * stride] = s.gm;
-        for (uint32_t m = s.run; m; m &= m - 1u) {
-          const uint32_t i = __ffs(m) - 1u;
-          ck[i * stride] = cur[i * stride];
-        }
-      } else {  // load a checkpoint, or the time-0 state for a root (no running tool)
+      } else {  // load a checkpoint's state words, or the time-0 state for a root
         const uint32_t* w = L == 0u ? S.ck0 : cw;
         const uint32_t ws = L == 0u ? 1u : stride;
         s.pend = w[0];
@@ -312,10 +312,6 @@ __device__ __forceinline__ void lt_lane(const LtShared& S, uint32_t* rows, uint3
         s.V = w[6u * ws];
         s.tc = w[7u * ws];
         s.gm = w[8u * ws];
-        for (uint32_t m = s.run; m; m &= m - 1u) {
-          const uint32_t i = __ffs(m) - 1u;
-          cur[i * stride] = ck[i * stride];
-        }
       }
       // Modes and index part of the new job's level: a root's three table
       // parts, or one level combination (the first, all cpu, on a descent).
