@@ -320,7 +320,13 @@ def _batch_call(fn, scns: Sequence[Scenario], stream, packed=None) -> List[Resul
     descs = packed.ctypes.data_as(ctypes.POINTER(Desc)) if count else None
     results = (CResult * max(count, 1))()
     _check(fn(descs, count, results, ctypes.c_void_p(_stream_handle(stream))))
-    return [_result(results[i], scns[i].n) for i in range(count)]
+    if not count:
+        return []
+    import numpy as np
+    arr = np.ctypeslib.as_array(results)  # one structured view instead of per-field ctypes reads
+    modes = arr["mode"][:, :max(sc.n for sc in scns)].tolist()
+    return [Result(i, m, bool(f), md[:sc.n]) for i, m, f, md, sc in
+            zip(arr["index"].tolist(), arr["makespan_us"].tolist(), arr["feasible"].tolist(), modes, scns)]
 
 
 def search_batch(scns: Sequence[Scenario], stream=None, packed=None) -> List[Result]:
