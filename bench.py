@@ -48,10 +48,11 @@ INT_LANES_PER_SM = 128  # 4 SMSPs x 32 lanes: one thread instruction each per cl
 
 # Committed ncu summaries of the enumerating kernels, one per standard workload.
 PROFILES = {"config0": "search_kernel_config0_n8.md", "config1": "search_kernel_config1_n12.md",
-            "config2": "search_kernel_config2_n16.md", "config3": "search_kernel_config3_n19.md",
+            "config2": "lanetree_single_kernel_config2_n16.md", "config3": "search_kernel_config3_n19.md",
             "config4_batch": "lanetree_kernel_config4.md"}
-# Translation unit each summary's fingerprint covers (_build.kernel_fingerprint).
-PROFILE_UNITS = {"config4_batch": "LANETREE_UNIT"}
+# Translation unit each summary's fingerprint covers (_build.kernel_fingerprint): the full search of
+# the 16-tool workload and the batch run the lane-tree kernels.
+PROFILE_UNITS = {"config2": "LANETREE_UNIT", "config4_batch": "LANETREE_UNIT"}
 PROFILE_KEYS = ("source_fingerprint", "dram_bytes_per_launch", "thread_instructions_per_mapping", "issue_active",
                 "warp_efficiency", "kernel_ms")
 

@@ -15,9 +15,9 @@
 
 // Per-handle scratch, one block on the device and a pinned mirror on the host:
 // the packed search key, the tree search's best record, bound and counters,
-// and the what-if probe list with its results.
+// the what-if probe list with its results, and the lane-tree record.
 struct bf_scratch {
-  bfk::SearchSync search;  // the search kernel's launch state; search.key of the host mirror receives its result
+  bfk::SearchSync search;  // whole-space searches' launch state; search.key of the host mirror receives their result
   unsigned long long key;
   uint32_t survivors;   // pruned search: number of surviving prefixes
   uint32_t pruned_bound;  // pruned search: the incumbent's makespan (set with survivors)
@@ -29,6 +29,7 @@ struct bf_scratch {
   uint64_t idx[BF_MAX_PROBES];
   uint32_t ms[BF_MAX_PROBES];
   uint8_t fe[BF_MAX_PROBES];
+  bfk::LaneTreeRecord lt;  // whole-space search by the lane-tree kernel (bf_scenario::lanetree)
 };
 
 struct bf_scenario {
@@ -45,6 +46,11 @@ struct bf_scenario {
   bfk::Plan rplan;
   bfk::Tables pwindow;  // bf_search_pruned: its window (of pplan, on rtables)
   bfk::Plan pplan;      // bf_search_pruned: its split (shorter prefixes: fewer to filter)
+  // Searches of the whole space by the lane-tree kernel (scenarios of
+  // kLtSingleMinTools to kLtMaxTools tools): its record's level boundary x
+  // and the blocks of a launch; lanetree false otherwise.
+  bool lanetree;
+  uint32_t lt_x, lt_blocks;
   int device;
   bf_scratch* d_scratch;      // device scratch
   bf_scratch* h_scratch;      // pinned host mirror

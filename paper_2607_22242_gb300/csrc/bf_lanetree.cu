@@ -1,6 +1,7 @@
-// bf_lanetree.cu -- the lane-tree batch kernel (bf_lanetree.cuh): the full
-// search of many small scenarios in one launch, one or more blocks per
-// scenario, every lane walking its roots' trees of checkpoints.
+// bf_lanetree.cu -- the lane-tree kernels (bf_lanetree.cuh): the full search
+// of many small scenarios in one launch, one or more blocks per scenario, and
+// the full search of one scenario by every lane of the GPU; every lane walks
+// its roots' trees of checkpoints.
 #include "bf_enum.cuh"
 #include "bf_lanetree_launch.h"
 #include "bf_launch.h"
@@ -8,12 +9,23 @@
 namespace bfk {
 namespace {
 
-constexpr int kLtThreads = 256;
+constexpr int kLtThreads = (int)kLtLaunchThreads;
+constexpr uint32_t kLtSingleChunks = 3;  // tables of the one-scenario search: up to 18 tools
 
 __device__ __forceinline__ unsigned long long lt_warp_min(unsigned long long v) {
 #pragma unroll
   for (int o = 16; o > 0; o >>= 1) v = min(v, __shfl_xor_sync(0xFFFFFFFFu, v, o));
   return v;
+}
+
+// The block's copy of a record and the tables derived from it.
+template <uint32_t NC>
+__device__ __forceinline__ void lt_load_record(LtSharedT<NC>& S, const LaneTreeRecord* rec) {
+  const uint32_t* src = reinterpret_cast<const uint32_t*>(rec);
+  uint32_t* dst = reinterpret_cast<uint32_t*>(&S.rec);
+  for (uint32_t w = threadIdx.x; w < sizeof(LaneTreeRecord) / 4; w += blockDim.x) dst[w] = src[w];
+  __syncthreads();
+  lt_fill_tables(S);
 }
 
 // Block b searches roots [3^x * j / nblocks, 3^x * (j + 1) / nblocks) of
@@ -32,13 +44,7 @@ __global__ void __launch_bounds__(kLtThreads) lanetree_kernel(const LaneTreeReco
     else hi = mid;
   }
   const uint32_t sc = lo;
-  {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(recs + sc);
-    uint32_t* dst = reinterpret_cast<uint32_t*>(&S.rec);
-    for (uint32_t w = threadIdx.x; w < sizeof(LaneTreeRecord) / 4; w += blockDim.x) dst[w] = src[w];
-  }
-  __syncthreads();
-  lt_fill_tables(S);
+  lt_load_record(S, recs + sc);
   if (threadIdx.x == 0) {
     uint32_t roots = 1u;
     for (uint32_t t = 0; t < S.rec.x; ++t) roots *= 3u;
@@ -59,16 +65,92 @@ __global__ void __launch_bounds__(kLtThreads) lanetree_kernel(const LaneTreeReco
   if ((threadIdx.x & 31u) == 0u && best != ~0ull) atomicMin(keys + sc, best);
 }
 
+// The whole search of one scenario, one block per resident slot of the GPU.
+// Roots [0, static_roots) are split evenly over the blocks and handed out by
+// a counter in each block's shared memory; a lane whose block has none left
+// takes the next root of [static_roots, 3^x) from sync->next_root (one
+// atomic per group of lanes of a warp asking at once), so lanes keep busy
+// until the last roots.  The lowest key goes to sync->key; the last block to
+// finish copies it to *host_key (pinned host memory the device addresses)
+// and puts sync back to (~0, 0, 0).
+__global__ void __launch_bounds__(kLtThreads) lanetree_single_kernel(const LaneTreeRecord* __restrict__ rec,
+                                                                    uint32_t static_roots, SearchSync* sync,
+                                                                    unsigned long long* host_key) {
+  extern __shared__ uint32_t lt_rows_smem[];
+  __shared__ LtSharedT<kLtSingleChunks> S;
+  lt_load_record(S, rec);
+  if (threadIdx.x == 0) {
+    const uint64_t j = blockIdx.x, nb = gridDim.x;
+    S.root_next = (uint32_t)(static_roots * j / nb);
+    S.root_end = (uint32_t)(static_roots * (j + 1u) / nb);
+  }
+  __syncthreads();
+  uint32_t roots = 1u;
+  for (uint32_t t = 0; t < S.rec.x; ++t) roots *= 3u;
+  MinKeySink sink;
+  LtSharedT<kLtSingleChunks>& Sref = S;
+  lt_lane(S, lt_rows_smem + threadIdx.x, blockDim.x,
+          [&Sref, sync, static_roots, roots]() {
+            const uint32_t r = atomicAdd(&Sref.root_next, 1u);
+            if (r < Sref.root_end) return r;
+            const uint32_t group = __activemask(), lane = threadIdx.x & 31u;
+            const uint32_t leader = __ffs(group) - 1u;
+            uint32_t base = 0u;
+            if (lane == leader) base = atomicAdd(&sync->next_root, (uint32_t)__popc(group));
+            base = __shfl_sync(group, base, leader);
+            const uint32_t t = static_roots + base + __popc(group & ((1u << lane) - 1u));
+            return t < roots ? t : 0xFFFFFFFFu;
+          },
+          sink);
+  const unsigned long long best = lt_warp_min(sink.best);
+  if ((threadIdx.x & 31u) == 0u && best != ~0ull) atomicMin(&sync->key, best);
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    __threadfence();
+    if (atomicAdd(&sync->blocks_done, 1u) == gridDim.x - 1u) {
+      *host_key = atomicExch(&sync->key, ~0ull);
+      sync->blocks_done = 0u;
+      sync->next_root = 0u;
+      __threadfence_system();
+    }
+  }
+}
+
+size_t lt_smem_bytes(uint32_t n) { return sizeof(uint32_t) * lt_rows(n) * kLtThreads; }
+
 }  // namespace
 
 cudaError_t launch_lanetree(const LaneTreeRecord* d_recs, const uint32_t* d_first_block, uint32_t count,
                             uint32_t blocks, uint32_t nmax, unsigned long long* keys, cudaStream_t st) {
   static std::atomic<uint64_t> ready{0};
-  const size_t smem = sizeof(uint32_t) * lt_rows(kLtBatchTools) * kLtThreads;
-  cudaError_t e = allow_dyn_smem(lanetree_kernel, smem, &ready);
+  cudaError_t e = allow_dyn_smem(lanetree_kernel, lt_smem_bytes(kLtBatchTools), &ready);
   if (e != cudaSuccess) return e;
-  lanetree_kernel<<<blocks, kLtThreads, sizeof(uint32_t) * lt_rows(nmax) * kLtThreads, st>>>(d_recs, d_first_block,
-                                                                                           count, keys);
+  lanetree_kernel<<<blocks, kLtThreads, lt_smem_bytes(nmax), st>>>(d_recs, d_first_block, count, keys);
+  return cudaGetLastError();
+}
+
+cudaError_t lanetree_single_blocks(uint32_t n, uint32_t* blocks) {
+  static std::atomic<uint64_t> ready{0};
+  cudaError_t e = allow_dyn_smem(lanetree_single_kernel, lt_smem_bytes(kLtMaxTools), &ready);
+  int dev = 0, sms = 0, per_sm = 0;
+  if (e == cudaSuccess) e = cudaGetDevice(&dev);
+  if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (e == cudaSuccess)
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lanetree_single_kernel, kLtThreads, lt_smem_bytes(n));
+  if (e != cudaSuccess) return e;
+  *blocks = (uint32_t)(sms > 0 ? sms : 1) * (uint32_t)(per_sm > 0 ? per_sm : 1);
+  return cudaSuccess;
+}
+
+cudaError_t launch_lanetree_single(const LaneTreeRecord* d_rec, uint32_t n, uint32_t x, uint32_t blocks,
+                                   SearchSync* sync, unsigned long long* host_key, cudaStream_t st) {
+  static std::atomic<uint64_t> ready{0};
+  cudaError_t e = allow_dyn_smem(lanetree_single_kernel, lt_smem_bytes(kLtMaxTools), &ready);
+  if (e != cudaSuccess) return e;
+  uint64_t roots = 1;
+  for (uint32_t t = 0; t < x; ++t) roots *= 3u;
+  const uint32_t static_roots = (uint32_t)(roots * kLtStaticShareNum / kLtStaticShareDen);
+  lanetree_single_kernel<<<blocks, kLtThreads, lt_smem_bytes(n), st>>>(d_rec, static_roots, sync, host_key);
   return cudaGetLastError();
 }
 

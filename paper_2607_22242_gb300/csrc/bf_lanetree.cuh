@@ -1,5 +1,6 @@
-// bf_lanetree.cuh -- the batched search of small scenarios (n <= 12 tools) as
-// a tree of checkpoints walked by each lane.
+// bf_lanetree.cuh -- the full search of a scenario of up to 16 tools as a
+// tree of checkpoints walked by each lane: many small scenarios in one launch
+// (the batch), or one scenario over the whole GPU.
 //
 // What it computes is the brute-force oracle of §2.3 / §4.1 under the integer
 // latency model declared in include/bf.h: for one scenario, the feasible
@@ -29,7 +30,8 @@
 //     event touches only the tools it admits, retires or scans for the next
 //     completion (bit loops over small sets) instead of every slot;
 //   * the VRAM in use is a table lookup on the set of running GPU tools, the
-//     ready set a lookup on the done set (two 6-bit chunks each);
+//     ready set a lookup on the done set (one lookup per 6-bit chunk of the
+//     tools: two up to 12 tools, three up to 16);
 //   * the queue is a FIFO list of 4-bit tool numbers in one 64-bit word:
 //     tools join it in the order they become ready (in index order within
 //     an instant), which is the model's (ready time, index) order, so its
@@ -54,20 +56,24 @@
 namespace bfk {
 
 constexpr uint32_t kLtBatchTools = 12;  // the batch sends scenarios of up to this many tools here
-constexpr uint32_t kLtMaxTools = 16;    // record capacity
-constexpr uint32_t kLtChunkBits = 6;    // readiness and VRAM tables: two 6-bit chunks (n <= 12)
+constexpr uint32_t kLtMaxTools = 16;    // record capacity (and the queue's 4-bit tool numbers)
+constexpr uint32_t kLtChunkBits = 6;    // readiness and VRAM tables: 6-bit chunks of the tools
 constexpr uint32_t kLtChunk = 1u << kLtChunkBits;
 constexpr uint32_t kLtPartTools = 4;    // tools per table-driven part of the mode combinations
 constexpr uint32_t kLtPartCombos = 81;  // 3^kLtPartTools
-constexpr uint32_t kLtParts = 5;        // root [0,4), root [4,8), root [8,x), level [x,y), level [y,n)
+constexpr uint32_t kLtRootParts = 4;    // root tools [0,4), [4,8), [8,12), [12,x)
+constexpr uint32_t kLtParts = kLtRootParts + 2;  // the root's parts, level [x,y), level [y,n)
 constexpr uint32_t kLtStateWords = 9;   // pend, run, qset, qlist (2 words), T, V, tc, gm
+
+// 6-bit chunks the tables of an n-tool scenario need.
+__host__ __device__ constexpr uint32_t lt_chunks(uint32_t n) { return (n + kLtChunkBits - 1u) / kLtChunkBits; }
 
 // One scenario of the batch, host-built (bf_plan.h lanetree_record); tools in
 // the renumbered order.
 struct LaneTreeRecord {
   uint32_t n, budget, all_mask, big_mask;  // big_mask: tools with m > M
   uint32_t x, y;                           // level boundaries, 1 <= x <= y <= n
-  uint32_t nblocks;                        // blocks the roots [0, 3^x) are split over
+  uint32_t nblocks;                        // batch: blocks the roots [0, 3^x) are split over
   uint32_t pad;
   uint32_t pred[kLtMaxTools];
   uint32_t dur[3][kLtMaxTools];  // per mode: c (us); (g + x) * 1024; (l + g + x) * 1024
@@ -78,11 +84,13 @@ struct LaneTreeRecord {
   uint64_t fmagic[kLtMaxTools + 1];
 };
 
-// Per block: the record and the tables derived from it.
-struct LtShared {
+// Per block: the record and the tables derived from it; NC 6-bit chunks
+// cover the record's tools (NC = lt_chunks(n) or more).
+template <uint32_t NC>
+struct LtSharedT {
   LaneTreeRecord rec;
-  uint32_t rt[2][kLtChunk];  // rt[c][v]: tools whose predecessors in chunk c are all in v
-  uint32_t lv[2][kLtChunk];  // lv[c][v]: VRAM of the tools of chunk c in v
+  uint32_t rt[NC][kLtChunk];  // rt[c][v]: tools whose predecessors in chunk c are all in v
+  uint32_t lv[NC][kLtChunk];  // lv[c][v]: VRAM of the tools of chunk c in v
   // Mode combinations of the parts (see kLtParts): now / queue masks and the
   // canonical index part of combination j of each part.
   uint32_t cnow[kLtParts][kLtPartCombos];
@@ -91,13 +99,14 @@ struct LtShared {
   uint32_t ck0[kLtStateWords];   // the state words at time 0 (a root's checkpoint)
   uint32_t root_next, root_end;  // this block's roots still to take: [root_next, root_end)
 };
+using LtShared = LtSharedT<2>;  // the batch: up to kLtBatchTools tools
 
 // Lane state held in registers; the per-tool words are shared-memory rows.
 // Every tool is pending, waiting in the queue (qset), running or done, so
 // done = ~(pend | run | qset) (the slots beyond n count as done).
 struct LtState {
   uint32_t pend, run, qset;
-  uint64_t qlist;  // waiting queued tools, head in bits 0-3, each as its index + 1
+  uint64_t qlist;  // waiting queued tools by index, head in bits 0-3; qset says how many
   uint32_t T, V;   // real time (us); virtual GPU clock (1/1024 us of isolated work, modulo 2^32)
   uint32_t tc;     // earliest end of a running CPU tool (0xFFFFFFFF if none)
   uint32_t gm;     // end stamp of the running GPU tool that ends first (when one runs)
@@ -112,18 +121,27 @@ struct LtState {
 // it or a later job may resume from.  A checkpoint is its state words alone.
 __host__ __device__ inline uint32_t lt_rows(uint32_t n) { return n + 2u * kLtStateWords; }
 
-__device__ __forceinline__ uint32_t lt_ready(const LtShared& S, uint32_t pend, uint32_t done) {
-  return pend & S.rt[0][done & (kLtChunk - 1u)] & S.rt[1][(done >> kLtChunkBits) & (kLtChunk - 1u)];
+template <uint32_t NC>
+__device__ __forceinline__ uint32_t lt_ready(const LtSharedT<NC>& S, uint32_t pend, uint32_t done) {
+  uint32_t r = pend;
+#pragma unroll
+  for (uint32_t c = 0; c < NC; ++c) r &= S.rt[c][(done >> (kLtChunkBits * c)) & (kLtChunk - 1u)];
+  return r;
 }
 
-__device__ __forceinline__ uint32_t lt_vram(const LtShared& S, uint32_t gpu_running) {
-  return S.lv[0][gpu_running & (kLtChunk - 1u)] + S.lv[1][(gpu_running >> kLtChunkBits) & (kLtChunk - 1u)];
+template <uint32_t NC>
+__device__ __forceinline__ uint32_t lt_vram(const LtSharedT<NC>& S, uint32_t gpu_running) {
+  uint32_t m = 0u;
+#pragma unroll
+  for (uint32_t c = 0; c < NC; ++c) m += S.lv[c][(gpu_running >> (kLtChunkBits * c)) & (kLtChunk - 1u)];
+  return m;
 }
 
 // Fill the block's tables from S.rec (block-cooperative; S.rec is in place).
-__device__ __forceinline__ void lt_fill_tables(LtShared& S) {
+template <uint32_t NC>
+__device__ __forceinline__ void lt_fill_tables(LtSharedT<NC>& S) {
   const LaneTreeRecord& R = S.rec;
-  for (uint32_t e = threadIdx.x; e < 2u * kLtChunk; e += blockDim.x) {
+  for (uint32_t e = threadIdx.x; e < NC * kLtChunk; e += blockDim.x) {
     const uint32_t c = e / kLtChunk, v = e % kLtChunk, lo = kLtChunkBits * c;
     uint32_t ready = 0u, mem = 0u;
     for (uint32_t t = 0; t < R.n; ++t) {
@@ -133,10 +151,11 @@ __device__ __forceinline__ void lt_fill_tables(LtShared& S) {
     S.rt[c][v] = ready;
     S.lv[c][v] = mem;
   }
-  // Parts: root tools [0, min(x,4)), [4, min(x,8)), [8, x); level tools [x, y), [y, n).
+  // Parts: root tools [0, min(x,4)), [4, min(x,8)), [8, min(x,12)), [12, x);
+  // level tools [x, y), [y, n).
   for (uint32_t p = 0; p < kLtParts; ++p) {
-    const uint32_t lo = p < 3u ? min(4u * p, R.x) : (p == 3u ? R.x : R.y);
-    const uint32_t hi = p < 3u ? min(4u * p + 4u, R.x) : (p == 3u ? R.y : R.n);
+    const uint32_t lo = p < kLtRootParts ? min(kLtPartTools * p, R.x) : (p == kLtRootParts ? R.x : R.y);
+    const uint32_t hi = p < kLtRootParts ? min(kLtPartTools * p + kLtPartTools, R.x) : (p == kLtRootParts ? R.y : R.n);
     uint32_t combos = 1u;
     for (uint32_t t = lo; t < hi; ++t) combos *= 3u;
     for (uint32_t j = threadIdx.x; j < combos; j += blockDim.x) {
@@ -172,8 +191,9 @@ enum LtStep : uint32_t { kLtContinue = 0, kLtFinished = 1, kLtInfeasible = 2, kL
 // Returns kLtFinished once every tool has ended (the makespan is s.T).  The
 // loops' bodies are written as selects: lanes of a warp are at different
 // points of their simulations, and a branch in a body would run both sides.
-__device__ __forceinline__ uint32_t lt_step(const LtShared& S, LtState& s, uint32_t now, uint32_t que, uint32_t stop,
-                                            uint32_t* e, uint32_t stride) {
+template <uint32_t NC>
+__device__ __forceinline__ uint32_t lt_step(const LtSharedT<NC>& S, LtState& s, uint32_t now, uint32_t que,
+                                            uint32_t stop, uint32_t* e, uint32_t stride) {
   const LaneTreeRecord& R = S.rec;
   const uint32_t gpu = now | que;
   const uint32_t ready = lt_ready(S, s.pend, ~(s.pend | s.run | s.qset));
@@ -196,14 +216,14 @@ __device__ __forceinline__ uint32_t lt_step(const LtShared& S, LtState& s, uint3
     // queued: join the FIFO in index order (a row is written when the tool starts)
     for (uint32_t m = ready & que; m; m &= m - 1u) {
       const uint32_t i = __ffs(m) - 1u;
-      s.qlist |= (uint64_t)(i + 1u) << (4u * __popc(s.qset));
+      s.qlist |= (uint64_t)i << (4u * __popc(s.qset));
       s.qset |= 1u << i;
     }
     if ((ready & now) && lt_vram(S, s.run & gpu) > R.budget) return kLtInfeasible;  // out of memory
   }
   // ---- queue head: the first tool of the FIFO --------------------------------
-  if (s.qlist && !(s.run & que)) {
-    const uint32_t h = (uint32_t)(s.qlist & 15u) - 1u, hb = 1u << h;
+  if (s.qset && !(s.run & que)) {
+    const uint32_t h = (uint32_t)(s.qlist & 15u), hb = 1u << h;
     if (hb & R.big_mask) return kLtInfeasible;  // a head larger than M can never start
     const uint32_t rg = s.run & gpu;
     if (lt_vram(S, rg | hb) <= R.budget) {  // no bypass: otherwise the head waits
@@ -257,8 +277,8 @@ __device__ __forceinline__ uint32_t lt_step(const LtShared& S, LtState& s, uint3
 // which loads the block's time-0 state like a checkpoint -- and a stopped
 // job saves its state as the next level's checkpoint and continues with that
 // level's first combination (every tool of it on the CPU).
-template <typename TakeRoot, typename Sink>
-__device__ __forceinline__ void lt_lane(const LtShared& S, uint32_t* rows, uint32_t stride, TakeRoot take_root,
+template <uint32_t NC, typename TakeRoot, typename Sink>
+__device__ __forceinline__ void lt_lane(const LtSharedT<NC>& S, uint32_t* rows, uint32_t stride, TakeRoot take_root,
                                         Sink& sink) {
   const LaneTreeRecord& R = S.rec;
   const uint32_t n = R.n;
@@ -313,17 +333,23 @@ __device__ __forceinline__ void lt_lane(const LtShared& S, uint32_t* rows, uint3
         s.tc = w[7u * ws];
         s.gm = w[8u * ws];
       }
-      // Modes and index part of the new job's level: a root's three table
-      // parts, or one level combination (the first, all cpu, on a descent).
+      // Modes and index part of the new job's level: a root's four table
+      // parts (base-81 digits of the root), or one level combination (the
+      // first, all cpu, on a descent).
       uint32_t cn, cq, xi;
       if (L == 0u) {
-        const uint32_t r0 = root % kLtPartCombos, rq = root / kLtPartCombos;
-        const uint32_t r1 = rq % kLtPartCombos, r2 = rq / kLtPartCombos;
-        cn = S.cnow[0][r0] | S.cnow[1][r1] | S.cnow[2][r2];
-        cq = S.cque[0][r0] | S.cque[1][r1] | S.cque[2][r2];
-        xi = S.cidx[0][r0] + S.cidx[1][r1] + S.cidx[2][r2];
+        uint32_t q = root;
+        cn = cq = xi = 0u;
+#pragma unroll
+        for (uint32_t p = 0; p < kLtRootParts; ++p) {
+          const uint32_t d = p + 1u < kLtRootParts ? q % kLtPartCombos : q;
+          q /= kLtPartCombos;
+          cn |= S.cnow[p][d];
+          cq |= S.cque[p][d];
+          xi += S.cidx[p][d];
+        }
       } else {
-        const uint32_t pa = L == 1u ? 3u : 4u, ia = L == 1u ? c1 : c2;
+        const uint32_t pa = L == 1u ? kLtRootParts : kLtRootParts + 1u, ia = L == 1u ? c1 : c2;
         cn = S.cnow[pa][ia];
         cq = S.cque[pa][ia];
         xi = S.cidx[pa][ia];

@@ -28,14 +28,15 @@ inline cudaError_t allow_dyn_smem(K kernel, size_t bytes, std::atomic<uint64_t>*
   return e;
 }
 
-// State of one launch of the search kernel, in device memory: the best key
-// found so far and the blocks that have finished.  It holds (~0, 0) between
-// launches: the last block of a launch writes the result out and puts it
-// back.
+// State of one launch of a whole-space search (the search kernel or the
+// lane-tree search of one scenario), in device memory: the best key found so
+// far, the blocks that have finished and the next root of the lane tree's
+// shared tail.  It holds (~0, 0, 0) between launches: the last block of a
+// launch writes the result out and puts it back.
 struct SearchSync {
   unsigned long long key;
   uint32_t blocks_done;
-  uint32_t pad;
+  uint32_t next_root;
 };
 
 // One scenario of a batched search: its tables, its window tables and plan,

@@ -484,29 +484,28 @@ inline bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n, uint32_t block_wa
 constexpr uint64_t kLtBlockMappings = 7381;
 constexpr uint64_t kLtMinRootsPerBlock = 512;
 
-// The levels of the lane-tree search of one scenario (n <= kLtBatchTools):
+// The levels of the lane-tree search of one scenario (n <= kLtMaxTools):
 // roots [0, x), then [x, y), then [y, n).  Each level below the root holds at
-// most kLtPartTools tools (its combinations come from one table), and x is
-// large enough that every block gets kLtMinRootsPerBlock roots or more.
-// Among those, the split with the fewest estimated events: with R[b] the
-// tools retired when the first tool >= b can become ready (retired_estimate),
-// a root simulates about R[x] events, a level-1 job R[y] - R[x] and a
-// level-2 job n - R[y]; each job also costs about half an event to set up.
-// 4096 layered 10-tool DAGs (48 checked by enumeration): 2.9 events per
-// mapping against 2.8 for the best split and 4.1 for the prefix/mid/inner
-// split of the other batch kernel.
+// most kLtPartTools tools (its combinations come from one table), and the
+// root at most kLtRootParts * kLtPartTools, with 3^x >= min_roots.  Among
+// those, the split with the fewest estimated events: with R[b] the tools
+// retired when the first tool >= b can become ready (retired_estimate), a
+// root simulates about R[x] events, a level-1 job R[y] - R[x] and a level-2
+// job n - R[y]; each job also costs about half an event to set up.  4096
+// layered 10-tool DAGs (48 checked by enumeration): 2.9 events per mapping
+// against 2.8 for the best split and 4.1 for the prefix/mid/inner split of
+// the other batch kernel.
 template <typename TB>
-inline void lanetree_split(const TB& t, uint32_t* x_out, uint32_t* y_out, uint32_t* nblocks) {
+inline double lanetree_levels(const TB& t, uint64_t min_roots, uint32_t* x_out, uint32_t* y_out) {
   const uint32_t n = t.n;
   uint32_t R[BF_MAX_TOOLS + 1] = {};
   retired_estimate(t, R);
-  const uint64_t want_blocks = (pow3(n) + kLtBlockMappings - 1) / kLtBlockMappings;
   uint32_t xmin = 0;
-  while (xmin < n && pow3(xmin) < kLtMinRootsPerBlock * want_blocks) ++xmin;
-  if (n > 3u * kLtPartTools && xmin < n - 2u * kLtPartTools) xmin = n - 2u * kLtPartTools;
+  while (xmin < n && pow3(xmin) < min_roots) ++xmin;
+  if (n > 2u * kLtPartTools && xmin < n - 2u * kLtPartTools) xmin = n - 2u * kLtPartTools;
   double best = -1.0;
   uint32_t bx = n, by = n;
-  for (uint32_t x = xmin; x <= n && x <= 3u * kLtPartTools; ++x) {
+  for (uint32_t x = xmin; x <= n && x <= kLtRootParts * kLtPartTools; ++x) {
     for (uint32_t y = (x == n ? n : x + 1u); y <= n; ++y) {
       if (y - x > kLtPartTools || n - y > kLtPartTools) continue;
       const double px = (double)pow3(x), py = (double)pow3(y), pn = (double)pow3(n);
@@ -520,7 +519,16 @@ inline void lanetree_split(const TB& t, uint32_t* x_out, uint32_t* y_out, uint32
   }
   *x_out = bx;
   *y_out = by;
-  const uint64_t cap = pow3(bx) / kLtMinRootsPerBlock;
+  return best;
+}
+
+// The batch's levels (every block gets kLtMinRootsPerBlock roots or more)
+// and the blocks its scenario's roots are split over.
+template <typename TB>
+inline void lanetree_split(const TB& t, uint32_t* x_out, uint32_t* y_out, uint32_t* nblocks) {
+  const uint64_t want_blocks = (pow3(t.n) + kLtBlockMappings - 1) / kLtBlockMappings;
+  lanetree_levels(t, kLtMinRootsPerBlock * want_blocks, x_out, y_out);
+  const uint64_t cap = pow3(*x_out) / kLtMinRootsPerBlock;
   uint64_t nb = want_blocks < cap ? want_blocks : cap;
   *nblocks = (uint32_t)(nb < 1 ? 1 : nb);
 }
@@ -531,13 +539,17 @@ struct LtView {
   uint32_t pred[BF_MAX_TOOLS], cpu[BF_MAX_TOOLS], wnow[BF_MAX_TOOLS];
 };
 
-// Record of one scenario of the lane-tree batch search: its tools renumbered
-// with the sources first (each group in the scenario's order: the order of
-// relabel_sources_first) and its levels.  Built straight from the desc; the
-// slowdown constants are those of build_tables, taken over from the previous
-// record built on this thread when the slowdown table is the same (the
-// scenarios of a batch usually share one).
-inline void lanetree_record(const bf_scenario_desc* d, bfk::LaneTreeRecord* r) {
+// Record of one scenario of a lane-tree search: its tools renumbered with the
+// sources first (each group in the scenario's order: the order of
+// relabel_sources_first) and its levels -- the batch's (min_roots == 0), or
+// those of a search whose lanes share 3^x >= min_roots roots (nblocks = 1).
+// Built straight from the desc; the slowdown constants are those of
+// build_tables, taken over from the previous record built on this thread
+// when the slowdown table is the same (the scenarios of a batch usually
+// share one).  *events (if given) receives the levels' estimated events
+// per mapping (lanetree_levels' cost over 3^n).
+inline void lanetree_record(const bf_scenario_desc* d, bfk::LaneTreeRecord* r, uint64_t min_roots = 0,
+                            double* events = nullptr) {
   const uint32_t n = d->n;
   uint32_t order[BF_MAX_TOOLS], pos[BF_MAX_TOOLS], k = 0;
   for (uint32_t v = 0; v < n; ++v)
@@ -577,7 +589,44 @@ inline void lanetree_record(const bf_scenario_desc* d, bfk::LaneTreeRecord* r) {
     r->fshift[j] = last.fshift[j];
     r->fmagic[j] = last.fmagic[j];
   }
-  lanetree_split(view, &r->x, &r->y, &r->nblocks);
+  if (min_roots == 0) {
+    lanetree_split(view, &r->x, &r->y, &r->nblocks);
+  } else {
+    const double cost = lanetree_levels(view, min_roots, &r->x, &r->y);
+    r->nblocks = 1;
+    if (events) *events = cost / (double)pow3(n);
+  }
+}
+
+// Whether a full search of a scenario goes to the one-scenario lane-tree
+// kernel (record rec, estimated events per mapping lt_events) rather than
+// the search kernel (whole-space tables rt, plan rp, window rw).  The search
+// kernel's cost per mapping grows with its events per mapping -- R-estimate
+// events after its prefix checkpoint shared by 3^(M+I) mappings, its mid
+// checkpoint by 3^I -- times its window width (each event scans the window),
+// at full warp efficiency when its lanes follow the same structure; the
+// lane tree's with its own events per mapping, at the divergence of lanes
+// on different mappings.  Measured (full searches, 152-SM GB300): the lane
+// tree is faster on every layered and fan-out/fan-in DAG of 12 to 16 tools
+// tried (16-tool layered workload 2.70 -> 1.70 ms; layered 14 tools 0.60 ->
+// 0.21 ms) and on the chain and spine DAGs of 13 and 14 tools; slower when
+// its roots are whole mappings (x = n: the 12-tool fan-out/fan-in 0.053 ->
+// 0.081 ms) and on chain and spine DAGs of 15 and 16 tools, whose narrow
+// windows (4 to 6 slots) make the search kernel's events cheap (16-tool
+// chain 0.67 ms against 0.82): there the search kernel's events x window
+// width is 4.4 to 6.8 times the lane tree's estimate, in the cases the lane
+// tree wins 6.7 to 21 times.
+constexpr double kLtPreferRatio = 8.0;
+inline bool lanetree_preferred(const bfk::Tables& rt, const bfk::Plan& rp, const bfk::Tables& rw,
+                               const bfk::LaneTreeRecord& rec, double lt_events) {
+  const uint32_t n = rt.n;
+  if (rec.x >= n) return false;
+  if (n <= 14u) return true;
+  uint32_t R[BF_MAX_TOOLS + 1] = {};
+  retired_estimate(rt, R);
+  const uint32_t P = rp.P, I = rp.I;
+  const double sk_events = R[P] / (double)pow3(rp.M + I) + (R[n - I] - R[P]) / (double)pow3(I) + (n - R[n - I]);
+  return sk_events * rw.n >= kLtPreferRatio * lt_events;
 }
 
 }  // namespace host

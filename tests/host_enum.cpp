@@ -210,25 +210,28 @@ extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bo
   return pruned_width<20>(tb, tw, plan);
 }
 
-// The lane-tree batch kernel's search (bf_lanetree.cuh) of one scenario,
-// with the record bf_search_batch builds for it: every block of its roots
-// with `lanes` lanes, lane l taking the block's roots l, l + lanes, ...
-// (the kernel hands roots out from a shared counter; any order gives the
-// same mappings).  Every mapping reported to the sink is stored at its
-// canonical index; out[] starts at 0xFFFFFFFF (infeasible mappings are not
-// reported) and a second report of one index stores 0xDEADBEEF.
-// info[0..2] = x, y, blocks.
-extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint32_t* out, uint32_t* info) {
-  if (d->n > kLtBatchTools || lanes == 0) return -1;
+// A lane-tree search (bf_lanetree.cuh) of one scenario: with min_roots == 0
+// the batch kernel's (the record bf_search_batch builds, 6-bit tables in two
+// chunks, n <= 12), otherwise the one-scenario kernel's (levels for at least
+// min_roots roots, three chunks, n <= 16).  The roots are split over the
+// record's blocks, and every block's with `lanes` lanes, lane l taking the
+// block's roots l, l + lanes, ... (the kernels hand roots out from counters;
+// any order gives the same mappings).  Every mapping reported to the sink is
+// stored at its canonical index; out[] starts at 0xFFFFFFFF (infeasible
+// mappings are not reported) and a second report of one index stores
+// 0xDEADBEEF.  info[0..2] = x, y, blocks.
+template <uint32_t NC>
+static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, uint32_t* out,
+                            uint32_t* info) {
   LaneTreeRecord rec;
-  host::lanetree_record(d, &rec);
+  host::lanetree_record(d, &rec, min_roots);
   info[0] = rec.x;
   info[1] = rec.y;
   info[2] = rec.nblocks;
   const uint64_t total = host::pow3(d->n), roots = host::pow3(rec.x);
   for (uint64_t j = 0; j < total; ++j) out[j] = 0xFFFFFFFFu;
-  std::vector<LtShared> shared(1);
-  LtShared& S = shared[0];
+  std::vector<LtSharedT<NC>> shared(1);
+  LtSharedT<NC>& S = shared[0];
   S.rec = rec;
   threadIdx.x = 0;
   blockDim.x = 1;
@@ -252,4 +255,11 @@ extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint32_t
     }
   }
   return 0;
+}
+
+extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, uint32_t* out,
+                             uint32_t* info) {
+  if (lanes == 0) return -1;
+  if (min_roots == 0) return d->n <= kLtBatchTools ? host_lanetree_nc<2>(d, lanes, 0, out, info) : -1;
+  return d->n <= kLtMaxTools ? host_lanetree_nc<3>(d, lanes, min_roots, out, info) : -1;
 }

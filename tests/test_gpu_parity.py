@@ -193,6 +193,32 @@ def test_late_sources_renumbered_searches():
     assert [(r.index, r.makespan_us) for r in bf.search_batch(scns)] == want
 
 
+def test_lanetree_whole_space_search():
+    """Full searches of 10 to 16 tools run the one-scenario lane-tree kernel (every lane of the GPU on
+    one scenario's roots, a shared tail of roots, the result written by the last block): random DAGs
+    with small integer times (queue ties, VRAM-blocked queues, infeasible starts), late sources and
+    last tools that wait for all others, up to 16 tools with queued tools numbered up to 15; each
+    searched twice on one handle (every launch resets its state), against the oracle."""
+    rng = np.random.default_rng(77)
+    for t in range(14):
+        n = 10 + t % 7
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.2, 0.35])), tight=bool(t % 3 != 2),
+                              contention=bool(t % 4), max_time=int(rng.choice([5, 9, 40])))
+        pred = list(base.pred_mask)
+        if t % 3 == 0:
+            pred[int(rng.integers(n // 2, n))] = 0
+        if t % 4 == 1:
+            pred[n - 1] = (1 << (n - 1)) - 1
+        scn = S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
+                         base.vram_budget_mib, base.slowdown_q10)
+        want = oracle.search(scn, THREADS)
+        with bf.create_scenario(scn) as h:
+            for _ in range(2):
+                r = bf.search_best(h)
+                assert (r.index, r.makespan_us) == want, (t, n)
+        assert r.modes == S.mapping_modes(r.index, n)
+
+
 def test_degenerate_budgets_all_paths():
     """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
     the batch, the branch and bound and the tree search, against the oracle."""

@@ -45,13 +45,15 @@ def host():
         assert lib.host_eval(ctypes.byref(d), first, count, mode, ms.ctypes.data, info.ctypes.data) == 0
         return ms.astype(np.uint64), info
     run.pruned = lambda scn, bound: lib.host_pruned(ctypes.byref(bf.to_desc(scn)), bound)
-    lib.host_lanetree.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint32, ctypes.c_void_p, ctypes.c_void_p]
+    lib.host_lanetree.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint32, ctypes.c_uint64, ctypes.c_void_p,
+                                  ctypes.c_void_p]
     lib.host_lanetree.restype = ctypes.c_int
 
-    def lanetree(scn, lanes):
+    def lanetree(scn, lanes, min_roots=0):
         ms = np.zeros(3 ** scn.n, np.uint32)
         info = np.zeros(3, np.uint32)
-        assert lib.host_lanetree(ctypes.byref(bf.to_desc(scn)), lanes, ms.ctypes.data, info.ctypes.data) == 0
+        assert lib.host_lanetree(ctypes.byref(bf.to_desc(scn)), lanes, min_roots, ms.ctypes.data,
+                                 info.ctypes.data) == 0
         return ms.astype(np.uint64), info
     run.lanetree = lanetree
     return run
@@ -145,8 +147,8 @@ def test_tie_order_scenarios_host(host):
             assert got == tuple(want), (t, bound, got, want)
 
 
-def _same_lanetree(host, scn, lanes):
-    got, info = host.lanetree(scn, lanes)
+def _same_lanetree(host, scn, lanes, min_roots=0):
+    got, info = host.lanetree(scn, lanes, min_roots)
     want, _ = oracle.eval_range(scn, 0, 3 ** scn.n, THREADS)
     bad = np.flatnonzero(got != want)
     assert bad.size == 0, (f"levels x={int(info[0])} y={int(info[1])}, {int(info[2])} blocks: {bad.size} "
@@ -187,3 +189,35 @@ def test_lanetree_workloads_and_ties(host):
         _same_lanetree(host, scn, 32)
     for scn in tie_order_scenarios():
         _same_lanetree(host, scn, 3)
+
+
+def test_lanetree_whole_space_records(host):
+    """The one-scenario lane-tree search (three 6-bit table chunks, roots of up to 16 tools, levels for
+    a given number of roots) on random DAGs of 10-14 tools -- queued tools numbered up to 13, late
+    sources, last tools that wait for all others -- and on the 16-tool layered workload's first 13
+    tools: every mapping against the oracle, with roots from 3^(n-8) up to the whole space."""
+    rng = np.random.default_rng(93)
+    xs = set()
+    for t in range(24):
+        n = int(rng.integers(10, 13)) if t % 6 else 14
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.25, 0.5])), tight=bool(t % 3),
+                              contention=bool(t % 4), max_time=int(rng.choice([3, 7, 40, 2000])))
+        pred = list(base.pred_mask)
+        if t % 3 == 0:
+            pred[int(rng.integers(n // 2, n))] = 0
+        if t % 4 == 1:
+            pred[n - 1] = (1 << (n - 1)) - 1
+        scn = S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
+                         base.vram_budget_mib, base.slowdown_q10)
+        min_roots = 3 ** int(rng.integers(n - 8, n + 1))
+        info = _same_lanetree(host, scn, (1, 3, 32)[t % 3], min_roots)
+        assert int(info[2]) == 1 and 3 ** int(info[0]) >= min_roots
+        xs.add(int(info[0]) == n)
+    assert xs == {False, True}
+    full = S.config(2)
+    m = 13
+    cut = S.Scenario(m, [p & ((1 << m) - 1) for p in full.pred_mask[:m]], full.cpu_us[:m], full.gpu_us[:m],
+                     full.xfer_us[:m], full.load_us[:m], full.vram_mib[:m], full.vram_budget_mib,
+                     full.slowdown_q10)
+    info = _same_lanetree(host, cut, 32, 3 ** 10)
+    assert int(info[0]) >= 10 and int(info[1]) < m
