@@ -124,9 +124,10 @@ int wait_stream(cudaStream_t st, const char* who) {
     const auto us = std::chrono::duration_cast<std::chrono::microseconds>(std::chrono::steady_clock::now() - t0).count();
     const uint32_t limit = g_wait_timeout_ms.load(std::memory_order_relaxed);
     if (limit && us > 1000LL * limit) return fail(BF_ETIMEOUT, "%s: GPU work not finished after %u ms", who, limit);
-    // Short waits (the tree search's level steps) are polled without sleeping
-    // for the first 200 us; longer ones sleep 20 us between polls.
-    if (us > 200) std::this_thread::sleep_for(std::chrono::microseconds(20));
+    // The first 5 ms are polled without sleeping: a sleep of 20 us lasts about
+    // 75 us on Linux, which would add up to that much to every search of a
+    // millisecond or two.  Longer waits sleep 20 us between polls.
+    if (us > 5000) std::this_thread::sleep_for(std::chrono::microseconds(20));
   }
 }
 
@@ -382,8 +383,10 @@ cudaError_t launch_list(const bf_scenario* scn, const uint64_t* idx, uint64_t co
   return e;
 }
 
-// One launch of the search kernel; its last warp writes the best key into the
-// host mirror (scn->h_scratch->search.key) and resets the launch state.
+// One launch of the search kernel -- or, for the whole space of a scenario
+// with a lane-tree record, of the lane-tree kernel; its last block writes
+// the best key into the host mirror (scn->h_scratch->search.key) and resets
+// the launch state.
 int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result* out,
                cudaStream_t st, const char* who) {
   if (count == 0) {
@@ -393,6 +396,15 @@ int run_search(const bf_scenario* scn, uint64_t first, uint64_t count, bf_result
   // The whole space runs on the renumbered tables; a part of it keeps the
   // scenario's numbering, in which an index range is a box of the split.
   const bool whole = first == 0 && count == pow3(scn->desc.n);
+  if (whole && scn->lanetree) {
+    const cudaError_t e = bfk::launch_lanetree_single(&scn->d_scratch->lt, scn->desc.n, scn->lt_x, scn->lt_blocks,
+                                                      &scn->d_scratch->search, scn->d_host_search_key, st);
+    if (e != cudaSuccess) return cuda_fail(e, who);
+    const int rc = wait_stream(st, who);
+    if (rc != BF_OK) return rc;
+    fill_result(*static_cast<volatile unsigned long long*>(&scn->h_scratch->search.key), scn->desc.n, first, out);
+    return BF_OK;
+  }
   const bfk::Tables& tb = whole ? scn->rtables : scn->tables;
   const bfk::Tables& tw = whole ? scn->rwindow : scn->window;
   const bfk::Plan plan = make_plan(whole ? scn->rplan : scn->plan, first, count, kSearchTasks);
@@ -431,6 +443,18 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
     split_and_window_pruned(s->rtables, &s->pplan, &s->pwindow);
   }
   cudaError_t e = cudaGetDevice(&s->device);
+  bfk::LaneTreeRecord ltrec;
+  if (e == cudaSuccess && desc->n >= bfk::kLtSingleMinTools && desc->n <= bfk::kLtMaxTools) {
+    e = bfk::lanetree_single_blocks(desc->n, &s->lt_blocks);
+    if (e == cudaSuccess) {
+      double lt_events = 0.0;
+      bfk::host::lanetree_record(desc, &ltrec,
+                                 (uint64_t)s->lt_blocks * bfk::kLtLaunchThreads * bfk::kLtSingleRootsPerLane,
+                                 &lt_events);
+      s->lanetree = bfk::host::lanetree_preferred(s->rtables, s->rplan, s->rwindow, ltrec, lt_events);
+      s->lt_x = ltrec.x;
+    }
+  }
   if (e == cudaSuccess) e = lib_malloc(reinterpret_cast<void**>(&s->d_scratch), sizeof(bf_scratch));
   if (e == cudaSuccess) e = lib_malloc_host(reinterpret_cast<void**>(&s->h_scratch), sizeof(bf_scratch));
   if (e != cudaSuccess) {
@@ -447,6 +471,8 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   void* mirror = nullptr;
   e = cudaMemset(&s->d_scratch->search, 0, sizeof(bfk::SearchSync));
   if (e == cudaSuccess) e = cudaMemset(&s->d_scratch->search.key, 0xFF, sizeof(unsigned long long));
+  if (e == cudaSuccess && s->lanetree)
+    e = cudaMemcpy(&s->d_scratch->lt, &ltrec, sizeof ltrec, cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaHostGetDevicePointer(&mirror, s->h_scratch, 0);
   if (e != cudaSuccess) {
     const int code = cuda_fail(e, "bf_create_scenario");
