@@ -476,11 +476,14 @@ inline bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n, uint32_t block_wa
   return make_plan(base, 0, pow3(n), (uint64_t)fill * groups);
 }
 
-// Mappings a block of the lane-tree batch kernel aims to search, and the
-// fewest roots a block hands out (two per lane of 256).  Many short blocks
-// keep every SM busy to the end of the launch: 4096 x 3^10 batch call, blocks
-// per scenario (roots per block) 1 (1024+) 16.2 ms, 2 15.4, 4 (512+) 15.1,
-// 8 (512+) 14.8, 8 (256+) 14.8, 16 (256+) 15.8, 32 (128+) 18.0.
+// Mappings a block of the lane-tree batch kernel aims to search (a 10-tool
+// scenario gets ceil(3^10 / 7381) = 9 blocks), and the fewest roots a block
+// hands out (two per lane of 256).  Many short blocks keep every SM busy to
+// the end of the launch: 4096 x 3^10 batch call, an earlier form of the
+// kernel, from 16.2 ms at one block per scenario (1024+ roots) to 14.8 ms at
+// 9 and 18.0 ms at 32 (128+); the current kernel at 7, 9, 12 and 16 blocks
+// per scenario 13.5, 13.4, 13.6 and 13.8 ms, at 9 blocks with 256+ roots
+// 13.4 ms.
 constexpr uint64_t kLtBlockMappings = 7381;
 constexpr uint64_t kLtMinRootsPerBlock = 512;
 
