@@ -605,12 +605,21 @@ def test_batch_two_kernel_groups():
     assert [(r.index, r.makespan_us) for r in res] == list(zip(o_i.tolist(), o_m.tolist()))
 
 
-def test_search_launch_state_across_calls():
+@pytest.mark.parametrize("which", ["fanout12", "layered13"])
+def test_search_launch_state_across_calls(which):
     """A search call is one launch whose last block writes the result to the handle's host mirror and
     resets the launch state: every kind of search, and empty and partial ranges, on one handle and on
-    two streams in turn, must each give the oracle's answer."""
+    two streams in turn, must each give the oracle's answer.  The 12-tool workload runs its full
+    search on the search kernel; the 16-tool workload's first 13 tools run theirs on the lane-tree
+    kernel, which shares the launch state with the range searches of the same handle."""
     import torch
-    scn = S.config1()
+    if which == "fanout12":
+        scn = S.config1()
+    else:
+        full, m = S.config2(), 13
+        scn = S.Scenario(m, [p & ((1 << m) - 1) for p in full.pred_mask[:m]], full.cpu_us[:m], full.gpu_us[:m],
+                         full.xfer_us[:m], full.load_us[:m], full.vram_mib[:m], full.vram_budget_mib,
+                         full.slowdown_q10)
     total = 3 ** scn.n
     want = oracle.search(scn, THREADS)
     part = (total // 3, total // 5)
@@ -625,6 +634,8 @@ def test_search_launch_state_across_calls():
             assert not empty.feasible and empty.index == 17
             r = bf.search_range(h, part[0], part[1], st)
             assert (r.index, r.makespan_us) == want_part
+            r = bf.search_best(h, st)
+            assert (r.index, r.makespan_us) == want
             r = bf.search_pruned(h, None, st)
             assert (r.index, r.makespan_us) == want
             rt, _ = bf.search_tree(h, bf.SPACE_FULL, True, None, st)
