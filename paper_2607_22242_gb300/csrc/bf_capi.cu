@@ -452,6 +452,10 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
                                  (uint64_t)s->lt_blocks * bfk::kLtLaunchThreads * bfk::kLtSingleRootsPerLane,
                                  &lt_events);
       s->lanetree = bfk::host::lanetree_preferred(s->rtables, s->rplan, s->rwindow, ltrec, lt_events);
+      if (s->lanetree)
+        bfk::host::lanetree_sampled_levels(ltrec, (uint64_t)s->lt_blocks * bfk::kLtLaunchThreads *
+                                                      bfk::kLtSingleRootsPerLane,
+                                           &ltrec.x, &ltrec.y);
       s->lt_x = ltrec.x;
     }
   }

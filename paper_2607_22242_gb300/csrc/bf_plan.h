@@ -536,6 +536,163 @@ inline void lanetree_split(const TB& t, uint32_t* x_out, uint32_t* y_out, uint32
   *nblocks = (uint32_t)(nb < 1 ? 1 : nb);
 }
 
+// Sampled work of a one-scenario lane-tree search, for choosing its levels.
+// A whole-GPU search runs millions of jobs per level, so its levels are
+// worth a closer estimate than the batch's: the closed-form estimate of
+// lanetree_levels took one level of 4 tools below roots of 12 for the
+// 16-tool layered workload (2.37 events and 0.60 jobs per mapping on the
+// host emulator, 1.67 ms), where one tool and then 3 take 2.17 and 0.63
+// (1.59 ms).
+//
+// lt_sample_events simulates one mapping (mode[t] per tool of the record's
+// numbering) with the model's arithmetic in 64-bit integers and returns, for
+// every b in [0, n], ev[b] = the events before the first tool >= b becomes
+// ready (all its events if none does) and reached[b] = whether one does
+// (the mapping has not been found infeasible before).  Estimates only: no
+// result depends on them.
+inline void lt_sample_events(const bfk::LaneTreeRecord& r, const uint8_t* mode, uint32_t* ev, bool* reached) {
+  const uint32_t n = r.n;
+  uint32_t first[bfk::kLtMaxTools];
+  uint64_t end[bfk::kLtMaxTools];  // CPU: real end; GPU: end stamp on the virtual clock
+  uint32_t fifo[bfk::kLtMaxTools], qhead = 0, qtail = 0;
+  uint32_t cpu = 0u, now = 0u, que = 0u;  // the modes as tool sets
+  for (uint32_t t = 0; t < n; ++t) {
+    first[t] = 0xFFFFFFFFu;
+    cpu |= mode[t] == 0 ? 1u << t : 0u;
+    now |= mode[t] == 1 ? 1u << t : 0u;
+    que |= mode[t] == 2 ? 1u << t : 0u;
+  }
+  uint32_t pend = r.all_mask, run = 0u, done = 0u;
+  uint64_t T = 0, V = 0, vram = 0;
+  uint32_t events = 0;
+  bool dead = false;
+  for (;;) {
+    uint32_t ready = 0u;
+    for (uint32_t m = pend; m; m &= m - 1u) {
+      const uint32_t t = (uint32_t)__builtin_ctz(m);
+      if ((r.pred[t] & ~done) == 0u) ready |= 1u << t;
+    }
+    pend &= ~ready;
+    for (uint32_t m = ready; m; m &= m - 1u) {
+      const uint32_t t = (uint32_t)__builtin_ctz(m);
+      first[t] = events;
+      if ((que >> t) & 1u) {
+        fifo[qtail++] = t;
+      } else {
+        end[t] = (cpu >> t) & 1u ? T + r.dur[0][t] : V + r.dur[1][t];
+        vram += (now >> t) & 1u ? r.vram[t] : 0u;
+        run |= 1u << t;
+      }
+    }
+    if ((ready & now) && vram > r.budget) {
+      dead = true;
+      break;
+    }
+    if (qhead < qtail && !(run & que)) {
+      const uint32_t h = fifo[qhead];
+      if ((r.big_mask >> h) & 1u) {
+        dead = true;
+        break;
+      }
+      if (vram + r.vram[h] <= r.budget) {
+        end[h] = V + r.dur[2][h];
+        vram += r.vram[h];
+        run |= 1u << h;
+        ++qhead;
+      }
+    }
+    if (!run) break;  // every tool has ended
+    uint32_t k = 0;
+    uint64_t tc = ~0ull, gm = ~0ull;
+    for (uint32_t m = run; m; m &= m - 1u) {
+      const uint32_t t = (uint32_t)__builtin_ctz(m);
+      if ((cpu >> t) & 1u) {
+        tc = end[t] < tc ? end[t] : tc;
+      } else {
+        ++k;
+        gm = end[t] < gm ? end[t] : gm;
+      }
+    }
+    const uint64_t f = r.f[k ? k : 1];
+    const uint64_t tg = k ? T + (((gm - V) * f + 0xFFFFFull) >> 20) : ~0ull;
+    const bool gpu_event = k && tg <= tc;
+    if (gpu_event) {
+      T = tg;
+      V = gm;
+    } else {
+      if (k) V += ((tc - T) << 20) / f;
+      T = tc;
+    }
+    ++events;
+    for (uint32_t m = run; m; m &= m - 1u) {
+      const uint32_t t = (uint32_t)__builtin_ctz(m);
+      const bool ends = (cpu >> t) & 1u ? end[t] == T : (gpu_event && end[t] == V);
+      if (ends) {
+        run &= ~(1u << t);
+        done |= 1u << t;
+        vram -= (cpu >> t) & 1u ? 0u : r.vram[t];
+      }
+    }
+  }
+  uint32_t earliest = 0xFFFFFFFFu;
+  ev[n] = events;
+  reached[n] = !dead;
+  for (uint32_t b = n; b-- > 0;) {
+    earliest = first[b] < earliest ? first[b] : earliest;
+    reached[b] = earliest != 0xFFFFFFFFu;
+    ev[b] = reached[b] ? earliest : events;
+  }
+}
+
+// Levels of a one-scenario record from kLtLevelSamples mappings drawn
+// uniformly (a fixed seed: the same choice on every machine), for records the
+// search will run (about 0.1 ms of host time at 16 tools): among the
+// splits lanetree_levels allows, the one of least sampled cost -- a root
+// runs its mappings' events up to ev[x], a level-1 job up to ev[y] from
+// there, a leaf to the end, and a job costs half an event more; jobs exist
+// only below checkpoints that were reached.
+constexpr uint32_t kLtLevelSamples = 128;
+inline void lanetree_sampled_levels(const bfk::LaneTreeRecord& r, uint64_t min_roots, uint32_t* x_out,
+                                    uint32_t* y_out) {
+  const uint32_t n = r.n;
+  uint64_t S[bfk::kLtMaxTools + 1] = {}, A[bfk::kLtMaxTools + 1] = {};
+  uint64_t state = 0x9E3779B97F4A7C15ull;
+  uint8_t mode[bfk::kLtMaxTools];
+  uint32_t ev[bfk::kLtMaxTools + 1];
+  bool reached[bfk::kLtMaxTools + 1];
+  for (uint32_t k = 0; k < kLtLevelSamples; ++k) {
+    for (uint32_t t = 0; t < n; ++t) {  // splitmix64 (Steele, Lea and Flood, OOPSLA 2014)
+      uint64_t z = (state += 0x9E3779B97F4A7C15ull);
+      z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+      z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+      mode[t] = (uint8_t)((z ^ (z >> 31)) % 3u);
+    }
+    lt_sample_events(r, mode, ev, reached);
+    for (uint32_t b = 0; b <= n; ++b) {
+      S[b] += ev[b];
+      A[b] += reached[b] ? 1u : 0u;
+    }
+  }
+  uint32_t xmin = 0;
+  while (xmin < n && pow3(xmin) < min_roots) ++xmin;
+  if (n > 2u * kLtPartTools && xmin < n - 2u * kLtPartTools) xmin = n - 2u * kLtPartTools;
+  uint64_t best = ~0ull;
+  for (uint32_t x = xmin; x <= n && x <= kLtRootParts * kLtPartTools; ++x) {
+    for (uint32_t y = (x == n ? n : x + 1u); y <= n; ++y) {
+      if (y - x > kLtPartTools || n - y > kLtPartTools) continue;
+      const uint64_t px = pow3(x), py = pow3(y), pn = pow3(n);
+      // Twice the cost, summed over the samples (half events are whole).
+      const uint64_t cost = 2u * (px * S[x] + py * (S[y] - S[x]) + pn * (S[n] - S[y])) + px * kLtLevelSamples +
+                            (x < n ? py * A[x] : 0u) + (y < n ? pn * A[y] : 0u);
+      if (cost < best) {
+        best = cost;
+        *x_out = x;
+        *y_out = y;
+      }
+    }
+  }
+}
+
 // The tables a lane-tree record's split estimate reads (n, pred, cpu, wnow).
 struct LtView {
   uint32_t n;

@@ -213,7 +213,9 @@ extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bo
 // A lane-tree search (bf_lanetree.cuh) of one scenario: with min_roots == 0
 // the batch kernel's (the record bf_search_batch builds, 6-bit tables in two
 // chunks, n <= 12), otherwise the one-scenario kernel's (levels for at least
-// min_roots roots, three chunks, n <= 16).  The roots are split over the
+// min_roots roots -- the closed-form estimate's, or with `sampled` those of
+// lanetree_sampled_levels, as bf_create_scenario takes them -- three
+// chunks, n <= 16).  The roots are split over the
 // record's blocks, and every block's with `lanes` lanes, lane l taking the
 // block's roots l, l + lanes, ... (the kernels hand roots out from counters;
 // any order gives the same mappings).  Every mapping reported to the sink is
@@ -221,10 +223,11 @@ extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bo
 // mappings are not reported) and a second report of one index stores
 // 0xDEADBEEF.  info[0..2] = x, y, blocks.
 template <uint32_t NC>
-static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, uint32_t* out,
-                            uint32_t* info) {
+static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, int sampled,
+                            uint32_t* out, uint32_t* info) {
   LaneTreeRecord rec;
   host::lanetree_record(d, &rec, min_roots);
+  if (sampled) host::lanetree_sampled_levels(rec, min_roots, &rec.x, &rec.y);
   info[0] = rec.x;
   info[1] = rec.y;
   info[2] = rec.nblocks;
@@ -257,9 +260,9 @@ static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t 
   return 0;
 }
 
-extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, uint32_t* out,
-                             uint32_t* info) {
+extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, int sampled,
+                             uint32_t* out, uint32_t* info) {
   if (lanes == 0) return -1;
-  if (min_roots == 0) return d->n <= kLtBatchTools ? host_lanetree_nc<2>(d, lanes, 0, out, info) : -1;
-  return d->n <= kLtMaxTools ? host_lanetree_nc<3>(d, lanes, min_roots, out, info) : -1;
+  if (min_roots == 0) return d->n <= kLtBatchTools ? host_lanetree_nc<2>(d, lanes, 0, 0, out, info) : -1;
+  return d->n <= kLtMaxTools ? host_lanetree_nc<3>(d, lanes, min_roots, sampled, out, info) : -1;
 }

@@ -45,14 +45,14 @@ def host():
         assert lib.host_eval(ctypes.byref(d), first, count, mode, ms.ctypes.data, info.ctypes.data) == 0
         return ms.astype(np.uint64), info
     run.pruned = lambda scn, bound: lib.host_pruned(ctypes.byref(bf.to_desc(scn)), bound)
-    lib.host_lanetree.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint32, ctypes.c_uint64, ctypes.c_void_p,
-                                  ctypes.c_void_p]
+    lib.host_lanetree.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint32, ctypes.c_uint64, ctypes.c_int,
+                                  ctypes.c_void_p, ctypes.c_void_p]
     lib.host_lanetree.restype = ctypes.c_int
 
-    def lanetree(scn, lanes, min_roots=0):
+    def lanetree(scn, lanes, min_roots=0, sampled=False):
         ms = np.zeros(3 ** scn.n, np.uint32)
         info = np.zeros(3, np.uint32)
-        assert lib.host_lanetree(ctypes.byref(bf.to_desc(scn)), lanes, min_roots, ms.ctypes.data,
+        assert lib.host_lanetree(ctypes.byref(bf.to_desc(scn)), lanes, min_roots, int(sampled), ms.ctypes.data,
                                  info.ctypes.data) == 0
         return ms.astype(np.uint64), info
     run.lanetree = lanetree
@@ -147,8 +147,8 @@ def test_tie_order_scenarios_host(host):
             assert got == tuple(want), (t, bound, got, want)
 
 
-def _same_lanetree(host, scn, lanes, min_roots=0):
-    got, info = host.lanetree(scn, lanes, min_roots)
+def _same_lanetree(host, scn, lanes, min_roots=0, sampled=False):
+    got, info = host.lanetree(scn, lanes, min_roots, sampled)
     want, _ = oracle.eval_range(scn, 0, 3 ** scn.n, THREADS)
     bad = np.flatnonzero(got != want)
     assert bad.size == 0, (f"levels x={int(info[0])} y={int(info[1])}, {int(info[2])} blocks: {bad.size} "
@@ -193,7 +193,7 @@ def test_lanetree_workloads_and_ties(host):
 
 def test_lanetree_whole_space_records(host):
     """The one-scenario lane-tree search (three 6-bit table chunks, roots of up to 16 tools, levels for
-    a given number of roots) on random DAGs of 10-14 tools -- queued tools numbered up to 13, late
+    a given number of roots, from the closed-form or the sampled estimate) on random DAGs of 10-14 tools -- queued tools numbered up to 13, late
     sources, last tools that wait for all others -- and on the 16-tool layered workload's first 13
     tools: every mapping against the oracle, with roots from 3^(n-8) up to the whole space."""
     rng = np.random.default_rng(93)
@@ -210,7 +210,7 @@ def test_lanetree_whole_space_records(host):
         scn = S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
                          base.vram_budget_mib, base.slowdown_q10)
         min_roots = 3 ** int(rng.integers(n - 8, n + 1))
-        info = _same_lanetree(host, scn, (1, 3, 32)[t % 3], min_roots)
+        info = _same_lanetree(host, scn, (1, 3, 32)[t % 3], min_roots, sampled=bool(t % 2))
         assert int(info[2]) == 1 and 3 ** int(info[0]) >= min_roots
         xs.add(int(info[0]) == n)
     assert xs == {False, True}
@@ -219,5 +219,5 @@ def test_lanetree_whole_space_records(host):
     cut = S.Scenario(m, [p & ((1 << m) - 1) for p in full.pred_mask[:m]], full.cpu_us[:m], full.gpu_us[:m],
                      full.xfer_us[:m], full.load_us[:m], full.vram_mib[:m], full.vram_budget_mib,
                      full.slowdown_q10)
-    info = _same_lanetree(host, cut, 32, 3 ** 10)
+    info = _same_lanetree(host, cut, 32, 3 ** 10, sampled=True)
     assert int(info[0]) >= 10 and int(info[1]) < m
