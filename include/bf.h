@@ -167,10 +167,11 @@ BF_API int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t coun
  * brute-force oracle of §2.3/§4.1 (as bf_search_best) for descs[i].  The paper
  * searches one workflow at a time; running many per launch is this library's
  * addition, for callers that score many workflows or many candidate
- * contention tables (the calibration of Table 2's S5 latencies) together.  All descs are validated first;
- * the first invalid one fails the call with BF_EINVAL naming its position.
- * Allocates and frees its device scratch (packed tables + one key per
- * scenario) per call.  Blocks until the results are on the host. */
+ * contention tables (the calibration of Table 2's S5 latencies) together.  All descs are validated
+ * before any GPU work; the first invalid one (lowest position) fails the call with BF_EINVAL naming
+ * its position.  Allocates its device scratch (packed tables + one key per scenario) from the
+ * device's default stream-ordered memory pool on cuda_stream and frees it there after its kernels,
+ * also when the wait times out (BF_ETIMEOUT).  Blocks until the results are on the host. */
 BF_API int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                     void* cuda_stream);
 

@@ -75,6 +75,14 @@ cudaError_t lib_malloc_host(void** p, size_t bytes) {
   return cudaMallocHost(p, bytes);
 }
 
+// Stream-ordered device memory from the device's default pool: no device-wide
+// synchronisation on free (cudaFree has one), and a free enqueued after a
+// call's kernels waits for them even when the host stopped waiting.
+cudaError_t lib_malloc_async(void** p, size_t bytes, cudaStream_t st) {
+  if (inject_alloc_failure()) return cudaErrorMemoryAllocation;
+  return cudaMallocAsync(p, bytes, st);
+}
+
 int validate(const bf_scenario_desc* d, const char* who) {
   if (!d) return fail(BF_EINVAL, "%s: desc is NULL", who);
   const uint32_t n = d->n;
@@ -287,17 +295,34 @@ void parallel_parts(uint32_t count, std::vector<Part>& parts, Work work) {
   work(0u, count, &parts[0]);
 }
 
+// Whether a desc can be searched by a batch (valid, n <= BF_MAX_TOOLS_ENUM);
+// the record builders check each desc before they read it, on the host pool,
+// and the caller reports the lowest failing position.  A failed check on a
+// pool thread writes that thread's error text only.
+bool batch_desc_ok(const bf_scenario_desc* d) {
+  try {  // a failed check formats its message, which may allocate; no exception leaves a pool thread
+    return validate(d, "bf_search_batch") == BF_OK && require_enum(*d, "bf_search_batch") == BF_OK;
+  } catch (...) {
+    return false;
+  }
+}
+
 // Batch-kernel records (tables, window tables, plan) of descs[ids[j]], j <
 // count; the largest window, task count and whether any plan has an inner
-// level are returned too.
+// level are returned too, and *bad lowered to the lowest position whose desc
+// fails batch_desc_ok (its record is left unbuilt).
 void build_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count, bfk::BatchRecord* recs,
-                   uint32_t* wmax, uint32_t* pmax, uint32_t* any_inner) {
+                   uint32_t* wmax, uint32_t* pmax, uint32_t* any_inner, uint32_t* bad) {
   struct Part {
-    uint32_t wmax = 0, pmax = 0, inner = 0;
+    uint32_t wmax = 0, pmax = 0, inner = 0, bad = 0xFFFFFFFFu;
   };
   std::vector<Part> parts;
   parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part* part) {
     for (uint32_t j = lo; j < hi; ++j) {
+      if (!batch_desc_ok(descs + ids[j])) {
+        part->bad = ids[j] < part->bad ? ids[j] : part->bad;
+        continue;
+      }
       bfk::BatchRecord& r = recs[j];
       std::memset(&r, 0, sizeof r);
       bfk::Plan base;
@@ -314,17 +339,27 @@ void build_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t 
     *wmax = p.wmax > *wmax ? p.wmax : *wmax;
     *pmax = p.pmax > *pmax ? p.pmax : *pmax;
     *any_inner |= p.inner;
+    *bad = p.bad < *bad ? p.bad : *bad;
   }
 }
 
-// Lane-tree records of descs[ids[j]], j < count.
+// Lane-tree records of descs[ids[j]], j < count; *bad as for build_records.
 void build_lanetree_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count,
-                            bfk::LaneTreeRecord* recs) {
-  struct Part {};
+                            bfk::LaneTreeRecord* recs, uint32_t* bad) {
+  struct Part {
+    uint32_t bad = 0xFFFFFFFFu;
+  };
   std::vector<Part> parts;
-  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part*) {
-    for (uint32_t j = lo; j < hi; ++j) lanetree_record(descs + ids[j], recs + j);
+  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part* part) {
+    for (uint32_t j = lo; j < hi; ++j) {
+      if (!batch_desc_ok(descs + ids[j])) {
+        part->bad = ids[j] < part->bad ? ids[j] : part->bad;
+        continue;
+      }
+      lanetree_record(descs + ids[j], recs + j);
+    }
   });
+  for (const Part& p : parts) *bad = p.bad < *bad ? p.bad : *bad;
 }
 
 // Where a batch's scenarios go: up to kLtBatchTools tools the lane-tree
@@ -737,20 +772,23 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
 static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
   if (count == 0) return BF_OK;
   if (!descs || !out) return fail(BF_EINVAL, "bf_search_batch: NULL argument");
-  for (uint32_t i = 0; i < count; ++i) {
-    int rc = validate(descs + i, "bf_search_batch");
-    if (rc == BF_OK) rc = require_enum(descs[i], "bf_search_batch");
-    if (rc != BF_OK) return fail(rc, "bf_search_batch: descs[%u]: %s", i, g_error.c_str());
-  }
+  // The descs are checked while their records are built (on the host pool);
+  // the lowest failing position is reported, as a check in order would.
   std::vector<uint32_t> small(count), large(count);
   const BatchSplit b = split_batch(descs, count, small, large);
   std::vector<bfk::LaneTreeRecord> lt(b.ns);
   std::vector<uint32_t> first_block(b.ns + 1, 0u);
   std::vector<bfk::BatchRecord> bk(b.nl);
-  build_lanetree_records(descs, small.data(), b.ns, lt.data());
-  for (uint32_t j = 0; j < b.ns; ++j) first_block[j + 1] = first_block[j] + lt[j].nblocks;
+  uint32_t bad = 0xFFFFFFFFu;
+  build_lanetree_records(descs, small.data(), b.ns, lt.data(), &bad);
   uint32_t wmax = 0, pmax = 0, any_inner = 0;
-  build_records(descs, large.data(), b.nl, bk.data(), &wmax, &pmax, &any_inner);
+  build_records(descs, large.data(), b.nl, bk.data(), &wmax, &pmax, &any_inner, &bad);
+  if (bad != 0xFFFFFFFFu) {
+    int rc = validate(descs + bad, "bf_search_batch");
+    if (rc == BF_OK) rc = require_enum(descs[bad], "bf_search_batch");
+    return fail(rc == BF_OK ? BF_EINVAL : rc, "bf_search_batch: descs[%u]: %s", bad, g_error.c_str());
+  }
+  for (uint32_t j = 0; j < b.ns; ++j) first_block[j + 1] = first_block[j] + lt[j].nblocks;
 
   // One device allocation: lane-tree records, their first blocks, batch
   // records, keys.
@@ -760,7 +798,7 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   unsigned char* d_base = nullptr;
   std::vector<unsigned long long> keys(count);
-  cudaError_t e = lib_malloc(reinterpret_cast<void**>(&d_base), off_keys + kbytes);
+  cudaError_t e = lib_malloc_async(reinterpret_cast<void**>(&d_base), off_keys + kbytes, st);
   auto* d_lt = reinterpret_cast<bfk::LaneTreeRecord*>(d_base);
   auto* d_fb = reinterpret_cast<uint32_t*>(d_base + off_fb);
   auto* d_bk = reinterpret_cast<bfk::BatchRecord*>(d_base + off_bk);
@@ -775,13 +813,16 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
   if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
   // Bounded wait first: a copy into pageable memory would block without limit.
   if (rc == BF_OK) rc = wait_stream(st, "bf_search_batch");
+  if (rc == BF_OK) e = cudaMemcpyAsync(keys.data(), d_keys, kbytes, cudaMemcpyDeviceToHost, st);
+  // Ordered after the kernels and the copy, also when the wait timed out.
+  if (d_base) {
+    const cudaError_t ef = cudaFreeAsync(d_base, st);
+    if (e == cudaSuccess) e = ef;
+  }
   if (rc == BF_OK) {
-    e = cudaMemcpyAsync(keys.data(), d_keys, kbytes, cudaMemcpyDeviceToHost, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
   }
-  // On timeout the kernels may still use the scratch: leak it rather than free in-use memory.
-  if (rc != BF_ETIMEOUT && d_base) cudaFree(d_base);
   if (rc != BF_OK) return rc;
   for (uint32_t j = 0; j < b.ns; ++j) fill_result(keys[j], descs[small[j]].n, 0, out + small[j]);
   for (uint32_t j = 0; j < b.nl; ++j) fill_result(keys[b.ns + j], descs[large[j]].n, 0, out + large[j]);

@@ -467,6 +467,24 @@ def test_wait_timeout_is_reported():
     assert r.feasible
 
 
+def test_batch_wait_timeout_then_next_call(golden):
+    """A batch call whose host wait runs out returns BF_ETIMEOUT; its scratch is freed in stream order
+    after its kernels, and the next call on the same stream gives the oracle's optima."""
+    import torch
+    batch = S.config4(1024)
+    want = list(zip(golden["4"]["best_index"][:1024], golden["4"]["best_makespan"][:1024]))
+    bf.set_wait_timeout_ms(1)
+    try:
+        with pytest.raises(bf.BfError) as ei:
+            bf.search_batch(batch)
+        assert ei.value.code == bf.BF_ETIMEOUT
+    finally:
+        bf.set_wait_timeout_ms(600000)
+    got = [(r.index, r.makespan_us) for r in bf.search_batch(batch)]
+    torch.cuda.synchronize()
+    assert got == want
+
+
 def test_shards_combine_to_full_search(golden):
     """The per-rank pieces of a sharded search (shard.gpu_search_range on each
     rank's range), combined by packed key, give the full N=19 optimum."""
