@@ -171,7 +171,10 @@ BF_API int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t coun
  * before any GPU work; the first invalid one (lowest position) fails the call with BF_EINVAL naming
  * its position.  Allocates its device scratch (packed tables + one key per scenario) from the
  * device's default stream-ordered memory pool on cuda_stream and frees it there after its kernels,
- * also when the wait times out (BF_ETIMEOUT).  Blocks until the results are on the host. */
+ * also when the wait times out (BF_ETIMEOUT).  A large batch launches part of its work on a stream
+ * the call creates and destroys; that work starts after the work already enqueued on cuda_stream,
+ * and work enqueued on cuda_stream after the call starts after it.  Blocks until the results are
+ * on the host. */
 BF_API int bf_search_batch(const bf_scenario_desc* descs, uint32_t count, bf_result* out,
                     void* cuda_stream);
 

@@ -277,11 +277,12 @@ class HostPool {
   uint32_t workers_ = 0, finished_ = 0;
 };
 
-// Run work(lo, hi, &parts[t]) over [0, count) in up to 16 parts (one per few
-// hundred scenarios) on the host pool; parts gets one entry per part.
+// Run work(lo, hi, &parts[t]) over [0, count) in up to 16 parts (one per 32
+// scenarios or more: a record takes about 2 us on the Arm host, a dispatch to
+// the pool some tens of us) on the host pool; parts gets one entry per part.
 template <typename Part, typename Work>
 void parallel_parts(uint32_t count, std::vector<Part>& parts, Work work) {
-  uint32_t nparts = count / 256u;
+  uint32_t nparts = count / 32u;
   if (nparts > 16u) nparts = 16u;
   parts.assign(nparts > 1 ? nparts : 1, Part{});
   if (nparts > 1) {
@@ -295,34 +296,41 @@ void parallel_parts(uint32_t count, std::vector<Part>& parts, Work work) {
   work(0u, count, &parts[0]);
 }
 
-// Whether a desc can be searched by a batch (valid, n <= BF_MAX_TOOLS_ENUM);
-// the record builders check each desc before they read it, on the host pool,
-// and the caller reports the lowest failing position.  A failed check on a
-// pool thread writes that thread's error text only.
-bool batch_desc_ok(const bf_scenario_desc* d) {
-  try {  // a failed check formats its message, which may allocate; no exception leaves a pool thread
-    return validate(d, "bf_search_batch") == BF_OK && require_enum(*d, "bf_search_batch") == BF_OK;
-  } catch (...) {
-    return false;
-  }
+// The lowest position in descs[0, count) whose desc a batch cannot search
+// (invalid, or n > BF_MAX_TOOLS_ENUM), checked on the host pool; 0xFFFFFFFF
+// if none.  A failed check on a pool thread writes that thread's error text
+// only: the caller checks that desc again to report it.
+uint32_t first_invalid(const bf_scenario_desc* descs, uint32_t count) {
+  struct Part {
+    uint32_t bad = 0xFFFFFFFFu;
+  };
+  std::vector<Part> parts;
+  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part* part) {
+    for (uint32_t i = lo; i < hi && part->bad == 0xFFFFFFFFu; ++i) {
+      bool ok = false;
+      try {  // a failed check formats its message, which may allocate; no exception leaves a pool thread
+        ok = validate(descs + i, "bf_search_batch") == BF_OK && require_enum(descs[i], "bf_search_batch") == BF_OK;
+      } catch (...) {
+      }
+      if (!ok) part->bad = i;
+    }
+  });
+  uint32_t bad = 0xFFFFFFFFu;
+  for (const Part& p : parts) bad = p.bad < bad ? p.bad : bad;
+  return bad;
 }
 
 // Batch-kernel records (tables, window tables, plan) of descs[ids[j]], j <
 // count; the largest window, task count and whether any plan has an inner
-// level are returned too, and *bad lowered to the lowest position whose desc
-// fails batch_desc_ok (its record is left unbuilt).
+// level are returned too.
 void build_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count, bfk::BatchRecord* recs,
-                   uint32_t* wmax, uint32_t* pmax, uint32_t* any_inner, uint32_t* bad) {
+                   uint32_t* wmax, uint32_t* pmax, uint32_t* any_inner) {
   struct Part {
-    uint32_t wmax = 0, pmax = 0, inner = 0, bad = 0xFFFFFFFFu;
+    uint32_t wmax = 0, pmax = 0, inner = 0;
   };
   std::vector<Part> parts;
   parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part* part) {
     for (uint32_t j = lo; j < hi; ++j) {
-      if (!batch_desc_ok(descs + ids[j])) {
-        part->bad = ids[j] < part->bad ? ids[j] : part->bad;
-        continue;
-      }
       bfk::BatchRecord& r = recs[j];
       std::memset(&r, 0, sizeof r);
       bfk::Plan base;
@@ -339,27 +347,17 @@ void build_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t 
     *wmax = p.wmax > *wmax ? p.wmax : *wmax;
     *pmax = p.pmax > *pmax ? p.pmax : *pmax;
     *any_inner |= p.inner;
-    *bad = p.bad < *bad ? p.bad : *bad;
   }
 }
 
-// Lane-tree records of descs[ids[j]], j < count; *bad as for build_records.
+// Lane-tree records of descs[ids[j]], j < count.
 void build_lanetree_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count,
-                            bfk::LaneTreeRecord* recs, uint32_t* bad) {
-  struct Part {
-    uint32_t bad = 0xFFFFFFFFu;
-  };
+                            bfk::LaneTreeRecord* recs) {
+  struct Part {};
   std::vector<Part> parts;
-  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part* part) {
-    for (uint32_t j = lo; j < hi; ++j) {
-      if (!batch_desc_ok(descs + ids[j])) {
-        part->bad = ids[j] < part->bad ? ids[j] : part->bad;
-        continue;
-      }
-      lanetree_record(descs + ids[j], recs + j);
-    }
+  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part*) {
+    for (uint32_t j = lo; j < hi; ++j) lanetree_record(descs + ids[j], recs + j);
   });
-  for (const Part& p : parts) *bad = p.bad < *bad ? p.bad : *bad;
 }
 
 // Where a batch's scenarios go: up to kLtBatchTools tools the lane-tree
@@ -769,46 +767,104 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   return BF_OK;
 }
 
+// Batches of at least this many lane-tree scenarios are pipelined: the first
+// eighth is built, copied and launched on the caller's stream, and the rest
+// is built while that kernel runs and launched on a second stream (created
+// for the call) that waits only for the key reset, so that the two kernels
+// overlap; the caller's stream waits for the second before the keys come
+// back.  4096 x 3^10: the kernel otherwise waits about 0.5 ms for the
+// records.
+constexpr uint32_t kBatchPipelineMin = 1024;
+
 static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
   if (count == 0) return BF_OK;
   if (!descs || !out) return fail(BF_EINVAL, "bf_search_batch: NULL argument");
-  // The descs are checked while their records are built (on the host pool);
-  // the lowest failing position is reported, as a check in order would.
-  std::vector<uint32_t> small(count), large(count);
-  const BatchSplit b = split_batch(descs, count, small, large);
-  std::vector<bfk::LaneTreeRecord> lt(b.ns);
-  std::vector<uint32_t> first_block(b.ns + 1, 0u);
-  std::vector<bfk::BatchRecord> bk(b.nl);
-  uint32_t bad = 0xFFFFFFFFu;
-  build_lanetree_records(descs, small.data(), b.ns, lt.data(), &bad);
-  uint32_t wmax = 0, pmax = 0, any_inner = 0;
-  build_records(descs, large.data(), b.nl, bk.data(), &wmax, &pmax, &any_inner, &bad);
+  const uint32_t bad = first_invalid(descs, count);
   if (bad != 0xFFFFFFFFu) {
     int rc = validate(descs + bad, "bf_search_batch");
     if (rc == BF_OK) rc = require_enum(descs[bad], "bf_search_batch");
     return fail(rc == BF_OK ? BF_EINVAL : rc, "bf_search_batch: descs[%u]: %s", bad, g_error.c_str());
   }
-  for (uint32_t j = 0; j < b.ns; ++j) first_block[j + 1] = first_block[j] + lt[j].nblocks;
+  std::vector<uint32_t> small(count), large(count);
+  const BatchSplit b = split_batch(descs, count, small, large);
+  const bool pipe = b.ns >= kBatchPipelineMin;
+  const uint32_t k1 = pipe ? b.ns / 8u : b.ns;  // lane-tree scenarios of the first launch
+  // Record buffers of the calling thread, grown as needed and reused: a
+  // fresh 2.8 MB array (4096 scenarios) cost about 0.4 ms of zeroing and page
+  // faults per call.  Every record is written whole before it is copied; a
+  // copy from pageable memory has read it by the time cudaMemcpyAsync
+  // returns, so the next call may reuse the buffers even after a timeout.
+  thread_local std::vector<bfk::LaneTreeRecord> lt;
+  thread_local std::vector<bfk::BatchRecord> bk;
+  if (lt.size() < b.ns) lt.resize(b.ns);
+  if (bk.size() < b.nl) bk.resize(b.nl);
+  std::vector<uint32_t> fb1(k1 + 1, 0u), fb2(b.ns - k1 + 1, 0u);  // first blocks of each launch
+  build_lanetree_records(descs, small.data(), k1, lt.data());
+  for (uint32_t j = 0; j < k1; ++j) fb1[j + 1] = fb1[j] + lt[j].nblocks;
 
-  // One device allocation: lane-tree records, their first blocks, batch
-  // records, keys.
-  const size_t lt_bytes = sizeof(bfk::LaneTreeRecord) * b.ns, fb_bytes = sizeof(uint32_t) * (b.ns + 1);
-  const size_t bk_bytes = sizeof(bfk::BatchRecord) * b.nl, kbytes = sizeof(unsigned long long) * count;
-  const size_t off_fb = align256(lt_bytes), off_bk = off_fb + align256(fb_bytes), off_keys = off_bk + align256(bk_bytes);
+  // One device allocation: lane-tree records, the two first-block arrays,
+  // batch records, keys.
+  const size_t lt_bytes = sizeof(bfk::LaneTreeRecord) * b.ns, kbytes = sizeof(unsigned long long) * count;
+  const size_t fb1_bytes = sizeof(uint32_t) * fb1.size(), fb2_bytes = sizeof(uint32_t) * fb2.size();
+  const size_t bk_bytes = sizeof(bfk::BatchRecord) * b.nl;
+  const size_t off_fb1 = align256(lt_bytes), off_fb2 = off_fb1 + align256(fb1_bytes);
+  const size_t off_bk = off_fb2 + align256(fb2_bytes), off_keys = off_bk + align256(bk_bytes);
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
+  cudaStream_t rest = st;  // stream of the later launches
+  cudaEvent_t reset_done = nullptr, rest_done = nullptr;
   unsigned char* d_base = nullptr;
   std::vector<unsigned long long> keys(count);
   cudaError_t e = lib_malloc_async(reinterpret_cast<void**>(&d_base), off_keys + kbytes, st);
   auto* d_lt = reinterpret_cast<bfk::LaneTreeRecord*>(d_base);
-  auto* d_fb = reinterpret_cast<uint32_t*>(d_base + off_fb);
+  auto* d_fb1 = reinterpret_cast<uint32_t*>(d_base + off_fb1);
+  auto* d_fb2 = reinterpret_cast<uint32_t*>(d_base + off_fb2);
   auto* d_bk = reinterpret_cast<bfk::BatchRecord*>(d_base + off_bk);
   auto* d_keys = reinterpret_cast<unsigned long long*>(d_base + off_keys);
-  if (e == cudaSuccess && b.ns) e = cudaMemcpyAsync(d_lt, lt.data(), lt_bytes, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess && b.ns) e = cudaMemcpyAsync(d_fb, first_block.data(), fb_bytes, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess && b.nl) e = cudaMemcpyAsync(d_bk, bk.data(), bk_bytes, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && pipe) {
+    e = cudaStreamCreateWithFlags(&rest, cudaStreamNonBlocking);
+    if (e != cudaSuccess) rest = st;
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&reset_done, cudaEventDisableTiming);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&rest_done, cudaEventDisableTiming);
+  }
+  if (e == cudaSuccess && k1) e = cudaMemcpyAsync(d_lt, lt.data(), sizeof(bfk::LaneTreeRecord) * k1, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && k1) e = cudaMemcpyAsync(d_fb1, fb1.data(), fb1_bytes, cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, kbytes, st);
-  if (e == cudaSuccess)
-    e = launch_batch_groups(b, d_lt, d_fb, first_block[b.ns], d_bk, wmax, pmax, any_inner, d_keys, st);
+  if (e == cudaSuccess && rest != st) e = cudaEventRecord(reset_done, st);
+  if (e == cudaSuccess && k1) e = bfk::launch_lanetree(d_lt, d_fb1, k1, fb1[k1], b.nmax_small, d_keys, st);
+  bool rest_used = false;  // work enqueued on `rest` that the caller's stream must wait for
+  if (e == cudaSuccess) {
+    // The rest of the records, built while the first launch runs.
+    build_lanetree_records(descs, small.data() + k1, b.ns - k1, lt.data() + k1);
+    for (uint32_t j = k1; j < b.ns; ++j) fb2[j - k1 + 1] = fb2[j - k1] + lt[j].nblocks;
+    uint32_t wmax = 0, pmax = 0, any_inner = 0;
+    build_records(descs, large.data(), b.nl, bk.data(), &wmax, &pmax, &any_inner);
+    if (rest != st) {
+      e = cudaStreamWaitEvent(rest, reset_done, 0);
+      rest_used = e == cudaSuccess;
+    }
+    const uint32_t k2 = b.ns - k1;
+    if (e == cudaSuccess && k2)
+      e = cudaMemcpyAsync(d_lt + k1, lt.data() + k1, sizeof(bfk::LaneTreeRecord) * k2, cudaMemcpyHostToDevice, rest);
+    if (e == cudaSuccess && k2) e = cudaMemcpyAsync(d_fb2, fb2.data(), fb2_bytes, cudaMemcpyHostToDevice, rest);
+    if (e == cudaSuccess && b.nl) e = cudaMemcpyAsync(d_bk, bk.data(), bk_bytes, cudaMemcpyHostToDevice, rest);
+    if (e == cudaSuccess && k2) e = bfk::launch_lanetree(d_lt + k1, d_fb2, k2, fb2[k2], b.nmax_small, d_keys + k1, rest);
+    if (e == cudaSuccess && b.nl) {
+      BatchSplit bl = b;
+      bl.ns = 0;  // the batch-kernel group alone, its keys after the lane-tree group's
+      e = launch_batch_groups(bl, nullptr, nullptr, 0, d_bk, wmax, pmax, any_inner, d_keys + b.ns, rest);
+    }
+  }
+  // The caller's stream waits for the later launches (also after an error,
+  // before the scratch is freed there); if that cannot be enqueued, the host
+  // waits for them.
+  if (rest_used) {
+    cudaError_t ew = cudaEventRecord(rest_done, rest);
+    if (ew == cudaSuccess) ew = cudaStreamWaitEvent(st, rest_done, 0);
+    if (ew != cudaSuccess) {
+      cudaStreamSynchronize(rest);
+      if (e == cudaSuccess) e = ew;
+    }
+  }
   int rc = BF_OK;
   if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
   // Bounded wait first: a copy into pageable memory would block without limit.
@@ -823,6 +879,11 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) rc = cuda_fail(e, "bf_search_batch");
   }
+  // Released once their work is done (destroying a stream or an event with
+  // work pending does not wait).
+  if (rest != st) cudaStreamDestroy(rest);
+  if (reset_done) cudaEventDestroy(reset_done);
+  if (rest_done) cudaEventDestroy(rest_done);
   if (rc != BF_OK) return rc;
   for (uint32_t j = 0; j < b.ns; ++j) fill_result(keys[j], descs[small[j]].n, 0, out + small[j]);
   for (uint32_t j = 0; j < b.nl; ++j) fill_result(keys[b.ns + j], descs[large[j]].n, 0, out + large[j]);

@@ -467,6 +467,29 @@ def test_wait_timeout_is_reported():
     assert r.feasible
 
 
+def test_pipelined_batch_with_both_groups(golden):
+    """A batch large enough to be pipelined (its first eighth of lane-tree scenarios launched while the
+    rest are built, the rest on a second stream), with 30 random scenarios of 1-14 tools interleaved
+    (those of 13 and 14 tools run the batch kernel, also on the second stream): every result at its
+    position against the oracle."""
+    small = S.config4(1200)
+    extra = mixed_group_batch(seed=99, count=30)
+    scns, origin = [], []  # origin: index into small, or -1 for an interleaved scenario
+    for i, scn in enumerate(small):
+        scns.append(scn)
+        origin.append(i)
+        if i % 40 == 0:
+            scns.append(extra[i // 40])
+            origin.append(-1)
+    assert sum(s.n <= 12 for s in scns) >= 1024 and any(s.n > 12 for s in scns)
+    o_i, o_m = oracle.search_batch(extra, THREADS)
+    want_extra = iter(zip(o_i.tolist(), o_m.tolist()))
+    res = bf.search_batch(scns)
+    for pos, (k, r) in enumerate(zip(origin, res)):
+        want = (golden["4"]["best_index"][k], golden["4"]["best_makespan"][k]) if k >= 0 else next(want_extra)
+        assert (r.index, r.makespan_us) == want, pos
+
+
 def test_batch_wait_timeout_then_next_call(golden):
     """A batch call whose host wait runs out returns BF_ETIMEOUT; its scratch is freed in stream order
     after its kernels, and the next call on the same stream gives the oracle's optima."""
