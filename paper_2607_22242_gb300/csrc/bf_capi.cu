@@ -478,8 +478,11 @@ int bf_create_scenario(const bf_scenario_desc* desc, bf_scenario** out) {
   cudaError_t e = cudaGetDevice(&s->device);
   bfk::LaneTreeRecord ltrec;
   if (e == cudaSuccess && desc->n >= bfk::kLtSingleMinTools && desc->n <= bfk::kLtMaxTools) {
-    e = bfk::lanetree_single_blocks(desc->n, &s->lt_blocks);
-    if (e == cudaSuccess) {
+    // Optional: if the lane-tree kernel's launch shape cannot be had, the
+    // search kernel runs every search of this handle.
+    if (bfk::lanetree_single_blocks(desc->n, &s->lt_blocks) != cudaSuccess) {
+      cudaGetLastError();
+    } else {
       double lt_events = 0.0;
       bfk::host::lanetree_record(desc, &ltrec,
                                  (uint64_t)s->lt_blocks * bfk::kLtLaunchThreads * bfk::kLtSingleRootsPerLane,
