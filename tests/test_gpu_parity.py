@@ -219,6 +219,21 @@ def test_lanetree_whole_space_search():
         assert r.modes == S.mapping_modes(r.index, n)
 
 
+def test_lanetree_full_queue_of_16():
+    """Sixteen tools without edges (every tool is ready at time 0) with small integer times: the
+    mapping that queues all of them fills the lane tree's 16-entry queue word, and ties between
+    tools ready at the same instant go by index.  Full searches against the oracle, with a loose
+    and a tight VRAM budget."""
+    rng = np.random.default_rng(16)
+    for tight in (False, True):
+        base = S.random_small(rng, 16, edge_p=0.0, tight=tight, contention=True, max_time=9)
+        assert all(p == 0 for p in base.pred_mask)
+        want = oracle.search(base, THREADS)
+        with bf.create_scenario(base) as h:
+            r = bf.search_best(h)
+        assert (r.index, r.makespan_us) == want, tight
+
+
 def test_degenerate_budgets_all_paths():
     """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
     the batch, the branch and bound and the tree search, against the oracle."""
