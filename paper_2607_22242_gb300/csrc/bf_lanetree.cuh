@@ -24,9 +24,9 @@
 // GB300 form.  Divergence, not arithmetic, bounds the batch: random layered
 // DAGs start most tools at once and lanes with different modes follow
 // different event sequences.  So
-//   * a lane's per-tool values live in shared memory (one word per tool: the
-//     end time of a running CPU tool, the end stamp of a running GPU tool on
-//     the virtual clock, the ready time of a waiting queued tool), and each
+//   * a lane's per-tool values live in shared memory (one word per tool,
+//     written when the tool starts: the end time of a CPU tool, the end stamp
+//     of a GPU tool on the virtual clock), and each
 //     event touches only the tools it admits, retires or scans for the next
 //     completion (bit loops over small sets) instead of every slot;
 //   * the VRAM in use is a table lookup on the set of running GPU tools, the
@@ -40,7 +40,9 @@
 //     next CPU end and GPU end stamp;
 //   * a lane moves to its next job (a level combination or a new root) the
 //     moment its current one ends, instead of waiting for the warp's slowest
-//     lane; roots come from a per-block counter in shared memory;
+//     lane; roots come from a per-block counter in shared memory (in the
+//     one-scenario search, once the block's share is gone, from a counter in
+//     device memory);
 //   * a checkpoint is nine state words: the per-tool words of the tools
 //     running at it are never written again while it can still be resumed.
 // Arithmetic is that of bf_sim.cuh: u32 real time, virtual clock modulo 2^32,
