@@ -15,7 +15,9 @@ constexpr int kLtThreads = (int)kLtLaunchThreads;
 // compiler picks unbounded, same occupancy: batch call 12.86 -> 12.70 ms,
 // 16-tool full search 1.60 -> 1.58 ms.
 constexpr int kLtBlocksPerSm = 5;
-constexpr uint32_t kLtSingleChunks = 3;  // tables of the one-scenario search: up to 18 tools
+// The wide one-scenario kernel (17 to 20 tools) holds 11 state words per
+// checkpoint and 20 per-tool words per lane: 4 blocks fit an SM.
+constexpr int kLtWideBlocksPerSm = 4;
 
 __device__ __forceinline__ unsigned long long lt_warp_min(unsigned long long v) {
 #pragma unroll
@@ -78,11 +80,14 @@ __global__ void __launch_bounds__(kLtThreads, kLtBlocksPerSm) lanetree_kernel(co
 // until the last roots.  The lowest key goes to sync->key; the last block to
 // finish copies it to *host_key (pinned host memory the device addresses)
 // and puts sync back to (~0, 0, 0).
-__global__ void __launch_bounds__(kLtThreads, kLtBlocksPerSm) lanetree_single_kernel(const LaneTreeRecord* __restrict__ rec,
-                                                                    uint32_t static_roots, SearchSync* sync,
-                                                                    unsigned long long* host_key) {
+// NC table chunks, W the wide queue form: <3, false> up to 16 tools, <4,
+// true> up to 20.
+template <uint32_t NC, bool W>
+__global__ void __launch_bounds__(kLtThreads, W ? kLtWideBlocksPerSm : kLtBlocksPerSm)
+    lanetree_single_kernel(const LaneTreeRecord* __restrict__ rec, uint32_t static_roots, SearchSync* sync,
+                           unsigned long long* host_key) {
   extern __shared__ uint32_t lt_rows_smem[];
-  __shared__ LtSharedT<kLtSingleChunks> S;
+  __shared__ LtSharedT<NC> S;
   lt_load_record(S, rec);
   if (threadIdx.x == 0) {
     const uint64_t j = blockIdx.x, nb = gridDim.x;
@@ -93,8 +98,8 @@ __global__ void __launch_bounds__(kLtThreads, kLtBlocksPerSm) lanetree_single_ke
   uint32_t roots = 1u;
   for (uint32_t t = 0; t < S.rec.x; ++t) roots *= 3u;
   MinKeySink sink;
-  LtSharedT<kLtSingleChunks>& Sref = S;
-  lt_lane(S, lt_rows_smem + threadIdx.x, blockDim.x,
+  LtSharedT<NC>& Sref = S;
+  lt_lane<NC, W>(S, lt_rows_smem + threadIdx.x, blockDim.x,
           [&Sref, sync, static_roots, roots]() {
             const uint32_t r = atomicAdd(&Sref.root_next, 1u);
             if (r < Sref.root_end) return r;
@@ -121,7 +126,23 @@ __global__ void __launch_bounds__(kLtThreads, kLtBlocksPerSm) lanetree_single_ke
   }
 }
 
-size_t lt_smem_bytes(uint32_t n) { return sizeof(uint32_t) * lt_rows(n) * kLtThreads; }
+template <bool W = false>
+size_t lt_smem_bytes(uint32_t n) { return sizeof(uint32_t) * lt_rows<W>(n) * kLtThreads; }
+
+// The one-scenario kernel for n tools, with its dynamic shared memory allowed
+// (once per device and form).
+using SingleKernel = void (*)(const LaneTreeRecord*, uint32_t, SearchSync*, unsigned long long*);
+cudaError_t single_kernel_for(uint32_t n, SingleKernel* k, size_t* smem) {
+  static std::atomic<uint64_t> ready_narrow{0}, ready_wide{0};
+  if (n <= kLtNarrowTools) {
+    *k = lanetree_single_kernel<3, false>;
+    *smem = lt_smem_bytes<false>(n);
+    return allow_dyn_smem(lanetree_single_kernel<3, false>, lt_smem_bytes<false>(kLtNarrowTools), &ready_narrow);
+  }
+  *k = lanetree_single_kernel<4, true>;
+  *smem = lt_smem_bytes<true>(n);
+  return allow_dyn_smem(lanetree_single_kernel<4, true>, lt_smem_bytes<true>(kLtMaxTools), &ready_wide);
+}
 
 }  // namespace
 
@@ -135,13 +156,13 @@ cudaError_t launch_lanetree(const LaneTreeRecord* d_recs, const uint32_t* d_firs
 }
 
 cudaError_t lanetree_single_blocks(uint32_t n, uint32_t* blocks) {
-  static std::atomic<uint64_t> ready{0};
-  cudaError_t e = allow_dyn_smem(lanetree_single_kernel, lt_smem_bytes(kLtMaxTools), &ready);
+  SingleKernel k = nullptr;
+  size_t smem = 0;
+  cudaError_t e = single_kernel_for(n, &k, &smem);
   int dev = 0, sms = 0, per_sm = 0;
   if (e == cudaSuccess) e = cudaGetDevice(&dev);
   if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (e == cudaSuccess)
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, lanetree_single_kernel, kLtThreads, lt_smem_bytes(n));
+  if (e == cudaSuccess) e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, k, kLtThreads, smem);
   if (e != cudaSuccess) return e;
   *blocks = (uint32_t)(sms > 0 ? sms : 1) * (uint32_t)(per_sm > 0 ? per_sm : 1);
   return cudaSuccess;
@@ -149,13 +170,14 @@ cudaError_t lanetree_single_blocks(uint32_t n, uint32_t* blocks) {
 
 cudaError_t launch_lanetree_single(const LaneTreeRecord* d_rec, uint32_t n, uint32_t x, uint32_t blocks,
                                    SearchSync* sync, unsigned long long* host_key, cudaStream_t st) {
-  static std::atomic<uint64_t> ready{0};
-  cudaError_t e = allow_dyn_smem(lanetree_single_kernel, lt_smem_bytes(kLtMaxTools), &ready);
+  SingleKernel k = nullptr;
+  size_t smem = 0;
+  cudaError_t e = single_kernel_for(n, &k, &smem);
   if (e != cudaSuccess) return e;
   uint64_t roots = 1;
   for (uint32_t t = 0; t < x; ++t) roots *= 3u;
   const uint32_t static_roots = (uint32_t)(roots * kLtStaticShareNum / kLtStaticShareDen);
-  lanetree_single_kernel<<<blocks, kLtThreads, lt_smem_bytes(n), st>>>(d_rec, static_roots, sync, host_key);
+  k<<<blocks, kLtThreads, smem, st>>>(d_rec, static_roots, sync, host_key);
   return cudaGetLastError();
 }
 

@@ -1,4 +1,4 @@
-// bf_lanetree.cuh -- the full search of a scenario of up to 16 tools as a
+// bf_lanetree.cuh -- the full search of a scenario of up to 20 tools as a
 // tree of checkpoints walked by each lane: many small scenarios in one launch
 // (the batch), or one scenario over the whole GPU.
 //
@@ -31,8 +31,9 @@
 //     completion (bit loops over small sets) instead of every slot;
 //   * the VRAM in use is a table lookup on the set of running GPU tools, the
 //     ready set a lookup on the done set (one lookup per 6-bit chunk of the
-//     tools: two up to 12 tools, three up to 16);
-//   * the queue is a FIFO list of 4-bit tool numbers in one 64-bit word:
+//     tools: two up to 12 tools, three up to 16, four up to 20);
+//   * the queue is a FIFO list of tool numbers -- 4-bit in one 64-bit word up
+//     to 16 tools, 5-bit in two words above (the "wide" form):
 //     tools join it in the order they become ready (in index order within
 //     an instant), which is the model's (ready time, index) order, so its
 //     head is the list's first entry;
@@ -43,8 +44,9 @@
 //     lane; roots come from a per-block counter in shared memory (in the
 //     one-scenario search, once the block's share is gone, from a counter in
 //     device memory);
-//   * a checkpoint is nine state words: the per-tool words of the tools
-//     running at it are never written again while it can still be resumed.
+//   * a checkpoint is nine state words (eleven in the wide form): the
+//     per-tool words of the tools running at it are never written again
+//     while it can still be resumed.
 // Arithmetic is that of bf_sim.cuh: u32 real time, virtual clock modulo 2^32,
 // GPU completion ceil(rem * f[k] / 2^20), the CPU-event advance
 // floor(dt * 2^20 / f[k]) by the per-k reciprocal of Granlund and Montgomery
@@ -58,7 +60,8 @@
 namespace bfk {
 
 constexpr uint32_t kLtBatchTools = 12;  // the batch sends scenarios of up to this many tools here
-constexpr uint32_t kLtMaxTools = 16;    // record capacity (and the queue's 4-bit tool numbers)
+constexpr uint32_t kLtMaxTools = 20;    // record capacity
+constexpr uint32_t kLtNarrowTools = 16; // up to this many tools the queue's numbers fit 4 bits
 constexpr uint32_t kLtChunkBits = 6;    // readiness and VRAM tables: 6-bit chunks of the tools
 constexpr uint32_t kLtChunk = 1u << kLtChunkBits;
 constexpr uint32_t kLtPartTools = 4;    // tools per table-driven part of the mode combinations
@@ -66,6 +69,11 @@ constexpr uint32_t kLtPartCombos = 81;  // 3^kLtPartTools
 constexpr uint32_t kLtRootParts = 4;    // root tools [0,4), [4,8), [8,12), [12,x)
 constexpr uint32_t kLtParts = kLtRootParts + 2;  // the root's parts, level [x,y), level [y,n)
 constexpr uint32_t kLtStateWords = 9;   // pend, run, qset, qlist (2 words), T, V, tc, gm
+constexpr uint32_t kLtWideStateWords = 11;  // and the wide queue's second word (2 words)
+
+// State words of a checkpoint in the narrow (W = false) or wide form.
+template <bool W>
+__host__ __device__ constexpr uint32_t lt_state_words() { return W ? kLtWideStateWords : kLtStateWords; }
 
 // 6-bit chunks the tables of an n-tool scenario need.
 __host__ __device__ constexpr uint32_t lt_chunks(uint32_t n) { return (n + kLtChunkBits - 1u) / kLtChunkBits; }
@@ -98,7 +106,7 @@ struct LtSharedT {
   uint32_t cnow[kLtParts][kLtPartCombos];
   uint32_t cque[kLtParts][kLtPartCombos];
   uint32_t cidx[kLtParts][kLtPartCombos];
-  uint32_t ck0[kLtStateWords];   // the state words at time 0 (a root's checkpoint)
+  uint32_t ck0[kLtWideStateWords];  // the state words at time 0 (a root's checkpoint)
   uint32_t root_next, root_end;  // this block's roots still to take: [root_next, root_end)
 };
 using LtShared = LtSharedT<2>;  // the batch: up to kLtBatchTools tools
@@ -108,20 +116,22 @@ using LtShared = LtSharedT<2>;  // the batch: up to kLtBatchTools tools
 // done = ~(pend | run | qset) (the slots beyond n count as done).
 struct LtState {
   uint32_t pend, run, qset;
-  uint64_t qlist;  // waiting queued tools by index, head in bits 0-3; qset says how many
+  uint64_t qlist;  // waiting queued tools by index, head in bits 0-3 (0-4 wide); qset says how many
+  uint64_t qhi;    // wide form: entries 12 and up, 5 bits each
   uint32_t T, V;   // real time (us); virtual GPU clock (1/1024 us of isolated work, modulo 2^32)
   uint32_t tc;     // earliest end of a running CPU tool (0xFFFFFFFF if none)
   uint32_t gm;     // end stamp of the running GPU tool that ends first (when one runs)
 };
 
 // Rows of one lane ([row][thread], `stride` threads): the per-tool words
-// [0, n), then the state words of checkpoint 1 [n, n + 9) and of checkpoint
-// 2 [n + 9, n + 18).  One set of per-tool words serves every level: a tool's
+// [0, n), then the state words of checkpoint 1 [n, n + w) and of checkpoint
+// 2 [n + w, n + 2w), w = lt_state_words<W>().  One set of per-tool words serves every level: a tool's
 // word is written once per simulation, when it starts, and only read after
 // that; a job resumed from a checkpoint starts only tools that were pending
 // there, so it never overwrites the word of a tool running at any checkpoint
 // it or a later job may resume from.  A checkpoint is its state words alone.
-__host__ __device__ inline uint32_t lt_rows(uint32_t n) { return n + 2u * kLtStateWords; }
+template <bool W = false>
+__host__ __device__ inline uint32_t lt_rows(uint32_t n) { return n + 2u * lt_state_words<W>(); }
 
 template <uint32_t NC>
 __device__ __forceinline__ uint32_t lt_ready(const LtSharedT<NC>& S, uint32_t pend, uint32_t done) {
@@ -182,6 +192,7 @@ __device__ __forceinline__ void lt_fill_tables(LtSharedT<NC>& S) {
     w[5] = w[6] = 0u;         // T, V
     w[7] = 0xFFFFFFFFu;       // tc: no CPU tool runs
     w[8] = 0u;                // gm
+    w[9] = w[10] = 0u;        // the wide queue's second word
   }
 }
 
@@ -193,7 +204,7 @@ enum LtStep : uint32_t { kLtContinue = 0, kLtFinished = 1, kLtInfeasible = 2, kL
 // Returns kLtFinished once every tool has ended (the makespan is s.T).  The
 // loops' bodies are written as selects: lanes of a warp are at different
 // points of their simulations, and a branch in a body would run both sides.
-template <uint32_t NC>
+template <uint32_t NC, bool W = false>
 __device__ __forceinline__ uint32_t lt_step(const LtSharedT<NC>& S, LtState& s, uint32_t now, uint32_t que,
                                             uint32_t stop, uint32_t* e, uint32_t stride) {
   const LaneTreeRecord& R = S.rec;
@@ -218,14 +229,21 @@ __device__ __forceinline__ uint32_t lt_step(const LtSharedT<NC>& S, LtState& s, 
     // queued: join the FIFO in index order (a row is written when the tool starts)
     for (uint32_t m = ready & que; m; m &= m - 1u) {
       const uint32_t i = __ffs(m) - 1u;
-      s.qlist |= (uint64_t)i << (4u * __popc(s.qset));
+      const uint32_t pos = __popc(s.qset);
+      if (W) {  // 12 entries of 5 bits in the first word, the rest in the second
+        const uint32_t sh = 5u * pos;
+        s.qlist |= pos < 12u ? (uint64_t)i << (sh & 63u) : 0ull;
+        s.qhi |= pos >= 12u ? (uint64_t)i << ((sh - 60u) & 63u) : 0ull;
+      } else {
+        s.qlist |= (uint64_t)i << (4u * pos);
+      }
       s.qset |= 1u << i;
     }
     if ((ready & now) && lt_vram(S, s.run & gpu) > R.budget) return kLtInfeasible;  // out of memory
   }
   // ---- queue head: the first tool of the FIFO --------------------------------
   if (s.qset && !(s.run & que)) {
-    const uint32_t h = (uint32_t)(s.qlist & 15u), hb = 1u << h;
+    const uint32_t h = (uint32_t)(s.qlist & (W ? 31u : 15u)), hb = 1u << h;
     if (hb & R.big_mask) return kLtInfeasible;  // a head larger than M can never start
     const uint32_t rg = s.run & gpu;
     if (lt_vram(S, rg | hb) <= R.budget) {  // no bypass: otherwise the head waits
@@ -234,7 +252,12 @@ __device__ __forceinline__ uint32_t lt_step(const LtSharedT<NC>& S, LtState& s, 
       e[h * stride] = val;
       s.run |= hb;
       s.qset &= ~hb;
-      s.qlist >>= 4;
+      if (W) {
+        s.qlist = (s.qlist >> 5) | ((s.qhi & 31ull) << 55);
+        s.qhi >>= 5;
+      } else {
+        s.qlist >>= 4;
+      }
     }
   }
   // ---- next event -----------------------------------------------------------
@@ -279,9 +302,10 @@ __device__ __forceinline__ uint32_t lt_step(const LtSharedT<NC>& S, LtState& s, 
 // which loads the block's time-0 state like a checkpoint -- and a stopped
 // job saves its state as the next level's checkpoint and continues with that
 // level's first combination (every tool of it on the CPU).
-template <uint32_t NC, typename TakeRoot, typename Sink>
+template <uint32_t NC, bool W = false, typename TakeRoot, typename Sink>
 __device__ __forceinline__ void lt_lane(const LtSharedT<NC>& S, uint32_t* rows, uint32_t stride, TakeRoot take_root,
                                         Sink& sink) {
+  constexpr uint32_t SW = lt_state_words<W>();
   const LaneTreeRecord& R = S.rec;
   const uint32_t n = R.n;
   uint32_t* const cur = rows;
@@ -312,7 +336,7 @@ __device__ __forceinline__ void lt_lane(const LtSharedT<NC>& S, uint32_t* rows, 
         root = take_root();
         if (root == 0xFFFFFFFFu) return;
       }
-      uint32_t* const cw = rows + (L == 2u ? n + kLtStateWords : n) * stride;  // checkpoint L's state words
+      uint32_t* const cw = rows + (L == 2u ? n + SW : n) * stride;  // checkpoint L's state words
       if (descend) {  // save the state words
         cw[0] = s.pend;
         cw[stride] = s.run;
@@ -323,6 +347,10 @@ __device__ __forceinline__ void lt_lane(const LtSharedT<NC>& S, uint32_t* rows, 
         cw[6u * stride] = s.V;
         cw[7u * stride] = s.tc;
         cw[8u * stride] = s.gm;
+        if (W) {
+          cw[9u * stride] = (uint32_t)s.qhi;
+          cw[10u * stride] = (uint32_t)(s.qhi >> 32);
+        }
       } else {  // load a checkpoint's state words, or the time-0 state for a root
         const uint32_t* w = L == 0u ? S.ck0 : cw;
         const uint32_t ws = L == 0u ? 1u : stride;
@@ -334,6 +362,7 @@ __device__ __forceinline__ void lt_lane(const LtSharedT<NC>& S, uint32_t* rows, 
         s.V = w[6u * ws];
         s.tc = w[7u * ws];
         s.gm = w[8u * ws];
+        if (W) s.qhi = (uint64_t)w[9u * ws] | ((uint64_t)w[10u * ws] << 32);
       }
       // Modes and index part of the new job's level: a root's four table
       // parts (base-81 digits of the root), or one level combination (the
@@ -366,7 +395,7 @@ __device__ __forceinline__ void lt_lane(const LtSharedT<NC>& S, uint32_t* rows, 
       lvl = L;
       steps = 0u;
     }
-    r = lt_step(S, s, now, que, stop, cur, stride);
+    r = lt_step<NC, W>(S, s, now, que, stop, cur, stride);
     if (++steps > bound && r == kLtContinue) {  // never taken by a correct simulation
       s.T = kStalled;
       r = kLtFinished;

@@ -779,6 +779,14 @@ inline void lanetree_record(const bf_scenario_desc* d, bfk::LaneTreeRecord* r, u
 // sparse, fan-out/fan-in, spines with branches) the rule chose the lane tree
 // for all 40, and it was the faster on all 40.
 constexpr double kLtPreferRatio = 8.0;
+// Above 16 tools the lane tree runs its wide form (5-bit queue entries in two
+// words, 55 registers, 4 blocks per SM), whose events cost more: on layered
+// DAGs of 17 to 20 tools it won 2.05 to 2.3 times at ratios of 18.4 to 19.8
+// (the 24-tool layered workload's first 20 tools 850 -> 363 ms), 1.4 times
+// at 17.3, and lost 1.6 times at 12.8; the 19-tool workload's ratio is 6.6.
+// On 12 further DAGs of 17 to 19 tools it chose the lane tree for all 12,
+// the faster on all 12.
+constexpr double kLtPreferRatioWide = 15.0;
 inline bool lanetree_preferred(const bfk::Tables& rt, const bfk::Plan& rp, const bfk::Tables& rw,
                                const bfk::LaneTreeRecord& rec, double lt_events) {
   const uint32_t n = rt.n;
@@ -788,7 +796,7 @@ inline bool lanetree_preferred(const bfk::Tables& rt, const bfk::Plan& rp, const
   retired_estimate(rt, R);
   const uint32_t P = rp.P, I = rp.I;
   const double sk_events = R[P] / (double)pow3(rp.M + I) + (R[n - I] - R[P]) / (double)pow3(I) + (n - R[n - I]);
-  return sk_events * rw.n >= kLtPreferRatio * lt_events;
+  return sk_events * rw.n >= (n > kLtNarrowTools ? kLtPreferRatioWide : kLtPreferRatio) * lt_events;
 }
 
 }  // namespace host

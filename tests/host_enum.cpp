@@ -214,15 +214,16 @@ extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bo
 // the batch kernel's (the record bf_search_batch builds, 6-bit tables in two
 // chunks, n <= 12), otherwise the one-scenario kernel's (levels for at least
 // min_roots roots -- the closed-form estimate's, or with `sampled` those of
-// lanetree_sampled_levels, as bf_create_scenario takes them -- three
-// chunks, n <= 16).  The roots are split over the
+// lanetree_sampled_levels, as bf_create_scenario takes them -- three chunks
+// and the narrow queue up to 16 tools, four chunks and the wide queue up to
+// 20, or the wide form at any size when `wide` is set).  The roots are split over the
 // record's blocks, and every block's with `lanes` lanes, lane l taking the
 // block's roots l, l + lanes, ... (the kernels hand roots out from counters;
 // any order gives the same mappings).  Every mapping reported to the sink is
 // stored at its canonical index; out[] starts at 0xFFFFFFFF (infeasible
 // mappings are not reported) and a second report of one index stores
 // 0xDEADBEEF.  info[0..2] = x, y, blocks.
-template <uint32_t NC>
+template <uint32_t NC, bool W>
 static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, int sampled,
                             uint32_t* out, uint32_t* info) {
   LaneTreeRecord rec;
@@ -243,12 +244,12 @@ static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t 
     uint32_t* out;
     void operator()(uint32_t idx, uint32_t ms) { out[idx] = out[idx] == 0xFFFFFFFFu ? ms : 0xDEADBEEFu; }
   } sink{out};
-  std::vector<uint32_t> rows((size_t)lt_rows(d->n) * lanes, 0xA5A5A5A5u);  // stale shared memory
+  std::vector<uint32_t> rows((size_t)lt_rows<W>(d->n) * lanes, 0xA5A5A5A5u);  // stale shared memory
   for (uint32_t b = 0; b < rec.nblocks; ++b) {
     const uint32_t r0 = (uint32_t)(roots * b / rec.nblocks), r1 = (uint32_t)(roots * (b + 1) / rec.nblocks);
     for (uint32_t lane = 0; lane < lanes; ++lane) {
       uint32_t next = r0 + lane;
-      lt_lane(S, rows.data() + lane, lanes,
+      lt_lane<NC, W>(S, rows.data() + lane, lanes,
               [&]() {
                 const uint32_t r = next;
                 next += lanes;
@@ -260,9 +261,11 @@ static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t 
   return 0;
 }
 
-extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, int sampled,
+extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, int sampled, int wide,
                              uint32_t* out, uint32_t* info) {
   if (lanes == 0) return -1;
-  if (min_roots == 0) return d->n <= kLtBatchTools ? host_lanetree_nc<2>(d, lanes, 0, 0, out, info) : -1;
-  return d->n <= kLtMaxTools ? host_lanetree_nc<3>(d, lanes, min_roots, sampled, out, info) : -1;
+  if (min_roots == 0) return d->n <= kLtBatchTools ? host_lanetree_nc<2, false>(d, lanes, 0, 0, out, info) : -1;
+  if (d->n > kLtMaxTools) return -1;
+  if (!wide && d->n <= kLtNarrowTools) return host_lanetree_nc<3, false>(d, lanes, min_roots, sampled, out, info);
+  return host_lanetree_nc<4, true>(d, lanes, min_roots, sampled, out, info);
 }

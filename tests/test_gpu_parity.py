@@ -234,6 +234,34 @@ def test_lanetree_full_queue_of_16():
         assert (r.index, r.makespan_us) == want, tight
 
 
+def _layered_scn(seed, sizes, budget):
+    rng = np.random.default_rng(seed)
+    n = sum(sizes)
+    c, g, x, m = S._ordinary(rng, n, 2048, 16384)
+    pred = S._layered_edges(rng, sizes, 0.4)
+    return S.Scenario(n, pred, c, g, x, [S._load_from_vram(v) for v in m], m, budget, S.slowdown_linear(kmax=n))
+
+
+def test_lanetree_wide_search():
+    """Full searches of 17 to 20 tools on the wide form of the one-scenario lane tree (four table chunks,
+    5-bit queue entries in two words): a 17-tool layered DAG and 17 tools without edges (all seventeen
+    queued at once in the all-queue mapping) against the oracle, and 18- and 20-tool layered DAGs
+    against the search kernel run as two half-range searches (range searches always take it)."""
+    for scn in (_layered_scn(61, [4, 4, 3, 3, 3], 24576),
+                S.random_small(np.random.default_rng(17), 17, edge_p=0.0, tight=True, contention=True, max_time=9)):
+        want = oracle.search(scn, THREADS)
+        with bf.create_scenario(scn) as h:
+            r = bf.search_best(h)
+        assert (r.index, r.makespan_us) == want
+    for scn in (_layered_scn(62, [4, 4, 4, 3, 3], 32768), _layered_scn(63, [4] * 5, 40960)):
+        total = 3 ** scn.n
+        with bf.create_scenario(scn) as h:
+            r = bf.search_best(h)
+            halves = [bf.search_range(h, 0, total // 2), bf.search_range(h, total // 2, total - total // 2)]
+        best = min((x.makespan_us, x.index) for x in halves if x.feasible)
+        assert (r.index, r.makespan_us) == (best[1], best[0]), scn.n
+
+
 def test_degenerate_budgets_all_paths():
     """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
     the batch, the branch and bound and the tree search, against the oracle."""

@@ -46,14 +46,14 @@ def host():
         return ms.astype(np.uint64), info
     run.pruned = lambda scn, bound: lib.host_pruned(ctypes.byref(bf.to_desc(scn)), bound)
     lib.host_lanetree.argtypes = [ctypes.POINTER(bf.Desc), ctypes.c_uint32, ctypes.c_uint64, ctypes.c_int,
-                                  ctypes.c_void_p, ctypes.c_void_p]
+                                  ctypes.c_int, ctypes.c_void_p, ctypes.c_void_p]
     lib.host_lanetree.restype = ctypes.c_int
 
-    def lanetree(scn, lanes, min_roots=0, sampled=False):
+    def lanetree(scn, lanes, min_roots=0, sampled=False, wide=False):
         ms = np.zeros(3 ** scn.n, np.uint32)
         info = np.zeros(3, np.uint32)
-        assert lib.host_lanetree(ctypes.byref(bf.to_desc(scn)), lanes, min_roots, int(sampled), ms.ctypes.data,
-                                 info.ctypes.data) == 0
+        assert lib.host_lanetree(ctypes.byref(bf.to_desc(scn)), lanes, min_roots, int(sampled), int(wide),
+                                 ms.ctypes.data, info.ctypes.data) == 0
         return ms.astype(np.uint64), info
     run.lanetree = lanetree
     return run
@@ -147,8 +147,8 @@ def test_tie_order_scenarios_host(host):
             assert got == tuple(want), (t, bound, got, want)
 
 
-def _same_lanetree(host, scn, lanes, min_roots=0, sampled=False):
-    got, info = host.lanetree(scn, lanes, min_roots, sampled)
+def _same_lanetree(host, scn, lanes, min_roots=0, sampled=False, wide=False):
+    got, info = host.lanetree(scn, lanes, min_roots, sampled, wide)
     want, _ = oracle.eval_range(scn, 0, 3 ** scn.n, THREADS)
     bad = np.flatnonzero(got != want)
     assert bad.size == 0, (f"levels x={int(info[0])} y={int(info[1])}, {int(info[2])} blocks: {bad.size} "
@@ -221,3 +221,21 @@ def test_lanetree_whole_space_records(host):
                      full.slowdown_q10)
     info = _same_lanetree(host, cut, 32, 3 ** 10, sampled=True)
     assert int(info[0]) >= 10 and int(info[1]) < m
+
+
+def test_lanetree_wide_queue_form(host):
+    """The wide form of the one-scenario lane tree (four table chunks, 5-bit queue entries in two words,
+    eleven state words per checkpoint), run at small sizes so that every mapping is checked: random DAGs
+    of 8-13 tools with small integer times, and 13 tools without edges whose all-queue mapping holds 13
+    waiting tools (the second queue word holds the 13th), each against the oracle."""
+    rng = np.random.default_rng(94)
+    for t in range(16):
+        n = int(rng.integers(8, 14))
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.0, 0.2, 0.4])), tight=bool(t % 3),
+                              contention=bool(t % 4), max_time=int(rng.choice([3, 7, 40])))
+        _same_lanetree(host, base, (1, 3, 32)[t % 3], 3 ** int(rng.integers(n - 6, n)), sampled=bool(t % 2),
+                       wide=True)
+    for tight in (False, True):
+        flat = S.random_small(rng, 13, edge_p=0.0, tight=tight, contention=True, max_time=9)
+        assert all(p == 0 for p in flat.pred_mask)
+        _same_lanetree(host, flat, 32, 3 ** 9, wide=True)
