@@ -770,14 +770,23 @@ int bf_search_pruned(const bf_scenario* scn_const, uint64_t hint_index, bf_resul
   return BF_OK;
 }
 
-// Batches of at least this many lane-tree scenarios are pipelined: the first
-// eighth is built, copied and launched on the caller's stream, and the rest
-// is built while that kernel runs and launched on a second stream (created
-// for the call) that waits only for the key reset, so that the two kernels
-// overlap; the caller's stream waits for the second before the keys come
-// back.  4096 x 3^10: the kernel otherwise waits about 0.5 ms for the
-// records.
+// A batch runs on the lane-tree batch kernel in up to three groups, one per
+// table form: up to kLtBatchTools tools, up to kLtNarrowTools, up to
+// kLtMaxTools (a 14-tool layered batch scenario ran on the prefix/mid/inner
+// batch kernel before; the no-alloc entry point still takes that kernel above
+// kLtBatchTools).  Batches of at least kBatchPipelineMin scenarios of the
+// first group are pipelined: the first eighth of that group is built, copied
+// and launched on the caller's stream, and the rest of the batch is built
+// while that kernel runs and launched on a second stream (created for the
+// call) that waits only for the key reset, so that the kernels overlap; the
+// caller's stream waits for the second before the keys come back.  4096 x
+// 3^10: the kernel otherwise waits about 0.5 ms for the records.
 constexpr uint32_t kBatchPipelineMin = 1024;
+constexpr uint32_t kBatchGroups = 3;
+
+inline uint32_t batch_group(uint32_t n) {
+  return n <= bfk::kLtBatchTools ? 0u : (n <= bfk::kLtNarrowTools ? 1u : 2u);
+}
 
 static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_result* out, void* cuda_stream) {
   if (count == 0) return BF_OK;
@@ -788,30 +797,45 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
     if (rc == BF_OK) rc = require_enum(descs[bad], "bf_search_batch");
     return fail(rc == BF_OK ? BF_EINVAL : rc, "bf_search_batch: descs[%u]: %s", bad, g_error.c_str());
   }
-  std::vector<uint32_t> small(count), large(count);
-  const BatchSplit b = split_batch(descs, count, small, large);
-  const bool pipe = b.ns >= kBatchPipelineMin;
-  const uint32_t k1 = pipe ? b.ns / 8u : b.ns;  // lane-tree scenarios of the first launch
+  // Positions ordered by group, each group in the batch's order; key j and
+  // record j belong to position ids[j].
+  uint32_t gcount[kBatchGroups] = {}, gnmax[kBatchGroups] = {};
+  for (uint32_t i = 0; i < count; ++i) ++gcount[batch_group(descs[i].n)];
+  std::vector<uint32_t> ids(count);
+  uint32_t fill[kBatchGroups] = {0u, gcount[0], gcount[0] + gcount[1]};
+  for (uint32_t i = 0; i < count; ++i) {
+    const uint32_t g = batch_group(descs[i].n);
+    ids[fill[g]++] = i;
+    gnmax[g] = descs[i].n > gnmax[g] ? descs[i].n : gnmax[g];
+  }
+  const bool pipe = gcount[0] >= kBatchPipelineMin;
+  const uint32_t k1 = pipe ? gcount[0] / 8u : gcount[0];
+  // Launch l covers positions [lb[l], lb[l + 1]): the first part of group 0,
+  // the rest of it, group 1, group 2; its first-block array has
+  // lb[l + 1] - lb[l] + 1 entries at fb[lb[l] + l].
+  const uint32_t lb[5] = {0u, k1, gcount[0], gcount[0] + gcount[1], count};
+  const uint32_t lnmax[4] = {gnmax[0], gnmax[0], gnmax[1], gnmax[2]};
   // Record buffers of the calling thread, grown as needed and reused: a
   // fresh 2.8 MB array (4096 scenarios) cost about 0.4 ms of zeroing and page
   // faults per call.  Every record is written whole before it is copied; a
   // copy from pageable memory has read it by the time cudaMemcpyAsync
   // returns, so the next call may reuse the buffers even after a timeout.
   thread_local std::vector<bfk::LaneTreeRecord> lt;
-  thread_local std::vector<bfk::BatchRecord> bk;
-  if (lt.size() < b.ns) lt.resize(b.ns);
-  if (bk.size() < b.nl) bk.resize(b.nl);
-  std::vector<uint32_t> fb1(k1 + 1, 0u), fb2(b.ns - k1 + 1, 0u);  // first blocks of each launch
-  build_lanetree_records(descs, small.data(), k1, lt.data());
-  for (uint32_t j = 0; j < k1; ++j) fb1[j + 1] = fb1[j] + lt[j].nblocks;
+  if (lt.size() < count) lt.resize(count);
+  std::vector<uint32_t> fb(count + 4, 0u);
+  auto build = [&](uint32_t l0, uint32_t l1) {  // records and first blocks of launches [l0, l1)
+    build_lanetree_records(descs, ids.data() + lb[l0], lb[l1] - lb[l0], lt.data() + lb[l0]);
+    for (uint32_t l = l0; l < l1; ++l) {
+      uint32_t* f = fb.data() + lb[l] + l;
+      for (uint32_t j = lb[l]; j < lb[l + 1]; ++j) f[j - lb[l] + 1] = f[j - lb[l]] + lt[j].nblocks;
+    }
+  };
+  build(0, 1);
 
-  // One device allocation: lane-tree records, the two first-block arrays,
-  // batch records, keys.
-  const size_t lt_bytes = sizeof(bfk::LaneTreeRecord) * b.ns, kbytes = sizeof(unsigned long long) * count;
-  const size_t fb1_bytes = sizeof(uint32_t) * fb1.size(), fb2_bytes = sizeof(uint32_t) * fb2.size();
-  const size_t bk_bytes = sizeof(bfk::BatchRecord) * b.nl;
-  const size_t off_fb1 = align256(lt_bytes), off_fb2 = off_fb1 + align256(fb1_bytes);
-  const size_t off_bk = off_fb2 + align256(fb2_bytes), off_keys = off_bk + align256(bk_bytes);
+  // One device allocation: records, first-block arrays, keys.
+  const size_t lt_bytes = sizeof(bfk::LaneTreeRecord) * count, fb_bytes = sizeof(uint32_t) * fb.size();
+  const size_t kbytes = sizeof(unsigned long long) * count;
+  const size_t off_fb = align256(lt_bytes), off_keys = off_fb + align256(fb_bytes);
   cudaStream_t st = static_cast<cudaStream_t>(cuda_stream);
   cudaStream_t rest = st;  // stream of the later launches
   cudaEvent_t reset_done = nullptr, rest_done = nullptr;
@@ -819,10 +843,14 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
   std::vector<unsigned long long> keys(count);
   cudaError_t e = lib_malloc_async(reinterpret_cast<void**>(&d_base), off_keys + kbytes, st);
   auto* d_lt = reinterpret_cast<bfk::LaneTreeRecord*>(d_base);
-  auto* d_fb1 = reinterpret_cast<uint32_t*>(d_base + off_fb1);
-  auto* d_fb2 = reinterpret_cast<uint32_t*>(d_base + off_fb2);
-  auto* d_bk = reinterpret_cast<bfk::BatchRecord*>(d_base + off_bk);
+  auto* d_fb = reinterpret_cast<uint32_t*>(d_base + off_fb);
   auto* d_keys = reinterpret_cast<unsigned long long*>(d_base + off_keys);
+  auto launch = [&](uint32_t l, cudaStream_t s) {
+    const uint32_t c = lb[l + 1] - lb[l];
+    if (c == 0) return cudaSuccess;
+    const uint32_t* f = fb.data() + lb[l] + l;
+    return bfk::launch_lanetree(d_lt + lb[l], d_fb + lb[l] + l, c, f[c], lnmax[l], d_keys + lb[l], s);
+  };
   if (e == cudaSuccess && pipe) {
     e = cudaStreamCreateWithFlags(&rest, cudaStreamNonBlocking);
     if (e != cudaSuccess) rest = st;
@@ -830,32 +858,24 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
     if (e == cudaSuccess) e = cudaEventCreateWithFlags(&rest_done, cudaEventDisableTiming);
   }
   if (e == cudaSuccess && k1) e = cudaMemcpyAsync(d_lt, lt.data(), sizeof(bfk::LaneTreeRecord) * k1, cudaMemcpyHostToDevice, st);
-  if (e == cudaSuccess && k1) e = cudaMemcpyAsync(d_fb1, fb1.data(), fb1_bytes, cudaMemcpyHostToDevice, st);
+  if (e == cudaSuccess && k1) e = cudaMemcpyAsync(d_fb, fb.data(), sizeof(uint32_t) * (k1 + 1), cudaMemcpyHostToDevice, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, kbytes, st);
   if (e == cudaSuccess && rest != st) e = cudaEventRecord(reset_done, st);
-  if (e == cudaSuccess && k1) e = bfk::launch_lanetree(d_lt, d_fb1, k1, fb1[k1], b.nmax_small, d_keys, st);
+  if (e == cudaSuccess) e = launch(0, st);
   bool rest_used = false;  // work enqueued on `rest` that the caller's stream must wait for
-  if (e == cudaSuccess) {
-    // The rest of the records, built while the first launch runs.
-    build_lanetree_records(descs, small.data() + k1, b.ns - k1, lt.data() + k1);
-    for (uint32_t j = k1; j < b.ns; ++j) fb2[j - k1 + 1] = fb2[j - k1] + lt[j].nblocks;
-    uint32_t wmax = 0, pmax = 0, any_inner = 0;
-    build_records(descs, large.data(), b.nl, bk.data(), &wmax, &pmax, &any_inner);
+  if (e == cudaSuccess && count > k1) {
+    build(1, 4);  // the other records, built while the first launch runs
     if (rest != st) {
       e = cudaStreamWaitEvent(rest, reset_done, 0);
       rest_used = e == cudaSuccess;
     }
-    const uint32_t k2 = b.ns - k1;
-    if (e == cudaSuccess && k2)
-      e = cudaMemcpyAsync(d_lt + k1, lt.data() + k1, sizeof(bfk::LaneTreeRecord) * k2, cudaMemcpyHostToDevice, rest);
-    if (e == cudaSuccess && k2) e = cudaMemcpyAsync(d_fb2, fb2.data(), fb2_bytes, cudaMemcpyHostToDevice, rest);
-    if (e == cudaSuccess && b.nl) e = cudaMemcpyAsync(d_bk, bk.data(), bk_bytes, cudaMemcpyHostToDevice, rest);
-    if (e == cudaSuccess && k2) e = bfk::launch_lanetree(d_lt + k1, d_fb2, k2, fb2[k2], b.nmax_small, d_keys + k1, rest);
-    if (e == cudaSuccess && b.nl) {
-      BatchSplit bl = b;
-      bl.ns = 0;  // the batch-kernel group alone, its keys after the lane-tree group's
-      e = launch_batch_groups(bl, nullptr, nullptr, 0, d_bk, wmax, pmax, any_inner, d_keys + b.ns, rest);
-    }
+    if (e == cudaSuccess)
+      e = cudaMemcpyAsync(d_lt + k1, lt.data() + k1, sizeof(bfk::LaneTreeRecord) * (count - k1),
+                          cudaMemcpyHostToDevice, rest);
+    if (e == cudaSuccess)  // first blocks of launches 1 to 3
+      e = cudaMemcpyAsync(d_fb + k1 + 1, fb.data() + k1 + 1, sizeof(uint32_t) * (fb.size() - k1 - 1),
+                          cudaMemcpyHostToDevice, rest);
+    for (uint32_t l = 1; l < 4 && e == cudaSuccess; ++l) e = launch(l, rest);
   }
   // The caller's stream waits for the later launches (also after an error,
   // before the scratch is freed there); if that cannot be enqueued, the host
@@ -888,8 +908,7 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
   if (reset_done) cudaEventDestroy(reset_done);
   if (rest_done) cudaEventDestroy(rest_done);
   if (rc != BF_OK) return rc;
-  for (uint32_t j = 0; j < b.ns; ++j) fill_result(keys[j], descs[small[j]].n, 0, out + small[j]);
-  for (uint32_t j = 0; j < b.nl; ++j) fill_result(keys[b.ns + j], descs[large[j]].n, 0, out + large[j]);
+  for (uint32_t j = 0; j < count; ++j) fill_result(keys[j], descs[ids[j]].n, 0, out + ids[j]);
   return BF_OK;
 }
 

@@ -38,12 +38,15 @@ __device__ __forceinline__ void lt_load_record(LtSharedT<NC>& S, const LaneTreeR
 // Block b searches roots [3^x * j / nblocks, 3^x * (j + 1) / nblocks) of
 // scenario s, where first_block[s] <= b < first_block[s + 1] and j = b -
 // first_block[s]; the lowest key (makespan << 32 | canonical index) it finds
-// goes to keys[s] by one atomicMin per warp.
-__global__ void __launch_bounds__(kLtThreads, kLtBlocksPerSm) lanetree_kernel(const LaneTreeRecord* __restrict__ recs,
-                                                             const uint32_t* __restrict__ first_block,
-                                                             uint32_t count, unsigned long long* keys) {
+// goes to keys[s] by one atomicMin per warp.  NC table chunks and the queue
+// form W as for the one-scenario kernel: <2, false> up to 12 tools, <3,
+// false> up to 16, <4, true> up to 20.
+template <uint32_t NC, bool W>
+__global__ void __launch_bounds__(kLtThreads, W ? kLtWideBlocksPerSm : kLtBlocksPerSm)
+    lanetree_kernel(const LaneTreeRecord* __restrict__ recs, const uint32_t* __restrict__ first_block, uint32_t count,
+                    unsigned long long* keys) {
   extern __shared__ uint32_t lt_rows_smem[];
-  __shared__ LtShared S;
+  __shared__ LtSharedT<NC> S;
   uint32_t lo = 0u, hi = count;  // first_block[lo] <= blockIdx.x < first_block[hi]
   while (hi - lo > 1u) {
     const uint32_t mid = (lo + hi) >> 1;
@@ -61,8 +64,8 @@ __global__ void __launch_bounds__(kLtThreads, kLtBlocksPerSm) lanetree_kernel(co
   }
   __syncthreads();
   MinKeySink sink;
-  LtShared& Sref = S;
-  lt_lane(S, lt_rows_smem + threadIdx.x, blockDim.x,
+  LtSharedT<NC>& Sref = S;
+  lt_lane<NC, W>(S, lt_rows_smem + threadIdx.x, blockDim.x,
           [&Sref]() {
             const uint32_t r = atomicAdd(&Sref.root_next, 1u);
             return r < Sref.root_end ? r : 0xFFFFFFFFu;
@@ -148,10 +151,25 @@ cudaError_t single_kernel_for(uint32_t n, SingleKernel* k, size_t* smem) {
 
 cudaError_t launch_lanetree(const LaneTreeRecord* d_recs, const uint32_t* d_first_block, uint32_t count,
                             uint32_t blocks, uint32_t nmax, unsigned long long* keys, cudaStream_t st) {
-  static std::atomic<uint64_t> ready{0};
-  cudaError_t e = allow_dyn_smem(lanetree_kernel, lt_smem_bytes(kLtBatchTools), &ready);
+  static std::atomic<uint64_t> ready2{0}, ready3{0}, ready4{0};
+  cudaError_t e = cudaSuccess;
+  if (nmax <= kLtBatchTools) {
+    e = allow_dyn_smem(lanetree_kernel<2, false>, lt_smem_bytes<false>(kLtBatchTools), &ready2);
+    if (e == cudaSuccess)
+      lanetree_kernel<2, false><<<blocks, kLtThreads, lt_smem_bytes<false>(nmax), st>>>(d_recs, d_first_block, count,
+                                                                                       keys);
+  } else if (nmax <= kLtNarrowTools) {
+    e = allow_dyn_smem(lanetree_kernel<3, false>, lt_smem_bytes<false>(kLtNarrowTools), &ready3);
+    if (e == cudaSuccess)
+      lanetree_kernel<3, false><<<blocks, kLtThreads, lt_smem_bytes<false>(nmax), st>>>(d_recs, d_first_block, count,
+                                                                                       keys);
+  } else {
+    e = allow_dyn_smem(lanetree_kernel<4, true>, lt_smem_bytes<true>(kLtMaxTools), &ready4);
+    if (e == cudaSuccess)
+      lanetree_kernel<4, true><<<blocks, kLtThreads, lt_smem_bytes<true>(nmax), st>>>(d_recs, d_first_block, count,
+                                                                                     keys);
+  }
   if (e != cudaSuccess) return e;
-  lanetree_kernel<<<blocks, kLtThreads, lt_smem_bytes(nmax), st>>>(d_recs, d_first_block, count, keys);
   return cudaGetLastError();
 }
 

@@ -10,9 +10,11 @@
 
 namespace bfk {
 
-// The lane-tree batch kernel: scenarios of up to kLtBatchTools tools;
+// The lane-tree batch kernel: scenarios of up to kLtMaxTools tools, one launch
+// per group of the same table form (up to kLtBatchTools tools, up to
+// kLtNarrowTools, up to kLtMaxTools; nmax, the group's largest n, picks it);
 // d_first_block[count + 1] holds each scenario's first block (prefix sums of
-// LaneTreeRecord::nblocks), `blocks` = its last entry, nmax the largest n.
+// LaneTreeRecord::nblocks), `blocks` = its last entry.
 // keys[s] must hold ~0 before the launch; it receives the lowest key
 // (makespan << 32 | canonical index) of scenario s.
 cudaError_t launch_lanetree(const LaneTreeRecord* d_recs, const uint32_t* d_first_block, uint32_t count,

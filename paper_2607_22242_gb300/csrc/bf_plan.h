@@ -486,6 +486,11 @@ inline bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n, uint32_t block_wa
 // 13.4 ms.
 constexpr uint64_t kLtBlockMappings = 7381;
 constexpr uint64_t kLtMinRootsPerBlock = 512;
+// Blocks one scenario of a batch gets at most: with 512 roots per block this
+// keeps the roots of a 16-tool scenario at 12 tools (as its full search over
+// the whole GPU takes them) instead of 14, and a 20-tool one's at 12 instead
+// of 18 (472,000 blocks).  Scenarios of up to 14 tools stay below it.
+constexpr uint64_t kLtMaxBlocksPerScenario = 1024;
 
 // The levels of the lane-tree search of one scenario (n <= kLtMaxTools):
 // roots [0, x), then [x, y), then [y, n).  Each level below the root holds at
@@ -529,7 +534,8 @@ inline double lanetree_levels(const TB& t, uint64_t min_roots, uint32_t* x_out, 
 // and the blocks its scenario's roots are split over.
 template <typename TB>
 inline void lanetree_split(const TB& t, uint32_t* x_out, uint32_t* y_out, uint32_t* nblocks) {
-  const uint64_t want_blocks = (pow3(t.n) + kLtBlockMappings - 1) / kLtBlockMappings;
+  uint64_t want_blocks = (pow3(t.n) + kLtBlockMappings - 1) / kLtBlockMappings;
+  if (want_blocks > kLtMaxBlocksPerScenario) want_blocks = kLtMaxBlocksPerScenario;
   lanetree_levels(t, kLtMinRootsPerBlock * want_blocks, x_out, y_out);
   const uint64_t cap = pow3(*x_out) / kLtMinRootsPerBlock;
   uint64_t nb = want_blocks < cap ? want_blocks : cap;

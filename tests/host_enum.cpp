@@ -211,8 +211,9 @@ extern "C" unsigned long long host_pruned(const bf_scenario_desc* d, uint32_t bo
 }
 
 // A lane-tree search (bf_lanetree.cuh) of one scenario: with min_roots == 0
-// the batch kernel's (the record bf_search_batch builds, 6-bit tables in two
-// chunks, n <= 12), otherwise the one-scenario kernel's (levels for at least
+// the batch kernel's (the record bf_search_batch builds, in its group's form:
+// two 6-bit table chunks up to 12 tools, three up to 16, four and the wide
+// queue above or when `wide` is set), otherwise the one-scenario kernel's (levels for at least
 // min_roots roots -- the closed-form estimate's, or with `sampled` those of
 // lanetree_sampled_levels, as bf_create_scenario takes them -- three chunks
 // and the narrow queue up to 16 tools, four chunks and the wide queue up to
@@ -263,9 +264,13 @@ static int host_lanetree_nc(const bf_scenario_desc* d, uint32_t lanes, uint64_t 
 
 extern "C" int host_lanetree(const bf_scenario_desc* d, uint32_t lanes, uint64_t min_roots, int sampled, int wide,
                              uint32_t* out, uint32_t* info) {
-  if (lanes == 0) return -1;
-  if (min_roots == 0) return d->n <= kLtBatchTools ? host_lanetree_nc<2, false>(d, lanes, 0, 0, out, info) : -1;
-  if (d->n > kLtMaxTools) return -1;
+  if (lanes == 0 || d->n > kLtMaxTools) return -1;
+  if (min_roots == 0) {  // the batch's records, in the form of the batch kernel's group
+    if (wide) return host_lanetree_nc<4, true>(d, lanes, 0, 0, out, info);
+    if (d->n <= kLtBatchTools) return host_lanetree_nc<2, false>(d, lanes, 0, 0, out, info);
+    if (d->n <= kLtNarrowTools) return host_lanetree_nc<3, false>(d, lanes, 0, 0, out, info);
+    return host_lanetree_nc<4, true>(d, lanes, 0, 0, out, info);
+  }
   if (!wide && d->n <= kLtNarrowTools) return host_lanetree_nc<3, false>(d, lanes, min_roots, sampled, out, info);
   return host_lanetree_nc<4, true>(d, lanes, min_roots, sampled, out, info);
 }

@@ -262,6 +262,22 @@ def test_lanetree_wide_search():
         assert (r.index, r.makespan_us) == (best[1], best[0]), scn.n
 
 
+def test_batch_of_larger_scenarios():
+    """Batches run scenarios of 13-16 tools and of 17-20 tools on the lane-tree batch kernel's larger
+    forms (three table chunks; four and the wide queue): a batch of layered DAGs of 10 and 13 to 19
+    tools, each result equal to that scenario's own full search (itself checked against the oracle)."""
+    scns = [_layered_scn(70 + k, sizes, 24576 + 8192 * (k % 2))
+            for k, sizes in enumerate([[4, 3, 3], [4, 4, 3, 2], [4, 4, 4, 3], [4, 4, 4, 4], [4, 4, 3, 3, 3],
+                                       [4, 4, 4, 4, 3], [3, 3, 4]])]
+    assert sorted(s.n for s in scns) == [10, 10, 13, 15, 16, 17, 19]
+    want = []
+    for scn in scns:
+        with bf.create_scenario(scn) as h:
+            r = bf.search_best(h)
+        want.append((r.index, r.makespan_us))
+    assert [(r.index, r.makespan_us) for r in bf.search_batch(scns)] == want
+
+
 def test_degenerate_budgets_all_paths():
     """Zero VRAM budget (only all-cpu feasible) and maximal contention, through the exhaustive search,
     the batch, the branch and bound and the tree search, against the oracle."""

@@ -239,3 +239,16 @@ def test_lanetree_wide_queue_form(host):
         flat = S.random_small(rng, 13, edge_p=0.0, tight=tight, contention=True, max_time=9)
         assert all(p == 0 for p in flat.pred_mask)
         _same_lanetree(host, flat, 32, 3 ** 9, wide=True)
+
+
+def test_lanetree_batch_records_of_larger_scenarios(host):
+    """The batch's records of scenarios of 13 and 14 tools (the batch kernel's three-chunk group; at
+    most 1,024 blocks per scenario) and, in the wide form, of 9-12 tools: every mapping against the
+    oracle."""
+    rng = np.random.default_rng(95)
+    for t in range(6):
+        n = 13 + t % 2 if t < 4 else int(rng.integers(9, 13))
+        base = S.random_small(rng, n, edge_p=float(rng.choice([0.2, 0.35])), tight=bool(t % 3),
+                              contention=True, max_time=int(rng.choice([5, 40])))
+        info = _same_lanetree(host, base, 32, 0, wide=t >= 4)
+        assert int(info[2]) >= 1
