@@ -163,7 +163,8 @@ BF_API int bf_search_best(const bf_scenario* scn, bf_result* out, void* cuda_str
 BF_API int bf_search_range(const bf_scenario* scn, uint64_t first, uint64_t count,
                     bf_result* out, void* cuda_stream);
 
-/* Full search of `count` independent scenarios in one launch: out[i] is the
+/* Full search of `count` independent scenarios in one call (one launch per
+ * group of scenarios of similar size, four at most): out[i] is the
  * brute-force oracle of §2.3/§4.1 (as bf_search_best) for descs[i].  The paper
  * searches one workflow at a time; running many per launch is this library's
  * addition, for callers that score many workflows or many candidate

@@ -330,7 +330,7 @@ def _batch_call(fn, scns: Sequence[Scenario], stream, packed=None) -> List[Resul
 
 
 def search_batch(scns: Sequence[Scenario], stream=None, packed=None) -> List[Result]:
-    """Full search of each scenario, one launch for the whole batch.  ``packed`` (from
+    """Full search of each scenario, the whole batch in one call.  ``packed`` (from
     :func:`pack_descs` of the same scenarios) skips the packing when a batch is searched repeatedly."""
     return _batch_call(load().bf_search_batch, scns, stream, packed)
 
