@@ -290,7 +290,7 @@ BF_API int bf_whatif(const bf_scenario* scn, uint64_t base_index, bf_probe* out,
  * must not let cudaMalloc/cudaFree synchronise the device between rounds.
  * The caller passes the inputs (descs) and outputs (out) as for
  * bf_search_batch; the scratch (packed scenario records and one key per
- * scenario, about 2.8 MiB for BF_NOALLOC_MAX_SCENARIOS) is a fixed array in
+ * scenario, about 0.84 MiB for BF_NOALLOC_MAX_SCENARIOS) is a fixed array in
  * the library's device image, held on every GPU that loads the library until
  * the process exits.  count > BF_NOALLOC_MAX_SCENARIOS fails with BF_EINVAL.
  * The first call on a device (and the first after a device reset) resolves

@@ -29,8 +29,6 @@ using bfk::host::make_plan;
 using bfk::host::pow3;
 using bfk::host::split_and_window;
 using bfk::host::split_and_window_pruned;
-using bfk::host::batch_plan;
-using bfk::host::batch_split;
 using bfk::host::kSearchTasks;
 using bfk::host::whole_space_tables;
 using bfk::host::lanetree_record;
@@ -320,36 +318,6 @@ uint32_t first_invalid(const bf_scenario_desc* descs, uint32_t count) {
   return bad;
 }
 
-// Batch-kernel records (tables, window tables, plan) of descs[ids[j]], j <
-// count; the largest window, task count and whether any plan has an inner
-// level are returned too.
-void build_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count, bfk::BatchRecord* recs,
-                   uint32_t* wmax, uint32_t* pmax, uint32_t* any_inner) {
-  struct Part {
-    uint32_t wmax = 0, pmax = 0, inner = 0;
-  };
-  std::vector<Part> parts;
-  parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part* part) {
-    for (uint32_t j = lo; j < hi; ++j) {
-      bfk::BatchRecord& r = recs[j];
-      std::memset(&r, 0, sizeof r);
-      bfk::Plan base;
-      batch_split(descs + ids[j], &r.full, &base, &r.window);
-      r.plan = batch_plan(base, descs[ids[j]].n, bfk::kThreads / 32);
-      r.mid_lanes = base.W0 == 0u ? 1u : 0u;
-      if (r.window.n > part->wmax) part->wmax = r.window.n;
-      const uint32_t tasks = r.plan.groups * r.plan.m_parts;
-      if (tasks > part->pmax) part->pmax = tasks;
-      part->inner |= r.plan.I;
-    }
-  });
-  for (const Part& p : parts) {
-    *wmax = p.wmax > *wmax ? p.wmax : *wmax;
-    *pmax = p.pmax > *pmax ? p.pmax : *pmax;
-    *any_inner |= p.inner;
-  }
-}
-
 // Lane-tree records of descs[ids[j]], j < count.
 void build_lanetree_records(const bf_scenario_desc* descs, const uint32_t* ids, uint32_t count,
                             bfk::LaneTreeRecord* recs) {
@@ -358,47 +326,6 @@ void build_lanetree_records(const bf_scenario_desc* descs, const uint32_t* ids, 
   parallel_parts(count, parts, [&](uint32_t lo, uint32_t hi, Part*) {
     for (uint32_t j = lo; j < hi; ++j) lanetree_record(descs + ids[j], recs + j);
   });
-}
-
-// Where a batch's scenarios go: up to kLtBatchTools tools the lane-tree
-// kernel (bf_lanetree.cuh), above it the batch kernel (bf_kernels.cu).  The
-// keys of the first group come first in the key array.
-struct BatchSplit {
-  uint32_t ns = 0, nl = 0;            // scenarios in each group
-  uint32_t nmax_small = 0, nmax_large = 0;
-};
-
-template <typename Ids>
-BatchSplit split_batch(const bf_scenario_desc* descs, uint32_t count, Ids& small, Ids& large) {
-  BatchSplit b;
-  for (uint32_t i = 0; i < count; ++i) {
-    const uint32_t n = descs[i].n;
-    if (n <= bfk::kLtBatchTools) {
-      small[b.ns++] = i;
-      b.nmax_small = n > b.nmax_small ? n : b.nmax_small;
-    } else {
-      large[b.nl++] = i;
-      b.nmax_large = n > b.nmax_large ? n : b.nmax_large;
-    }
-  }
-  return b;
-}
-
-// Launch both groups of a batch on `st` (records already on the device; keys
-// reset to ~0): keys[0, ns) for the lane-tree group, keys[ns, ns + nl) for
-// the other.
-cudaError_t launch_batch_groups(const BatchSplit& b, const bfk::LaneTreeRecord* d_lt, const uint32_t* d_first_block,
-                                uint32_t lt_blocks, const bfk::BatchRecord* d_bk, uint32_t wmax, uint32_t pmax,
-                                uint32_t any_inner, unsigned long long* d_keys, cudaStream_t st) {
-  cudaError_t e = cudaSuccess;
-  if (b.ns) e = bfk::launch_lanetree(d_lt, d_first_block, b.ns, lt_blocks, b.nmax_small, d_keys, st);
-  if (e == cudaSuccess && b.nl) {
-    const uint32_t bps = (pmax + (bfk::kThreads / 32) - 1) / (bfk::kThreads / 32);
-#define CALL(NW) launch_batch_nw##NW(d_bk, b.nl, b.nmax_large, any_inner, bps, d_keys + b.ns, st)
-    BF_DISPATCH(bfk::bucket_for(wmax), CALL)
-#undef CALL
-  }
-  return e;
 }
 
 inline size_t align256(size_t x) { return (x + 255) / 256 * 256; }
@@ -924,14 +851,13 @@ static int search_batch_impl(const bf_scenario_desc* descs, uint32_t count, bf_r
 
 namespace {
 
-// Regions of the array: lane-tree records, their first blocks, batch-kernel
-// records, keys; each sized for BF_NOALLOC_MAX_SCENARIOS scenarios.
+// Regions of the array: lane-tree records, the first-block arrays of the
+// groups' launches (one entry more per group), keys; each sized for
+// BF_NOALLOC_MAX_SCENARIOS scenarios.
 constexpr size_t kNoAllocFirstBlockOffset =
     (sizeof(bfk::LaneTreeRecord) * BF_NOALLOC_MAX_SCENARIOS + 255) / 256 * 256;
-constexpr size_t kNoAllocRecordOffset =
-    kNoAllocFirstBlockOffset + (sizeof(uint32_t) * (BF_NOALLOC_MAX_SCENARIOS + 1) + 255) / 256 * 256;
 constexpr size_t kNoAllocKeyOffset =
-    kNoAllocRecordOffset + (sizeof(bfk::BatchRecord) * BF_NOALLOC_MAX_SCENARIOS + 255) / 256 * 256;
+    kNoAllocFirstBlockOffset + (sizeof(uint32_t) * (BF_NOALLOC_MAX_SCENARIOS + kBatchGroups) + 255) / 256 * 256;
 constexpr size_t kNoAllocBytes = kNoAllocKeyOffset + sizeof(unsigned long long) * BF_NOALLOC_MAX_SCENARIOS;
 
 }  // namespace
@@ -1029,54 +955,50 @@ int search_batch_noalloc_locked(NoAllocDevice& dv, const bf_scenario_desc* descs
   }
   auto* d_lt = reinterpret_cast<bfk::LaneTreeRecord*>(dv.base);
   auto* d_fb = reinterpret_cast<uint32_t*>(dv.base + kNoAllocFirstBlockOffset);
-  auto* d_bk = reinterpret_cast<bfk::BatchRecord*>(dv.base + kNoAllocRecordOffset);
   auto* d_keys = reinterpret_cast<unsigned long long*>(dv.base + kNoAllocKeyOffset);
-  uint32_t small[BF_NOALLOC_MAX_SCENARIOS], large[BF_NOALLOC_MAX_SCENARIOS];
-  uint32_t first_block[BF_NOALLOC_MAX_SCENARIOS + 1];
-  const BatchSplit b = split_batch(descs, count, small, large);
+  // Positions ordered by group (as bf_search_batch): key j and record j
+  // belong to position ids[j]; group g's first-block array has gcount[g] + 1
+  // entries at fb[gbeg[g] + g].
+  uint32_t ids[BF_NOALLOC_MAX_SCENARIOS], fb[BF_NOALLOC_MAX_SCENARIOS + kBatchGroups];
+  uint32_t gcount[kBatchGroups] = {}, gnmax[kBatchGroups] = {};
+  for (uint32_t i = 0; i < count; ++i) ++gcount[batch_group(descs[i].n)];
+  const uint32_t gbeg[kBatchGroups + 1] = {0u, gcount[0], gcount[0] + gcount[1], count};
+  uint32_t fill[kBatchGroups] = {gbeg[0], gbeg[1], gbeg[2]};
+  for (uint32_t i = 0; i < count; ++i) {
+    const uint32_t g = batch_group(descs[i].n);
+    ids[fill[g]++] = i;
+    gnmax[g] = descs[i].n > gnmax[g] ? descs[i].n : gnmax[g];
+  }
 
   // Pack the records a few at a time through stack buffers (a copy from
   // pageable memory has left the buffer when cudaMemcpyAsync returns).
   constexpr uint32_t kChunk = 8;
   cudaError_t e = cudaSuccess;
-  first_block[0] = 0u;
   {
     bfk::LaneTreeRecord chunk[kChunk];
-    for (uint32_t j0 = 0; j0 < b.ns && e == cudaSuccess; j0 += kChunk) {
-      const uint32_t nrec = (b.ns - j0 < kChunk) ? (b.ns - j0) : kChunk;
-      for (uint32_t j = 0; j < nrec; ++j) {
-        lanetree_record(descs + small[j0 + j], chunk + j);
-        first_block[j0 + j + 1] = first_block[j0 + j] + chunk[j].nblocks;
+    for (uint32_t g = 0; g < kBatchGroups; ++g) {
+      uint32_t* f = fb + gbeg[g] + g;
+      f[0] = 0u;
+      for (uint32_t j0 = gbeg[g]; j0 < gbeg[g + 1] && e == cudaSuccess; j0 += kChunk) {
+        const uint32_t nrec = (gbeg[g + 1] - j0 < kChunk) ? (gbeg[g + 1] - j0) : kChunk;
+        for (uint32_t j = 0; j < nrec; ++j) {
+          lanetree_record(descs + ids[j0 + j], chunk + j);
+          f[j0 + j - gbeg[g] + 1] = f[j0 + j - gbeg[g]] + chunk[j].nblocks;
+        }
+        e = cudaMemcpyAsync(d_lt + j0, chunk, sizeof(bfk::LaneTreeRecord) * nrec, cudaMemcpyHostToDevice, st);
       }
-      e = cudaMemcpyAsync(d_lt + j0, chunk, sizeof(bfk::LaneTreeRecord) * nrec, cudaMemcpyHostToDevice, st);
     }
   }
-  if (e == cudaSuccess && b.ns)
-    e = cudaMemcpyAsync(d_fb, first_block, sizeof(uint32_t) * (b.ns + 1), cudaMemcpyHostToDevice, st);
-  uint32_t wmax = 0, pmax = 0, any_inner = 0;
-  {
-    bfk::BatchRecord chunk[kChunk];
-    for (uint32_t j0 = 0; j0 < b.nl && e == cudaSuccess; j0 += kChunk) {
-      const uint32_t nrec = (b.nl - j0 < kChunk) ? (b.nl - j0) : kChunk;
-      for (uint32_t j = 0; j < nrec; ++j) {
-        bfk::BatchRecord& r = chunk[j];
-        std::memset(&r, 0, sizeof r);
-        bfk::Plan plan;
-        batch_split(descs + large[j0 + j], &r.full, &plan, &r.window);
-        r.plan = batch_plan(plan, descs[large[j0 + j]].n, bfk::kThreads / 32);
-        r.mid_lanes = plan.W0 == 0u ? 1u : 0u;
-        if (r.window.n > wmax) wmax = r.window.n;
-        const uint32_t tasks = r.plan.groups * r.plan.m_parts;
-        if (tasks > pmax) pmax = tasks;
-        any_inner |= r.plan.I;
-      }
-      e = cudaMemcpyAsync(d_bk + j0, chunk, sizeof(bfk::BatchRecord) * nrec, cudaMemcpyHostToDevice, st);
-    }
-  }
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(d_fb, fb, sizeof(uint32_t) * (count + kBatchGroups), cudaMemcpyHostToDevice, st);
   // The keys keep the previous call's values: reset them to "nothing found".
   if (e == cudaSuccess) e = cudaMemsetAsync(d_keys, 0xFF, sizeof(unsigned long long) * count, st);
-  if (e == cudaSuccess)
-    e = launch_batch_groups(b, d_lt, d_fb, first_block[b.ns], d_bk, wmax, pmax, any_inner, d_keys, st);
+  for (uint32_t g = 0; g < kBatchGroups && e == cudaSuccess; ++g) {
+    const uint32_t c = gbeg[g + 1] - gbeg[g];
+    if (c == 0) continue;
+    const uint32_t* f = fb + gbeg[g] + g;
+    e = bfk::launch_lanetree(d_lt + gbeg[g], d_fb + gbeg[g] + g, c, f[c], gnmax[g], d_keys + gbeg[g], st);
+  }
   if (e != cudaSuccess) return cuda_fail(e, who);
   rc = wait_stream(st, who);
   if (rc == BF_ETIMEOUT) {
@@ -1092,7 +1014,7 @@ int search_batch_noalloc_locked(NoAllocDevice& dv, const bf_scenario_desc* descs
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);
     if (e != cudaSuccess) return cuda_fail(e, who);
     for (uint32_t j = 0; j < nk; ++j) {
-      const uint32_t k = i0 + j, i = k < b.ns ? small[k] : large[k - b.ns];
+      const uint32_t i = ids[i0 + j];
       fill_result(keys[j], descs[i].n, 0, out + i);
     }
   }

@@ -190,72 +190,6 @@ __device__ __forceinline__ void warp_task(const TBF& tb, const SmemTables& sd, c
                       stride, sink);
 }
 
-// The other assignment of lanes, for DAGs where the prefix settles nothing
-// (the window is the whole DAG: most tools start at once, so lanes holding
-// different early modes diverge from the first event): the warp shares
-// prefix p (each lane simulates it, identically) and lane l takes mid
-// combinations l, l + 32, ...; the lanes then differ only in later tools.
-// Measured on 4096 random layered 10-tool DAGs: 8 % faster than lanes owning
-// prefixes.
-template <int NP, int NW, typename TBF, typename TBW, typename Sink>
-__device__ __forceinline__ void mid_lane_task(const TBF& tb, const SmemTables& sd, const uint32_t* rt, const TBW& tw,
-                                              const SmemTables& sdw, const uint32_t* rtw, const Plan& plan,
-                                              const uint32_t* mpart, uint32_t p, uint32_t* slotA, uint32_t* slotB,
-                                              uint32_t stride, Sink& sink) {
-  Digits dgp{0u, 0u};
-  uint32_t T_check = 0u;
-  const bool ok = prefix_checkpoint<NP, NW>(tb, sd, rt, plan, p, &dgp, &T_check, slotA, stride);
-  const uint32_t shm = plan.P - plan.W0;
-  const uint32_t shi = shm + plan.M;
-  const uint32_t inner_mask = tw.all_mask & ~((1u << shi) - 1u);
-  const TaskIndex<true> ix{index_part(plan, dgp, 0u, plan.P), mpart, 0u};
-  const Digits dgw{dgp.now >> plan.W0, dgp.que >> plan.W0};
-  const uint32_t lane = threadIdx.x & 31u;
-  for (uint32_t m0 = 0; m0 < plan.pow3M; m0 += 32u) {
-    const uint32_t m = m0 + lane;
-    if (m >= plan.pow3M) continue;
-    const Digits dm = decode(m, plan.M);
-    const uint64_t base = ix.base(plan, m);
-    if (!ok) {
-      for (uint32_t i = 0; i < plan.pow3I; ++i) sink((uint32_t)(base + ix.inner(plan, i)), kInfeasible);
-      continue;
-    }
-    const Digits dmid{dgw.now | (dm.now << shm), dgw.que | (dm.que << shm)};
-    State<NW> w;
-    uint32_t r = kRunInfeasible;
-    if ((dmid.que & tw.big_mask) == 0u) {
-      load_lane(slotA, stride, w);
-      r = run<NW>(w, tw, sdw, rtw, dmid, inner_mask);
-    }
-    if (plan.I == 0u) {
-      sink((uint32_t)base, r == kRunFinished ? w.T : kInfeasible);
-      continue;
-    }
-    if (r != (plan.last_apart ? kRunFinished : kRunStopped)) {
-      for (uint32_t i = 0; i < plan.pow3I; ++i) sink((uint32_t)(base + ix.inner(plan, i)), kInfeasible);
-      continue;
-    }
-    if (plan.last_apart || (plan.I == 1u && (w.done | inner_mask) == 0xFFFFFFFFu)) {  // the last tool runs alone
-      for (uint32_t i = 0; i < plan.pow3I; ++i) {
-        const uint32_t d = plan.alone[i];
-        sink((uint32_t)(base + ix.last(plan, i)), d == kInfeasible ? kInfeasible : w.T + d);
-      }
-      continue;
-    }
-    save_lane(w, slotB, stride);
-    for (uint32_t i = 0; i < plan.pow3I; ++i) {
-      const Digits di = decode(i, plan.I);
-      const Digits dg{dmid.now | (di.now << shi), dmid.que | (di.que << shi)};
-      uint32_t ms = kInfeasible;
-      if ((dg.que & tw.big_mask) == 0u) {
-        if (i != 0u) load_lane(slotB, stride, w);
-        ms = run<NW>(w, tw, sdw, rtw, dg, 0u) == kRunFinished ? w.T : kInfeasible;
-      }
-      sink((uint32_t)(base + ix.inner(plan, i)), ms);
-    }
-  }
-}
-
 struct MinKeySink {
   unsigned long long best = ~0ull;
   __device__ __forceinline__ void operator()(uint32_t idx, uint32_t ms) {

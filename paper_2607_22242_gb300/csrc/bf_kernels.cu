@@ -40,9 +40,6 @@
 #define BF_MIN_BLOCKS 2
 #endif
 #endif
-#ifndef BF_MIN_BLOCKS_BATCH
-#define BF_MIN_BLOCKS_BATCH 2
-#endif
 
 namespace bfk {
 namespace {
@@ -160,55 +157,6 @@ __global__ void __launch_bounds__(kSearchThreads, kSearchMinBlocks) search_kerne
       __threadfence_system();
     }
   }
-}
-
-// One record per scenario of a batch: full tables, window tables and plan.
-template <int NP>
-__global__ void __launch_bounds__(kThreads, BF_MIN_BLOCKS_BATCH) batch_kernel(const BatchRecord* __restrict__ recs,
-                                                                              uint32_t blocks_per_scenario,
-                                                                              unsigned long long* keys) {
-  extern __shared__ uint32_t dyn_smem[];  // mid-part table (3^6 entries at most), then the lane states
-  uint32_t* const mpart = dyn_smem;
-  uint32_t* const lane_state = dyn_smem + kMaxMidPartWords;
-  __shared__ BatchRecord rec;
-  __shared__ SmemTables sd, sdw;
-  __shared__ uint32_t rt[ReadyTable<NP>::size], rtw[ReadyTable<BF_NW>::size];
-  const uint32_t sc = blockIdx.x / blocks_per_scenario;
-  const uint32_t b = blockIdx.x - sc * blocks_per_scenario;
-  {
-    const uint32_t* src = reinterpret_cast<const uint32_t*>(recs + sc);
-    uint32_t* dst = reinterpret_cast<uint32_t*>(&rec);
-    for (uint32_t w = threadIdx.x; w < sizeof(BatchRecord) / 4; w += blockDim.x) dst[w] = src[w];
-  }
-  __syncthreads();
-  load_smem_tables(rec.full, sd);
-  load_smem_tables(rec.window, sdw);
-  fill_ready_table<NP>(rec.full, rt);
-  fill_ready_table<BF_NW>(rec.window, rtw);
-  fill_mid_parts(rec.plan, mpart);
-  __syncthreads();
-  const uint32_t warp = b * kWarps + (threadIdx.x >> 5);
-  MinKeySink sink;
-  if (rec.mid_lanes) {  // block-uniform
-    // mid_lanes <=> W0 == 0: the window tables are the full tables, tool for
-    // tool.  With equal slot counts the run reads one copy, so the compiler
-    // keeps one set of table values in registers instead of two (fewer
-    // spills at 2 blocks/SM; 2.5 % faster on 4096 layered 10-tool DAGs).
-    for (uint32_t p = warp; p < rec.plan.pow3P; p += blocks_per_scenario * kWarps) {
-      if constexpr (NP == BF_NW)
-        mid_lane_task<NP, BF_NW>(rec.full, sd, rt, rec.full, sd, rt, rec.plan, mpart, p, lane_state + threadIdx.x,
-                                 lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
-      else
-        mid_lane_task<NP, BF_NW>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, mpart, p,
-                                 lane_state + threadIdx.x,
-                                 lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
-    }
-  } else if (warp < rec.plan.groups * rec.plan.m_parts) {
-    warp_task<NP, BF_NW, true>(rec.full, sd, rt, rec.window, sdw, rtw, rec.plan, mpart, warp / rec.plan.m_parts,
-                         warp % rec.plan.m_parts, lane_state + threadIdx.x,
-                         lane_state + kLaneWords * kThreads + threadIdx.x, kThreads, sink);
-  }
-  block_min_to(sink.best, keys + sc);
 }
 
 // Index-list evaluation: one mapping per thread (grid-stride), simulated from
@@ -371,14 +319,6 @@ cudaError_t BF_PASTE(launch_list_nw, BF_NW)(const Tables& tb, uint64_t total, co
                                             uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st) {
   list_kernel<BF_NW><<<grid, kThreads, 0, st>>>(tb, total, idx, count, ms, fe);
   return cudaGetLastError();
-}
-
-cudaError_t BF_PASTE(launch_batch_nw, BF_NW)(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,
-                                             uint32_t any_inner, uint32_t blocks_per_scenario,
-                                             unsigned long long* keys, cudaStream_t st) {
-  const unsigned blocks = (unsigned)((uint64_t)count * blocks_per_scenario);
-  BF_LAUNCH(batch_kernel, nmax <= (uint32_t)BF_NW, any_inner, kMaxMidPartWords, blocks, d_recs, blocks_per_scenario,
-            keys);
 }
 
 }  // namespace bfk

@@ -39,24 +39,11 @@ struct SearchSync {
   uint32_t next_root;
 };
 
-// One scenario of a batched search: its tables, its window tables and plan,
-// and how its warps assign lanes (0: a prefix per lane, warp_task; 1: a mid
-// combination per lane, mid_lane_task).
-struct BatchRecord {
-  Tables full;
-  Tables window;
-  Plan plan;
-  uint32_t mid_lanes;
-};
-
 #define BF_DECLARE_BUCKET(NW)                                                                       \
   cudaError_t launch_eval_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan, uint32_t* ms, \
                                  uint8_t* fe, cudaStream_t st);                                     \
   cudaError_t launch_search_nw##NW(const Tables& tb, const Tables& tw, const Plan& plan,             \
                                    SearchSync* sync, unsigned long long* host_key, cudaStream_t st);  \
-  cudaError_t launch_batch_nw##NW(const BatchRecord* d_recs, uint32_t count, uint32_t nmax,           \
-                                  uint32_t any_inner, uint32_t blocks_per_scenario,                  \
-                                  unsigned long long* keys, cudaStream_t st);                        \
   cudaError_t launch_list_nw##NW(const Tables& tb, uint64_t total, const uint64_t* idx, uint64_t count, \
                                  uint32_t* ms, uint8_t* fe, int grid, cudaStream_t st);             \
   cudaError_t launch_prefix_filter_nw##NW(const Tables& tb, const Plan& plan, const uint32_t* cand_ms,   \

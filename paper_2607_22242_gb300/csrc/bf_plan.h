@@ -58,9 +58,8 @@ inline void build_tables(const bf_scenario_desc* d, bfk::TablesT<CAP>* t) {
   t->fmagic[0] = 1ull << 54;
 }
 
-// Number of mid tools M when a warp's lanes take mid combinations under one
-// prefix (the batch kernel's whole-DAG windows): large enough to keep 32
-// lanes busy, small enough to leave many prefixes (warps).
+// Number of mid tools M of the pruned search's split (bf_search_pruned):
+// more mid tools than the search's 4 leave fewer, shorter prefixes to filter.
 inline uint32_t mid_tools(uint32_t n) {
   if (n >= 13) return 6;   // 729 combinations: 23 rounds of 32 lanes, 1% idle
   if (n >= 9) return 5;    // 243 combinations
@@ -318,18 +317,6 @@ inline void split_and_window(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w
   }
 }
 
-// Plan of one scenario of a batch.  A window that is the whole DAG (W0 = 0)
-// runs with lanes taking mid combinations under a shared prefix, which wants
-// mid_tools(n) mid tools to fill the lanes (4096 layered 10-tool DAGs: M = 5
-// 38.2 ms, M = 4 41.1 ms); other scenarios take the search plan.
-inline void split_and_window_batch(const bfk::Tables& t, bfk::Plan* pl, bfk::Tables* w) {
-  uint32_t anc[BF_MAX_TOOLS] = {}, R[BF_MAX_TOOLS + 1] = {};
-  ancestors(t, anc);
-  retired_estimate(t, R);
-  plan_for(t, anc, R, mid_tools(t.n), false, pl, w);
-  if (pl->W0 != 0u) split_and_window(t, pl, w);
-}
-
 // Whether a renumbered split (tables rt, plan rp, window rw) should replace
 // the scenario-numbered one (t, p, w): its prefix snapshot settles more tools
 // (estimated), its window is narrower, or it has a deeper inner level.  The
@@ -434,11 +421,11 @@ inline bfk::Plan make_plan(const bfk::Plan& base, uint64_t first, uint64_t count
 // of the GPU's resident warps, so that uneven tasks even out.
 constexpr uint64_t kSearchTasks = 32768;
 
-// Whole-space searches (bf_search_best and bf_search_range over the whole
-// space, bf_search_pruned, the batch) run on the tables renumbered with the
-// sources first when that gives a better split (renumbering_helps); otherwise
-// on t0 with its own split p0 and window w0.  split: split_and_window, or
-// split_and_window_batch for the scenarios of a batch.
+// Whole-space searches on the search kernel (bf_search_best and
+// bf_search_range over the whole space, bf_search_pruned) run on the tables
+// renumbered with the sources first when that gives a better split
+// (renumbering_helps); otherwise on t0 with its own split p0 and window w0.
+// split: split_and_window, or the pruned search's split.
 template <typename Split>
 inline void whole_space_tables(const bfk::Tables& t0, const bfk::Plan& p0, const bfk::Tables& w0, Split split,
                                bfk::Tables* tb, bfk::Plan* plan, bfk::Tables* tw) {
@@ -456,24 +443,6 @@ inline void whole_space_tables(const bfk::Tables& t0, const bfk::Plan& p0, const
   *tb = t0;
   *plan = p0;
   *tw = w0;
-}
-
-// Tables, split and window of one scenario of a batch (a whole-space search).
-inline void batch_split(const bf_scenario_desc* d, bfk::Tables* tb, bfk::Plan* plan, bfk::Tables* tw) {
-  bfk::Tables t0, w0;
-  bfk::Plan p0;
-  build_tables(d, &t0);
-  split_and_window_batch(t0, &p0, &w0);
-  whole_space_tables(t0, p0, w0, split_and_window_batch, tb, plan, tw);
-}
-
-// Plan of one scenario of a batch, which one block of `block_warps` warps
-// searches: a scenario with fewer prefix groups than warps splits its mid
-// combinations so that as many warps as possible share it.
-inline bfk::Plan batch_plan(const bfk::Plan& base, uint32_t n, uint32_t block_warps) {
-  const uint32_t groups = (base.pow3P + 31u) / 32u;
-  const uint32_t fill = groups < block_warps ? block_warps / groups : 1u;
-  return make_plan(base, 0, pow3(n), (uint64_t)fill * groups);
 }
 
 // Mappings a block of the lane-tree batch kernel aims to search (a 10-tool

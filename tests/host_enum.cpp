@@ -29,7 +29,6 @@ using namespace bfk;
 
 namespace {
 
-constexpr uint32_t kBlockWarps = 8;  // warps of the batch kernel's blocks (kThreads / 32 in the library)
 
 struct StoreAll {
   uint32_t first;
@@ -45,7 +44,7 @@ struct Lanes {
 };
 
 template <int NP, int NW, bool RL>
-void run_tasks(const Tables& tb, const Tables& tw, const Plan& plan, bool mid_lanes, uint32_t* out) {
+void run_tasks(const Tables& tb, const Tables& tw, const Plan& plan, uint32_t* out) {
   threadIdx.x = 0;
   SmemTables sd, sdw;
   load_smem_tables(tb, sd);
@@ -56,17 +55,6 @@ void run_tasks(const Tables& tb, const Tables& tw, const Plan& plan, bool mid_la
   fill_mid_parts(plan, mpart.data());
   const int lw = LaneWords<NW>::value;
   StoreAll sink{plan.first, out};
-  if (mid_lanes) {
-    for (uint32_t p = 0; p < plan.pow3P; ++p) {
-      Lanes lanes(lw);
-      for (unsigned lane = 0; lane < 32; ++lane) {
-        threadIdx.x = lane;
-        mid_lane_task<NP, NW>(tb, sd, rt.data(), tw, sdw, rtw.data(), plan, mpart.data(), p, lanes.words.data() + lane,
-                              lanes.words.data() + lw * 32 + lane, 32, sink);
-      }
-    }
-    return;
-  }
   for (uint32_t g = 0; g < plan.groups; ++g)
     for (uint32_t part = 0; part < plan.m_parts; ++part) {
       Lanes lanes(lw);
@@ -79,14 +67,14 @@ void run_tasks(const Tables& tb, const Tables& tw, const Plan& plan, bool mid_la
 }
 
 template <int NW>
-void run_width(const Tables& tb, const Tables& tw, const Plan& plan, bool mid_lanes, uint32_t* out) {
+void run_width(const Tables& tb, const Tables& tw, const Plan& plan, uint32_t* out) {
   const bool rl = plan.relabeled != 0u;
   if (tb.n <= (uint32_t)NW) {
-    if (rl) run_tasks<NW, NW, true>(tb, tw, plan, mid_lanes, out);
-    else run_tasks<NW, NW, false>(tb, tw, plan, mid_lanes, out);
+    if (rl) run_tasks<NW, NW, true>(tb, tw, plan, out);
+    else run_tasks<NW, NW, false>(tb, tw, plan, out);
   } else {
-    if (rl) run_tasks<kMaxTools, NW, true>(tb, tw, plan, mid_lanes, out);
-    else run_tasks<kMaxTools, NW, false>(tb, tw, plan, mid_lanes, out);
+    if (rl) run_tasks<kMaxTools, NW, true>(tb, tw, plan, out);
+    else run_tasks<kMaxTools, NW, false>(tb, tw, plan, out);
   }
 }
 
@@ -95,18 +83,15 @@ void run_width(const Tables& tb, const Tables& tw, const Plan& plan, bool mid_la
 // mode 0: the searches' plan in the scenario's numbering, over [first, first+count).
 // mode 1: the whole space, renumbered with the sources first (when that
 //         changes the order), as the whole-space searches may run it.
-// mode 2: the whole space with a batch record's plan (renumbered when that
-//         improves the split; lanes take mid combinations for whole-DAG windows).
 // Slots beyond a window count as done, so a width of 4, 7, 10, 14 or 20 slots
 // serves every window up to it (the library compiles every width).
-// info[0..5] = P, M, I, W0, window tools, flags (1 renumbered, 2 last tool apart, 4 mid lanes).
+// info[0..5] = P, M, I, W0, window tools, flags (1 renumbered, 2 last tool apart).
 extern "C" int host_eval(const bf_scenario_desc* d, uint64_t first, uint64_t count, uint32_t mode, uint32_t* out,
                          uint32_t* info) {
   Tables t0, tb, tw;
   Plan base;
   host::build_tables(d, &t0);
   const uint64_t total = host::pow3(d->n);
-  bool mid_lanes = false;
   Plan plan;
   if (mode == 0) {
     tb = t0;
@@ -114,28 +99,23 @@ extern "C" int host_eval(const bf_scenario_desc* d, uint64_t first, uint64_t cou
     plan = host::make_plan(base, first, count, host::kSearchTasks);
   } else {
     if (first != 0 || count != total) return -1;
-    if (mode == 1) {
-      host::relabel_sources_first(t0, &tb);
-      host::split_and_window(tb, &base, &tw);
-      plan = host::make_plan(base, first, count, host::kSearchTasks);
-    } else {
-      host::batch_split(d, &tb, &base, &tw);
-      plan = host::batch_plan(base, d->n, kBlockWarps);
-      mid_lanes = base.W0 == 0u;
-    }
+    if (mode != 1) return -1;
+    host::relabel_sources_first(t0, &tb);
+    host::split_and_window(tb, &base, &tw);
+    plan = host::make_plan(base, first, count, host::kSearchTasks);
   }
   info[0] = plan.P;
   info[1] = plan.M;
   info[2] = plan.I;
   info[3] = plan.W0;
   info[4] = tw.n;
-  info[5] = (tb.relabeled ? 1u : 0u) | (plan.last_apart ? 2u : 0u) | (mid_lanes ? 4u : 0u);
+  info[5] = (tb.relabeled ? 1u : 0u) | (plan.last_apart ? 2u : 0u);
   for (uint64_t j = 0; j < count; ++j) out[j] = 0xDEADBEEFu;
-  if (tw.n <= 4) run_width<4>(tb, tw, plan, mid_lanes, out);
-  else if (tw.n <= 7) run_width<7>(tb, tw, plan, mid_lanes, out);
-  else if (tw.n <= 10) run_width<10>(tb, tw, plan, mid_lanes, out);
-  else if (tw.n <= 14) run_width<14>(tb, tw, plan, mid_lanes, out);
-  else run_width<20>(tb, tw, plan, mid_lanes, out);
+  if (tw.n <= 4) run_width<4>(tb, tw, plan, out);
+  else if (tw.n <= 7) run_width<7>(tb, tw, plan, out);
+  else if (tw.n <= 10) run_width<10>(tb, tw, plan, out);
+  else if (tw.n <= 14) run_width<14>(tb, tw, plan, out);
+  else run_width<20>(tb, tw, plan, out);
   return 0;
 }
 

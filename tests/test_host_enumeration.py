@@ -3,10 +3,10 @@
 tests/host_enum.cpp compiles bf_plan.h, bf_enum.cuh and bf_sim.cuh -- the code the kernels run --
 with g++ and executes each plan's warp tasks lane by lane.  Every mapping's makespan, stored at its
 canonical index, must equal the oracle's: in the scenario's numbering over whole spaces and index
-ranges, over whole spaces renumbered with the sources first, and with a batch record's plan (lanes
-taking mid combinations).  This checks splits, windows, the closed-form last tool, the
-renumbering and the canonical index arithmetic on every CPU test run; the GPU tests check the
-same on the hardware.
+ranges, and over whole spaces renumbered with the sources first.  This checks splits, windows, the
+closed-form last tool, the renumbering and the canonical index arithmetic on every CPU test run;
+the GPU tests check the same on the hardware.  The lane-tree kernels' code (bf_lanetree.cuh) is
+run the same way, lane by lane, by the lanetree tests below.
 """
 import ctypes
 import os
@@ -70,8 +70,8 @@ def _same(host, scn, first, count, mode):
 
 def test_random_dags_every_mode(host):
     """Random DAGs of 1-9 tools with small integer times (ties, blocked queues, infeasible
-    starts), some with late sources or a last tool that waits for all others: every mapping in all
-    three modes, and random index ranges in the scenario's numbering."""
+    starts), some with late sources or a last tool that waits for all others: every mapping in both
+    modes, and random index ranges in the scenario's numbering."""
     rng = np.random.default_rng(90)
     flags = 0
     for t in range(240):
@@ -86,12 +86,12 @@ def test_random_dags_every_mode(host):
         scn = S.Scenario(n, pred, base.cpu_us, base.gpu_us, base.xfer_us, base.load_us, base.vram_mib,
                          base.vram_budget_mib, base.slowdown_q10)
         total = 3 ** n
-        for mode in (0, 1, 2):
+        for mode in (0, 1):
             flags |= int(_same(host, scn, 0, total, mode)[5])
         if total > 3:
             a = int(rng.integers(0, total - 2))
             _same(host, scn, a, int(rng.integers(1, total - a + 1)), 0)
-    assert flags == 7, flags  # renumbered, last tool apart and mid lanes all exercised
+    assert flags == 3, flags  # renumbered and last tool apart both exercised
 
 
 def test_standard_workloads_host(host):
@@ -99,7 +99,7 @@ def test_standard_workloads_host(host):
     ranges of the 16-tool one."""
     for cfg in (0, 1):
         scn = S.config(cfg)
-        for mode in (0, 1, 2):
+        for mode in (0, 1):
             _same(host, scn, 0, 3 ** scn.n, mode)
     scn = S.config2()
     total = 3 ** scn.n
@@ -134,11 +134,11 @@ def test_branch_and_bound_host(host):
 
 def test_tie_order_scenarios_host(host):
     """Queue-heavy tiny DAGs with late sources, some with tied optima whose lowest member differs
-    between the canonical and the renumbered order: every mapping in all three modes at its
+    between the canonical and the renumbered order: every mapping in both modes at its
     canonical index, and bf_search_pruned's optimum (ties to the lowest canonical index) from the
     optimum's makespan and from no incumbent."""
     for t, scn in enumerate(tie_order_scenarios()):
-        for mode in (0, 1, 2):
+        for mode in (0, 1):
             _same(host, scn, 0, 3 ** scn.n, mode)
         want = oracle.search(scn)
         for bound in (want[1], 0xFFFFFFFF):
