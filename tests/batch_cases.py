@@ -1,8 +1,8 @@
 """Seeded batches shared by the GPU tests (input generation only, no arithmetic of the method).
 
-mixed_group_batch(): scenarios of 1-12 tools (searched by the lane-tree kernel) interleaved with
-scenarios of 13 and 14 tools (searched by the batch kernel), so that a batch call's results must come
-back to their positions from both kernel groups.
+mixed_group_batch(): scenarios of 1-12 tools interleaved with scenarios of 13 and 14 tools, which a
+batch call searches in two groups (the lane-tree batch kernel's two- and three-chunk forms), so that
+its results must come back to their positions from both groups.
 """
 import numpy as np
 

@@ -529,8 +529,8 @@ def test_wait_timeout_is_reported():
 def test_pipelined_batch_with_both_groups(golden):
     """A batch large enough to be pipelined (its first eighth of lane-tree scenarios launched while the
     rest are built, the rest on a second stream), with 30 random scenarios of 1-14 tools interleaved
-    (those of 13 and 14 tools run the batch kernel, also on the second stream): every result at its
-    position against the oracle."""
+    (those of 13 and 14 tools run the lane-tree batch kernel's three-chunk form, also on the second
+    stream): every result at its position against the oracle."""
     small = S.config4(1200)
     extra = mixed_group_batch(seed=99, count=30)
     scns, origin = [], []  # origin: index into small, or -1 for an interleaved scenario
@@ -693,11 +693,12 @@ def test_pruned_search_batch_scenarios(golden):
         assert (r.index, r.makespan_us) == (want_i[k], want_m[k]), k
 
 
-# --------------------------------------------------------------------------- the batch's two kernel groups
+# --------------------------------------------------------------------------- the batch's two groups
 
-def test_batch_two_kernel_groups():
-    """Scenarios of up to 12 tools (lane-tree kernel) interleaved with scenarios of 13 and 14 tools
-    (batch kernel) in one call: every result at its position, equal to the oracle's."""
+def test_batch_two_groups():
+    """Scenarios of up to 12 tools interleaved with scenarios of 13 and 14 tools (the lane-tree batch
+    kernel's two- and three-chunk groups) in one call: every result at its position, equal to the
+    oracle's."""
     scns = mixed_group_batch()
     assert {s.n > 12 for s in scns} == {True, False}
     o_i, o_m = oracle.search_batch(scns, THREADS)

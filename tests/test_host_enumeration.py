@@ -242,7 +242,7 @@ def test_lanetree_wide_queue_form(host):
 
 
 def test_lanetree_batch_records_of_larger_scenarios(host):
-    """The batch's records of scenarios of 13 and 14 tools (the batch kernel's three-chunk group; at
+    """The batch's records of scenarios of 13 and 14 tools (the lane-tree batch kernel's three-chunk group; at
     most 1,024 blocks per scenario) and, in the wide form, of 9-12 tools: every mapping against the
     oracle."""
     rng = np.random.default_rng(95)

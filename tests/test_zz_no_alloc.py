@@ -105,9 +105,10 @@ def test_noalloc_rejects_oversized_batch():
     assert str(bf.NOALLOC_MAX_SCENARIOS) in ei.value.message
 
 
-def test_noalloc_two_kernel_groups():
-    """Scenarios of up to 12 tools and of 13 and 14 tools interleaved in one call: both regions of the
-    fixed scratch in use, every result at its position, equal to the oracle's."""
+def test_noalloc_two_groups():
+    """Scenarios of up to 12 tools and of 13 and 14 tools interleaved in one call: two groups of the
+    lane-tree batch kernel over the fixed scratch, every result at its position, equal to the
+    oracle's."""
     from batch_cases import mixed_group_batch
     scns = mixed_group_batch()
     o_i, o_m = oracle.search_batch(scns, oracle.default_threads())
