@@ -114,3 +114,23 @@ def test_noalloc_two_groups():
     o_i, o_m = oracle.search_batch(scns, oracle.default_threads())
     got = bf.search_batch_noalloc(scns)
     assert [(r.index, r.makespan_us) for r in got] == list(zip(o_i.tolist(), o_m.tolist()))
+
+
+def test_noalloc_all_three_groups():
+    """A batch with scenarios of every lane-tree group -- up to 12 tools, 13 to 16, and 17 to 20 (the
+    wide form) -- interleaved in one call: every result at its position, equal to bf_search_batch's
+    (whose groups are checked against the oracle and against each scenario's full search)."""
+    def layered(seed, sizes, budget):
+        rng = np.random.default_rng(seed)
+        n = sum(sizes)
+        c, g, x, m = S._ordinary(rng, n, 2048, 16384)
+        pred = S._layered_edges(rng, sizes, 0.4)
+        return S.Scenario(n, pred, c, g, x, [S._load_from_vram(v) for v in m], m, budget,
+                          S.slowdown_linear(kmax=n))
+    scns = list(S.config4(6))
+    scns.insert(2, layered(81, [4, 4, 3, 3, 3], 32768))   # 17 tools
+    scns.insert(4, layered(82, [4, 4, 3, 2], 24576))      # 13 tools
+    scns.append(layered(83, [4, 4, 4, 3, 3], 24576))      # 18 tools
+    assert {0, 1, 2} == {0 if s.n <= 12 else (1 if s.n <= 16 else 2) for s in scns}
+    got = bf.search_batch_noalloc(scns)
+    assert _same(got, bf.search_batch(scns))
